@@ -1,0 +1,40 @@
+"""Oracle: the acceptance pass of one block of positions, from given logits.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+For each row b of a block of P positions with c_b positions already committed
+(left-aligned, so the window starts at p = c_b):
+  * confidence of every uncommitted position from its logits (Eq. 2; top-1 id and
+    probability; top-2 probability for reporting),
+  * K over the window [p, p + L') with L' = min(L, P - p)          (Eq. compute_k),
+  * commit x[p:p+K] and refresh drafts at i >= p + L                (Eq. draft_update),
+using the same readings as ``oracle.decode``.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import decode, model
+
+
+def accept(logits: np.ndarray, committed: np.ndarray, x: np.ndarray,
+           cfg: decode.DecodeConfig, window: int):
+    """logits float [B][P][V] (bf16 values); committed int [B]; x int [B][P] (copied).
+
+    Returns (K [B], x_out [B][P], ids [B][P], p1 [B][P], p2 [B][P]); confidences of
+    committed positions are reported as 0 and id -1 (they are never read).
+    """
+    B, P, _ = logits.shape
+    x_out = np.array(x, dtype=np.int32, copy=True)
+    ids = np.full((B, P), -1, dtype=np.int32)
+    p1 = np.zeros((B, P))
+    p2 = np.zeros((B, P))
+    K = np.zeros(B, dtype=np.int32)
+    for b in range(B):
+        p = int(committed[b])
+        if p >= P:
+            continue
+        i_, c1, c2 = model.confidence(logits[b, p:].astype(np.float64))
+        ids[b, p:], p1[b, p:], p2[b, p:] = i_, c1, c2
+        K[b] = decode.commit_and_draft(x_out[b], p, ids[b], p1[b], cfg, window)
+    return K, x_out, ids, p1, p2

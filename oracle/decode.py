@@ -1,0 +1,128 @@
+"""Oracle: Dynamic Contiguous Verification with draft-guided decoding (Algorithm 1).
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+One iteration (Sec. 3.3, "Inference with Drafts") does, in order:
+  (i)   draft invalidation: x[p + i] <- MASK for i in [0, L)            (Eq. remasking)
+  (ii)  one forward pass giving the top-1 id and confidence everywhere   (Eq. 2)
+  (iii) K = sum_{i<L} prod_{j<=i} 1(c_{p+j} > tau_commit)               (Eq. compute_k)
+  (iv)  commit x[p:p+K] <- x_hat[p:p+K]; for every i >= p + L,
+        x_i <- x_hat_i if c_i > tau_draft (else keep)                    (Eq. draft_update)
+  then p <- p + K; loop while p is inside the sequence                   (Algorithm 1)
+
+Readings where the paper is silent or inconsistent (each one is also a test):
+  * indices are absolute: the loop runs while p < N + M and drafts cover
+    [p + L, N + M) (Algorithm 1 mixes a relative bound with an absolute p);
+  * both thresholds are strict ``>`` (Eq. compute_k, Eq. draft_update and Algorithm 1;
+    the prose of Sec. 3.2 says ``>=``);
+  * the window is clipped to the sequence end: L' = min(L, N + M - p);
+  * K = 0 would repeat the same deterministic state forever, so K is raised to
+    ``min_commit`` (default 1; 0 keeps the literal rule, bounded by ``max_steps``);
+  * p in the draft region is the window start of the current iteration, before the
+    advance (the order of Algorithm 1);
+  * drafts are refreshed at every future position, masked or already drafted;
+  * decisions compare the confidence and the threshold as float32 values, the
+    precision in which the CUDA kernel takes them.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+
+@dataclasses.dataclass
+class DecodeConfig:
+    tau_commit: float = 0.70      # Sec. 4.1 default
+    tau_draft: float = 0.98       # Sec. 4.1 default
+    max_window: int = 0           # L; 0 means gen_len // 2 (Sec. 4.1)
+    block_len: int = 32           # semi-AR block (Sec. 4.1); sets the prefix-cache refresh
+    gen_len: int = 0              # M
+    min_commit: int = 1
+    contiguous_drafts: bool = False  # App. E variant: drafts only as an unbroken chain
+    kv_cache: int = 0
+
+    def window(self) -> int:
+        return self.max_window if self.max_window > 0 else max(1, self.gen_len // 2)
+
+
+def exceeds(c, tau) -> np.ndarray:
+    """1(c > tau), taken in float32 (the precision of the CUDA decision)."""
+    return np.asarray(c, dtype=np.float32) > np.float32(tau)
+
+
+def window_length(c_window, tau_commit: float) -> int:
+    """Eq. compute_k: K = sum_i prod_{j<=i} 1(c_j > tau_commit) over the given window."""
+    ind = exceeds(c_window, tau_commit).astype(np.int64)
+    return int(np.cumprod(ind).sum())
+
+
+def remask(x: np.ndarray, p: int, window: int, mask_id: int) -> None:
+    """Eq. remasking, clipped to the sequence end (in place on one row)."""
+    x[p:min(p + window, x.shape[0])] = mask_id
+
+
+def commit_and_draft(x: np.ndarray, p: int, ids: np.ndarray, c: np.ndarray,
+                     cfg: DecodeConfig, window: int) -> int:
+    """Steps (iii)-(iv) on one row; ids/c are indexed by absolute position.  Returns K."""
+    T = x.shape[0]
+    w_eff = min(window, T - p)
+    K = window_length(c[p:p + w_eff], cfg.tau_commit)
+    K = min(max(K, cfg.min_commit), w_eff)
+    x[p:p + K] = ids[p:p + K]                                   # commit verified tokens
+    lo = p + window                                             # future region i >= p + L
+    if lo < T:
+        ok = exceeds(c[lo:T], cfg.tau_draft)
+        if cfg.contiguous_drafts:                               # App. E: unbroken chain only
+            ok = np.cumprod(ok.astype(np.int64)).astype(bool)
+        seg = x[lo:T]
+        seg[ok] = ids[lo:T][ok]
+    return K
+
+
+def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
+             max_steps: int = 1 << 30, record: bool = True) -> dict:
+    """Algorithm 1 for a batch of independent rows.
+
+    predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) for the generation positions.
+    Returns the final x [B][T], per-row steps, the K of every step, and (if ``record``)
+    the forward input of every step and the predictions it produced.
+    """
+    prompt = np.atleast_2d(np.asarray(prompt, dtype=np.int32))
+    B, N = prompt.shape
+    M = cfg.gen_len
+    T = N + M
+    L = cfg.window()
+    x = np.full((B, T), mask_id, dtype=np.int32)
+    x[:, :N] = prompt
+    p = np.full(B, N, dtype=np.int64)
+    steps = np.zeros(B, dtype=np.int64)
+    ks, inputs, preds = [], [], []
+    n_iter = 0
+    while (p < T).any() and n_iter < max_steps:
+        k_step = np.zeros(B, dtype=np.int64)
+        in_step = np.empty((B, T), dtype=np.int32)
+        pr = np.zeros((3, B, M))
+        for b in range(B):
+            if p[b] >= T:
+                in_step[b] = x[b]
+                continue
+            remask(x[b], int(p[b]), L, mask_id)                  # (i)
+            in_step[b] = x[b]
+            ids, p1, p2 = predict_fn(x[b].copy())                # (ii)
+            full_ids = np.zeros(T, dtype=np.int32)
+            full_c = np.zeros(T, dtype=np.float64)
+            full_ids[N:] = ids
+            full_c[N:] = p1
+            k_step[b] = commit_and_draft(x[b], int(p[b]), full_ids, full_c, cfg, L)  # (iii)-(iv)
+            p[b] += k_step[b]                                    # dynamically advance
+            steps[b] += 1
+            pr[0, b], pr[1, b], pr[2, b] = ids, p1, p2
+        ks.append(k_step)
+        if record:
+            inputs.append(in_step)
+            preds.append(pr)
+        n_iter += 1
+    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "inputs": inputs,
+            "preds": preds, "n_iter": n_iter, "done": bool((p >= T).all())}
+

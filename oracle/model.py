@@ -1,0 +1,131 @@
+"""Oracle: bidirectional transformer forward and per-position confidence, fp64.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+The paper fixes what the forward produces (Sec. 2.1, Eq. 2: a categorical
+distribution per position from one non-causal pass over prompt + generation,
+bidirectional per App. B.2) but not the architecture; the architecture below is
+the LLaDA/Dream family as configured: RMSNorm, rotate-half RoPE, multi-head (or
+grouped-query) attention over ALL positions, SwiGLU MLP, final RMSNorm, untied LM
+head, no biases.  Weights are read as given (bf16-exact values) and every
+operation runs in float64.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def rms_norm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
+    """x / sqrt(mean(x^2) + eps) * gain over the last axis."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * np.asarray(gain, np.float64)
+
+
+def rope_angles(n_pos: int, head_dim: int, theta: float) -> np.ndarray:
+    """Angle[t, j] = t * theta^(-2j/head_dim) for j < head_dim/2 (positions 0..n_pos-1)."""
+    j = np.arange(head_dim // 2, dtype=np.float64)
+    inv_freq = theta ** (-2.0 * j / head_dim)
+    return np.outer(np.arange(n_pos, dtype=np.float64), inv_freq)
+
+
+def apply_rope(x: np.ndarray, angles: np.ndarray) -> np.ndarray:
+    """Rotate-half RoPE: pairs (j, j + hd/2) rotated by angle[t, j].  x: [T, heads, hd]."""
+    half = x.shape[-1] // 2
+    c = np.cos(angles)[:, None, :]
+    s = np.sin(angles)[:, None, :]
+    x1, x2 = x[..., :half], x[..., half:]
+    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
+    """Non-causal softmax(q k^T / sqrt(hd)) v; every query sees every key.
+
+    q: [T, H, hd]; k, v: [T, G, hd] with H a multiple of G (query head h reads kv head
+    h // (H/G)).  Returns [T, H*hd].
+    """
+    T, H, hd = q.shape
+    G = k.shape[1]
+    rep = H // G
+    out = np.empty((T, H, hd), dtype=np.float64)
+    for h in range(H):
+        g = h // rep
+        s = q[:, h, :] @ k[:, g, :].T / np.sqrt(hd)
+        s = s - s.max(axis=1, keepdims=True)
+        w = np.exp(s)
+        w = w / w.sum(axis=1, keepdims=True)
+        out[:, h, :] = w @ v[:, g, :]
+    return out.reshape(T, H * hd)
+
+
+def silu(x: np.ndarray) -> np.ndarray:
+    return x / (1.0 + np.exp(-x))
+
+
+def _f64(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+def block(shape, lw: dict, h: np.ndarray, angles: np.ndarray) -> np.ndarray:
+    """One transformer block on the residual stream h [T, d] (returns the new stream)."""
+    T = h.shape[0]
+    H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    xn = rms_norm(h, lw["attn_norm"], shape.rms_eps)
+    q = (xn @ _f64(lw["wq"]).T).reshape(T, H, hd)
+    k = (xn @ _f64(lw["wk"]).T).reshape(T, G, hd)
+    v = (xn @ _f64(lw["wv"]).T).reshape(T, G, hd)
+    q = apply_rope(q, angles)
+    k = apply_rope(k, angles)
+    h = h + attention(q, k, v) @ _f64(lw["wo"]).T
+    xn = rms_norm(h, lw["mlp_norm"], shape.rms_eps)
+    a = silu(xn @ _f64(lw["w_gate"]).T) * (xn @ _f64(lw["w_up"]).T)
+    return h + a @ _f64(lw["w_down"]).T
+
+
+def forward_hidden(shape, weights: dict, tokens: np.ndarray) -> np.ndarray:
+    """Final-normed hidden states [T, d] of one sequence (one full bidirectional pass)."""
+    tokens = np.asarray(tokens)
+    if tokens.min() < 0 or tokens.max() >= shape.vocab:
+        raise ValueError("token id out of range")
+    h = _f64(weights["embed"])[tokens]
+    angles = rope_angles(len(tokens), shape.head_dim, shape.rope_theta)
+    for lw in weights["layers"]:
+        h = block(shape, lw, h, angles)
+    return rms_norm(h, weights["final_norm"], shape.rms_eps)
+
+
+def logits(weights: dict, hidden: np.ndarray) -> np.ndarray:
+    """LM-head logits z = hidden @ W_lm^T, [R, V]."""
+    return np.asarray(hidden, np.float64) @ _f64(weights["lm_head"]).T
+
+
+def softmax(z: np.ndarray) -> np.ndarray:
+    """Eq. 2: softmax over the whole vocabulary, per row."""
+    z = np.asarray(z, dtype=np.float64)
+    e = np.exp(z - z.max(axis=-1, keepdims=True))
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def confidence(z: np.ndarray):
+    """Top-1 id, top-1 probability c = max_v P (Eq. threshold_pd) and top-2 probability.
+
+    Ties go to the lowest index; the top-2 probability is the largest probability at an
+    index other than the top-1 index, so a tie at the top gives p2 == p1.
+    Returns (ids int32 [R], p1 float64 [R], p2 float64 [R]).
+    """
+    z = np.atleast_2d(np.asarray(z, dtype=np.float64))
+    ids = np.argmax(z, axis=1)                      # first maximal index
+    m = z[np.arange(z.shape[0]), ids]
+    e = np.exp(z - m[:, None])
+    s = e.sum(axis=1)
+    rest = z.copy()
+    rest[np.arange(z.shape[0]), ids] = -np.inf
+    z2 = rest.max(axis=1)
+    return ids.astype(np.int32), 1.0 / s, np.exp(z2 - m) / s
+
+
+def predict(shape, weights: dict, tokens: np.ndarray, rows=None):
+    """Forward + confidence: (ids, p1, p2) for positions ``rows`` (all positions by default)."""
+    hid = forward_hidden(shape, weights, tokens)
+    if rows is not None:
+        hid = hid[rows]
+    return confidence(logits(weights, hid))
