@@ -1,0 +1,463 @@
+#!/usr/bin/env python3
+"""Throughput of the DC-Leap denoise step on GB300.
+
+A step is one pass of the whole hot path: re-mask the window, one bidirectional
+forward over prompt + generation (embedding, 32 x {RMSNorm, QKV+RoPE GEMM, non-causal
+attention, O GEMM + residual, RMSNorm, gate/up GEMM + SwiGLU, down GEMM + residual},
+final RMSNorm, LM-head GEMM fused with softmax top-1/top-2), then the contiguous
+commit / draft update / advance.  The default workload is the LLaDA-8B shape at batch 1,
+prompt 256, generation 256, block 32, window 128, full recompute, with random-init bf16
+weights (seed 1) and a random prompt.
+
+Timed region: K steps (one CUDA-graph launch each) on the context stream, bracketed
+by CUDA events, inputs resident in HBM; generations of the same prompt run back to
+back (an on-device restart when a generation finishes), so `value` counts the tokens
+committed in exactly those K steps.  Per-kernel times come from a second pass of the
+same steps with timing events captured around every kernel.  `e2e` runs whole
+generations through the public API (prompt from pinned host memory, result read back).
+
+--impl reference times the CPU oracle (tests' reference implementation) on a bounded
+sample of the same step on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "generated tokens/s and ms/denoise-step, LLaDA-8B shape, 1×GB300; % roofline"
+
+WORKLOADS = {
+    # LLaDA-8B shape, batch 1, prompt 256, gen 256, block 32, L = M/2, full recompute
+    "llada8b": dict(shape="llada8b", batch=1, n_prompt=256, gen=256, block=32, window=128,
+                    seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
+    # the same architecture, long generation: prompt 512, gen 1024, batch 1
+    "llada8b-long": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
+                         seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
+    # 2-layer test model (latency-bound)
+    "tiny": dict(shape="tiny", batch=1, n_prompt=32, gen=64, block=32, window=32,
+                 seed=0, lm_scale=40.0, tau_c=0.70, tau_d=0.98),
+}
+
+
+def _env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def step_work(shape, B, N, M):
+    """Algorithmic flops per step by kernel class, and the minimum HBM bytes of a step."""
+    T = N + M
+    R = B * T
+    d, H, G, hd, F, V = (shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
+                         shape.ffn_dim, shape.vocab)
+    L = shape.n_layers
+    flops = {
+        "gemm_qkv": 2.0 * R * d * (H + 2 * G) * hd,
+        "gemm_o": 2.0 * R * H * hd * d,
+        "gemm_gateup": 2.0 * R * d * 2 * F,
+        "gemm_down": 2.0 * R * F * d,
+        "attention": 4.0 * B * T * T * H * hd,
+    }
+    per_layer = dict(flops)
+    total = {k: v * L for k, v in flops.items()}
+    total["gemm_lmhead"] = 2.0 * B * M * d * V
+    w_layer = 2.0 * (d * (H + 2 * G) * hd + H * hd * d + 2 * F * d + F * d + 2 * d)
+    bytes_ = L * w_layer + 2.0 * V * d + 2.0 * R * d + 2.0 * d
+    return per_layer, total, bytes_
+
+
+# ---------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid=None):
+        self.uuid = uuid
+        self.proc = None
+        self.f = None
+
+    def start(self):
+        try:
+            self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                   "-lms", "200"]
+            if self.uuid:
+                cmd += ["-i", self.uuid]
+            self.proc = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.count(",") >= 8]
+        self.f.close()
+        os.unlink(self.f.name)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if "Active" in v and "Not" not in v})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------- oracle timing
+def _layer_weights(shape, seed, layer):
+    import synthetic as syn
+    K = syn.TensorKind
+    d, H, G, hd, F = shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn_dim
+    dims = {"attn_norm": (K.ATTN_NORM, (d,)), "wq": (K.WQ, (H * hd, d)), "wk": (K.WK, (G * hd, d)),
+            "wv": (K.WV, (G * hd, d)), "wo": (K.WO, (d, H * hd)), "mlp_norm": (K.MLP_NORM, (d,)),
+            "w_gate": (K.W_GATE, (F, d)), "w_up": (K.W_UP, (F, d)), "w_down": (K.W_DOWN, (d, F))}
+    out = {}
+    for name, (kind, shp) in dims.items():
+        n = int(np.prod(shp))
+        if kind in K.NORMS:
+            v = syn.weight_values(seed, syn.tensor_id(kind, layer), 0, n, 0.0, 1.0)
+        else:
+            v = syn.weight_values(seed, syn.tensor_id(kind, layer), 0, n, 0.02)
+        out[name] = v.reshape(shp)
+    return out
+
+
+class OracleSample:
+    """A bounded sample of one step of the oracle: one transformer block over all T rows,
+    and the LM head + confidence over 16 generation rows x 1/16 of the vocabulary; scaled
+    to a step as n_layers x block + (B*M/16) x 16 x LM-head sample."""
+
+    def __init__(self, wl):
+        import synthetic as syn
+        self.syn = syn
+        self.shape = syn.SHAPES[wl["shape"]]
+        self.wl = wl
+        sh = self.shape
+        B, N, M = wl["batch"], wl["n_prompt"], wl["gen"]
+        self.T = N + M
+        prompt = syn.prompt_ids(1000, 1, N, sh.mask_id)[0]
+        tokens = np.concatenate([prompt, np.full(M, sh.mask_id, np.int32)])
+        rows = {}
+        for t in np.unique(tokens):
+            rows[int(t)] = syn.weight_values(wl["seed"], syn.tensor_id(syn.TensorKind.EMBED, 0),
+                                             int(t) * sh.d_model, sh.d_model, 0.02)
+        self.h = np.stack([rows[int(t)] for t in tokens]).astype(np.float64)
+        self.lw = _layer_weights(sh, wl["seed"], 0)
+        self.vslice = max(1, sh.vocab // 16)
+        std = float(np.float32(0.02) * np.float32(wl["lm_scale"]))
+        self.lm = syn.weight_values(wl["seed"], syn.tensor_id(syn.TensorKind.LM_HEAD, 0), 0,
+                                    self.vslice * sh.d_model, std).reshape(self.vslice, sh.d_model)
+        self.lm_rows = min(16, B * M)
+        self.scale_lm = (B * M / self.lm_rows) * (sh.vocab / self.vslice)
+        self.B = B
+
+    def step_seconds(self):
+        from oracle import model
+        sh = self.shape
+        ang = model.rope_angles(self.T, sh.head_dim, sh.rope_theta)
+        t0 = time.perf_counter()
+        for _ in range(self.B):
+            h1 = model.block(sh, self.lw, self.h, ang)
+        t_block = time.perf_counter() - t0
+        hn = model.rms_norm(h1[-self.lm_rows:], np.ones(sh.d_model), sh.rms_eps)
+        t0 = time.perf_counter()
+        model.confidence(model.logits({"lm_head": self.lm}, hn))
+        t_lm = time.perf_counter() - t0
+        return sh.n_layers * t_block + self.scale_lm * t_lm, t_block + t_lm
+
+    def describe(self):
+        sh = self.shape
+        return (f"one transformer block over all {self.T} rows x batch {self.B} (x{sh.n_layers} layers) "
+                f"+ LM head/confidence on {self.lm_rows} rows x {self.vslice} vocab rows "
+                f"(x{self.scale_lm:.0f}); fp64 numpy, weight generation untimed")
+
+
+def run_reference(args):
+    rank = _env_int("RANK", 0)
+    if rank != 0:
+        return 0
+    wl = WORKLOADS[args.workload]
+    samp = OracleSample(wl)
+    for _ in range(args.warmup):
+        samp.step_seconds()
+    secs, cpu = [], 0.0
+    for _ in range(args.steps):
+        s, c = samp.step_seconds()
+        secs.append(s)
+        cpu += c
+    ms = 1e3 * statistics.mean(secs)
+    tps = wl["batch"] * 1.0 / (ms / 1e3)  # one committed token per row per step (see below)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": tps, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": _config(wl, args),
+        "cpu_baseline": {"value": tps, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": samp.describe() + "; tokens/s assumes one committed token per row "
+                         "per step (the oracle cannot afford a full 8B-shape trajectory)",
+                         "cpu_seconds_timed": cpu},
+        "e2e": {"value": tps, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def _config(wl, args):
+    return {"workload": f"{wl['shape']}-shape batch {wl['batch']}, prompt {wl['n_prompt']}, gen {wl['gen']}, "
+                        f"block {wl['block']}, window {wl['window']}, tau_commit {wl['tau_c']}, "
+                        f"tau_draft {wl['tau_d']}, full recompute",
+            "global_batch": wl["batch"] * max(1, args.gpus), "seq_len": wl["n_prompt"] + wl["gen"],
+            "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single",
+            "l2": "no flush needed: every step streams all weights (>> 129 MB L2)"}
+
+
+# ---------------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+
+    import synthetic as syn
+    rank, world, local = _env_int("RANK", 0), _env_int("WORLD_SIZE", 1), _env_int("LOCAL_RANK", 0)
+    dist = None
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if local == 0:
+        import __graft_entry__
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    import paper_2607_20467_gb300 as dcl
+
+    wl = WORKLOADS[args.workload]
+    shape = syn.SHAPES[wl["shape"]]
+    B, N, M = wl["batch"], wl["n_prompt"], wl["gen"]
+    T = N + M
+    stream = torch.cuda.Stream()
+    ctx = dcl.Context(shape, max_batch=B, max_seq=T, stream=stream.cuda_stream)
+    ctx.init_random_weights(wl["seed"], 0.02, wl["lm_scale"], 0.0)
+    prompt = syn.prompt_ids(1000 + rank, B, N, shape.mask_id)
+    cfg = dcl.decode_config(tau_commit=wl["tau_c"], tau_draft=wl["tau_d"], max_window=wl["window"],
+                            block_len=wl["block"], gen_len=M)
+    ctx.set_prompt(prompt, cfg)
+
+    # one generation step by step: the trajectory (tokens committed per step) + warm-up
+    ks = []
+    while sum(ks) < B * M and len(ks) < 4 * M:
+        ks.append(int(ctx.step(return_k=True).sum()))
+    S = len(ks)
+    ctx.restart()
+    for _ in range(args.warmup):
+        ctx.step()
+    torch.cuda.synchronize()
+
+    def timed(nsteps, profiled=False):
+        ctx.restart()
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        j = tokens = 0
+        t0.record(stream)
+        for _ in range(nsteps):
+            if j == S:
+                ctx.restart()
+                j = 0
+            ctx.step()
+            tokens += ks[j]
+            j += 1
+        t1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        _, p = ctx.get_state()
+        assert int((p - N).sum()) == sum(ks[:j]), "step trajectory did not replay deterministically"
+        return t0.elapsed_time(t1), tokens
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        uuid = None
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    ms, tokens = timed(args.steps)
+    clocks = sampler.stop()
+
+    # per-kernel device times: the same steps with timing events around every kernel
+    ctx.set_profiling(True)
+    ms_prof, _ = timed(min(args.steps, max(3, S)))
+    kern_ms, kern_kind = ctx.profile_last_step()
+    ctx.set_profiling(False)
+
+    # e2e through the public API: set_prompt (pinned host prompt) + generate (pinned out)
+    pin_prompt = torch.from_numpy(prompt.copy()).pin_memory().numpy()
+    pin_out = torch.zeros((B, M), dtype=torch.int32).pin_memory().numpy()
+    e2e_s, e2e_steps = [], []
+    for _ in range(args.e2e_iters):
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t = time.perf_counter()
+        ctx.set_prompt(pin_prompt, cfg)
+        _, st, _ = ctx.generate(max_steps=4 * M, out=pin_out)
+        e2e_s.append(time.perf_counter() - t)
+        e2e_steps.append(int(st.steps))
+        assert st.done == 1
+
+    # aggregate over ranks (timing only: max time, summed tokens)
+    def allmax(v):
+        if not dist:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def allsum(v):
+        if not dist:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return float(t.item())
+
+    ms_max = allmax(ms)
+    tokens_all = allsum(tokens)
+    e2e_mean = allmax(statistics.mean(e2e_s))
+    peaks = _peaks()
+    per_layer, total_flops, step_bytes = step_work(shape, B, N, M)
+
+    # per-kernel table and the dominant kernel's roofline
+    names = dcl.KERNEL_KINDS
+    table = {}
+    for t_ms, k in zip(kern_ms, kern_kind):
+        e = table.setdefault(names[k], {"launches": 0, "ms": 0.0})
+        e["launches"] += 1
+        e["ms"] += float(t_ms)
+    tot = sum(e["ms"] for e in table.values())
+    for e in table.values():
+        e["share"] = e["ms"] / tot if tot else 0.0
+    gemms = {k: v for k, v in table.items() if k.startswith("gemm") and k in total_flops}
+    dom = max(gemms, key=lambda k: gemms[k]["ms"])
+    avg_ms = gemms[dom]["ms"] / gemms[dom]["launches"]
+    flops_launch = total_flops[dom] / gemms[dom]["launches"]
+    achieved = flops_launch / (avg_ms / 1e3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    for k, e in table.items():
+        if k in total_flops:
+            e["tflops"] = total_flops[k] / (e["ms"] / 1e3) / 1e12
+    step_flops = sum(total_flops.values())
+    ms_step = ms_max / args.steps
+    t_roof = max(step_flops / (peak * 1e12), step_bytes / (peaks["hbm_gbs"] * 1e9))
+    traffic = _traffic_from_profiles(dom)
+
+    # CPU oracle on a bounded sample (rank 0, one GPU only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        samp = OracleSample(wl)
+        s, c = samp.step_seconds()
+        tps_cpu = (tokens / args.steps) / s
+        cpu = {"value": tps_cpu, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": samp.describe() + "; scaled to one step, tokens per step taken from the "
+                         "GPU run of the same trajectory", "ms_per_step": 1e3 * s, "cpu_seconds_timed": c}
+
+    line = {
+        "metric": METRIC, "value": tokens_all / (ms_max / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": f"synthetic: random-init bf16 weights (seed {wl['seed']}, LM head x{wl['lm_scale']}), "
+                f"random prompts",
+        "config": _config(wl, argparse.Namespace(gpus=world)),
+        "steps_per_token": (args.steps * B) / max(1.0, tokens),
+        "trajectory_steps": S,
+        "step_roofline": {"flops": step_flops, "bytes": step_bytes, "t_roof_ms": 1e3 * t_roof,
+                          "frac": 1e3 * t_roof / ms_step, "peak_tflops": peak,
+                          "peak_source": peaks["source"] + " sustained"},
+        "roofline": {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
+                     "avg_launch_ms": avg_ms, "flops_per_launch": flops_launch},
+        "kernels": table,
+        "ms_per_step_profiled": ms_prof / min(args.steps, max(3, S)),
+        "gpu_launches": args.steps * len(kern_ms),
+        "clocks": clocks,
+        "e2e": {"value": world * B * M / e2e_mean, "unit": "tokens/s",
+                "h2d_bytes_per_step": 4 * B * T + 12 * B + 4,
+                "d2h_bytes_per_step": 4 * B * M + 8 * B + 4 * (statistics.mean(e2e_steps) + 1),
+                "step": "one dcl_set_prompt + dcl_generate call (a whole generation)",
+                "ms_per_generation": 1e3 * e2e_mean, "steps_per_generation": statistics.mean(e2e_steps)},
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+    ctx.close()
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def _traffic_from_profiles(kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if present."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            return json.load(f).get(kernel)
+    except (OSError, ValueError):
+        return None
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="llada8b")
+    ap.add_argument("--e2e-iters", type=int, default=2)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,256 @@
+/*
+ * dcleap.h - C ABI of libdcleap.so: the DC-Leap denoise step of a masked-diffusion
+ * LM on one NVIDIA GB300 (sm_103a), in hand-written CUDA.
+ *
+ * The calls follow the paper's statement of the problem: Algorithm 1 takes a model,
+ * a prompt, a generation length, a maximum window size L and the two thresholds
+ * (tau_commit, tau_draft) and returns the sequence x.  One denoise step is the
+ * four-step iteration of Sec. 3.3: (i) re-mask the window [p, p+L) (Eq. remasking),
+ * (ii) one bidirectional forward giving per-position softmax confidences (Eq. 2),
+ * (iii) K by the prefix-product rule (Eq. compute_k), (iv) commit x[p:p+K] and
+ * refresh drafts at every position >= p+L (Eq. draft_update); then p += K.
+ *
+ * Conventions (all calls):
+ *   - Every call returns a dcl_status and never aborts the process; on failure the
+ *     message is available from dcl_last_error(ctx).
+ *   - Pointers named *_dev are device pointers owned by the caller; pointers without
+ *     that suffix are host pointers owned by the caller.  The context owns every
+ *     device buffer it allocates (weights, activations, scratch) and frees them in
+ *     dcl_destroy.
+ *   - Work is stream-ordered on the stream given to dcl_create.  Calls that return
+ *     host data (dcl_step with k_out, dcl_generate, dcl_get_state) synchronise that
+ *     stream; the others are asynchronous.
+ *   - Token ids are int32 in [0, vocab).  Matrices are row-major bf16 in the
+ *     nn.Linear layout [out_features][in_features].
+ *   - Decisions compare float32 confidences with float32 thresholds, strictly (>).
+ */
+#ifndef DCLEAP_H
+#define DCLEAP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DCL_OK = 0,
+  DCL_ERR_INVALID_ARG = 1, /* a NULL/negative/oversized argument or an out-of-range id */
+  DCL_ERR_STATE = 2,       /* call out of order (e.g. dcl_step before dcl_set_prompt) */
+  DCL_ERR_OOM = 3,         /* device allocation failed */
+  DCL_ERR_CUDA = 4,        /* a CUDA runtime/driver error, or a kernel-reported fault */
+  DCL_ERR_TIMEOUT = 5,     /* dcl_generate ran max_steps without finishing, or a device-side
+                              bounded wait gave up (the kernel returned without hanging) */
+  DCL_ERR_UNSUPPORTED = 6  /* a shape the kernels do not support (see dcl_create) */
+} dcl_status;
+
+/* Transformer shape (Sec. 2.1: one bidirectional network over prompt + generation).
+ * Supported: head_dim in {64, 128}; d_model, ffn_dim multiples of 128;
+ * n_heads a multiple of n_kv_heads; (n_heads + n_kv_heads) * head_dim a multiple of 128. */
+typedef struct {
+  int32_t n_layers, d_model, n_heads, n_kv_heads, head_dim, ffn_dim, vocab, mask_id;
+  float rope_theta, rms_eps;
+} dcl_model_config;
+
+/* Decoding hyper-parameters (Algorithm 1 inputs; defaults of Sec. 4.1 in comments). */
+typedef struct {
+  float tau_commit;          /* 0.70: commit threshold of Eq. compute_k (strict >) */
+  float tau_draft;           /* 0.98: draft threshold of Eq. draft_update (strict >) */
+  int32_t max_window;        /* L; 0 means gen_len / 2 */
+  int32_t block_len;         /* 32: semi-autoregressive block length */
+  int32_t gen_len;           /* M, the number of generated positions */
+  int32_t kv_cache;          /* 0: full recompute every step (the only mode built) */
+  int32_t min_commit;        /* 1: K = max(K, min_commit) so every step makes progress;
+                                0 keeps the literal rule (may stall; bounded by max_steps) */
+  int32_t contiguous_drafts; /* 0; 1 = App. E variant (drafts only as an unbroken chain) */
+} dcl_decode_config;
+
+typedef struct {
+  int64_t steps;      /* denoise iterations run */
+  int64_t tokens;     /* generated tokens committed (all rows) */
+  double elapsed_ms;  /* wall time of dcl_generate, host clock */
+  int32_t done;       /* 1 if every row reached p = N + M */
+} dcl_stats;
+
+/* Optional device allocator (e.g. a framework's caching allocator). */
+typedef struct {
+  void* (*alloc)(size_t bytes, void* user); /* returns a device pointer or NULL */
+  void (*free)(void* ptr, void* user);
+  void* user;
+} dcl_allocator;
+
+/* Weight kinds for dcl_set_weight (shapes with H = n_heads, G = n_kv_heads, hd =
+ * head_dim, d = d_model, F = ffn_dim, V = vocab). */
+typedef enum {
+  DCL_W_EMBED = 0,      /* [V][d]     token embedding           (global) */
+  DCL_W_ATTN_NORM = 1,  /* [d]        RMSNorm gain before attention */
+  DCL_W_Q = 2,          /* [H*hd][d] */
+  DCL_W_K = 3,          /* [G*hd][d] */
+  DCL_W_V = 4,          /* [G*hd][d] */
+  DCL_W_O = 5,          /* [d][H*hd] */
+  DCL_W_MLP_NORM = 6,   /* [d]        RMSNorm gain before the MLP */
+  DCL_W_GATE = 7,       /* [F][d]     SwiGLU gate */
+  DCL_W_UP = 8,         /* [F][d]     SwiGLU up */
+  DCL_W_DOWN = 9,       /* [d][F] */
+  DCL_W_FINAL_NORM = 10,/* [d]        final RMSNorm gain        (global) */
+  DCL_W_LM_HEAD = 11    /* [V][d]     untied LM head            (global) */
+} dcl_weight_kind;
+
+typedef struct dcl_ctx dcl_ctx;
+
+/* Create a context on the current CUDA device.
+ *   cfg        model shape, or NULL for an ops-only context (dcl_accept, dcl_op_*).
+ *   max_batch  largest batch (rows) later passed to dcl_set_prompt.
+ *   max_seq    largest N + M later passed to dcl_set_prompt.
+ *   cuda_stream a cudaStream_t that all work goes to; NULL makes the context create and
+ *              own a blocking stream (ordered with the legacy default stream).  The
+ *              step is captured into a CUDA graph on this stream, so it must not be the
+ *              legacy default stream itself.
+ *   alloc      optional allocator; NULL uses cudaMalloc/cudaFree.
+ * Weights are allocated (uninitialised) here: 2 bytes per parameter.
+ * Errors: INVALID_ARG, UNSUPPORTED (shape), OOM, CUDA.  *out is NULL on failure. */
+dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t max_seq,
+                      void* cuda_stream, const dcl_allocator* alloc, dcl_ctx** out);
+
+/* Copy one weight tensor (bf16, layout above) into the context; `layer` is ignored for
+ * global tensors.  src is a host pointer (src_is_device = 0) or a device pointer (1).
+ * The context keeps its own copy (re-laid out internally).  Errors: INVALID_ARG, CUDA. */
+dcl_status dcl_set_weight(dcl_ctx* ctx, int32_t kind, int32_t layer, const void* src,
+                          int32_t src_is_device);
+
+/* Fill every weight on the device from the counter-based generator of the synthetic
+ * workloads (SplitMix64 of seed<<48 | tensor<<32 | index, sum of four 16-bit fields,
+ * scaled to `std`, rounded to bf16).  The LM head uses std * lm_head_scale; RMSNorm
+ * gains are 1 + the same draw scaled to norm_gain_std.  seed < 65536.  Async. */
+dcl_status dcl_init_random_weights(dcl_ctx* ctx, uint64_t seed, float std, float lm_head_scale,
+                                   float norm_gain_std);
+
+/* Algorithm 1 initialisation: x = prompt ++ [MASK]^M and p = N for every row
+ * (Eq. 1).  prompt is host int32 [batch][n_prompt]; batch <= max_batch,
+ * n_prompt + cfg->gen_len <= max_seq.  Validates ids, uploads the state and builds
+ * (or reuses) the CUDA graph of one step for this shape.
+ * Errors: INVALID_ARG, UNSUPPORTED (kv_cache != 0), CUDA. */
+dcl_status dcl_set_prompt(dcl_ctx* ctx, int32_t batch, const int32_t* prompt, int32_t n_prompt,
+                          const dcl_decode_config* cfg);
+
+/* One denoise step (Sec. 3.3 steps (i)-(iv) and the advance), one CUDA-graph launch on
+ * the context stream.  Rows already finished are left unchanged.  If k_out is not
+ * NULL it receives the K of every row (host int32 [batch]; the call synchronises).
+ * Errors: STATE (no prompt), CUDA. */
+dcl_status dcl_step(dcl_ctx* ctx, int32_t* k_out);
+
+/* Run steps until every row has p = N + M (Algorithm 1's loop) or max_steps steps
+ * have run.  out (host int32 [batch][M], may be NULL) receives x[N:N+M]; st (may be
+ * NULL) the counters.  Synchronises.  Errors: STATE, CUDA, TIMEOUT (max_steps reached;
+ * out still holds the partial result). */
+dcl_status dcl_generate(dcl_ctx* ctx, int32_t max_steps, int32_t* out, dcl_stats* st);
+
+/* Reset the decoding state to the one the last dcl_set_prompt made (x = prompt ++ MASK,
+ * p = N, counters 0), asynchronously on the context stream (device-to-device copies; no
+ * host synchronisation).  Lets a caller run generations of the same prompt back to back.
+ * Errors: STATE, CUDA. */
+dcl_status dcl_restart(dcl_ctx* ctx);
+
+/* Read / write the decoding state (x: host int32 [batch][N+M], p: host int32 [batch]),
+ * e.g. to resume a run or to drive teacher-forced parity.  get synchronises.
+ * set validates ids and N <= p <= N+M.  Errors: STATE, INVALID_ARG, CUDA. */
+dcl_status dcl_get_state(dcl_ctx* ctx, int32_t* x, int32_t* p);
+dcl_status dcl_set_state(dcl_ctx* ctx, const int32_t* x, const int32_t* p);
+
+/* Parity hook: step (i) and (ii) only (re-mask, forward, confidence) on the current
+ * state, without committing.  Any output may be NULL:
+ *   logits_dev bf16 [batch][M][V] logits of the generation rows (an extra plain GEMM),
+ *   top1_dev int32 [batch][M], p1_dev / p2_dev float [batch][M] from the fused
+ *   LM-head epilogue (the values the step itself uses).
+ * Errors: STATE, CUDA. */
+dcl_status dcl_forward_debug(dcl_ctx* ctx, void* logits_dev, int32_t* top1_dev, float* p1_dev,
+                             float* p2_dev);
+
+/* Parity hook: the residual stream after the embedding (layer = -1) or after
+ * transformer block `layer` of the last forward, copied to h_dev (float [batch*(N+M)][d]).
+ * Call after dcl_forward_debug.  Errors: STATE, INVALID_ARG, CUDA. */
+dcl_status dcl_debug_hidden(dcl_ctx* ctx, int32_t layer, float* h_dev);
+
+/* Acceptance pass of one block from given logits (Eq. 2 confidence + Eq. compute_k +
+ * Eq. draft_update), for B independent rows of P positions:
+ *   logits_dev    bf16 [B][P][V]; only uncommitted positions are read.
+ *   committed_dev int32 [B]: c_b positions already committed (left-aligned), so the
+ *                 window starts at p = c_b; rows with c_b >= P are left unchanged.
+ *   x_dev         int32 [B][P], in/out: receives the committed ids and new drafts.
+ *   cfg           thresholds, max_window (0 = P/2), min_commit, contiguous_drafts.
+ *   k_dev         int32 [B] out: K of every row.
+ * Async; P <= 4096, B*P <= 1<<20.  Errors: INVALID_ARG, CUDA. */
+dcl_status dcl_accept(dcl_ctx* ctx, const void* logits_dev, int32_t B, int32_t P, int32_t V,
+                      const int32_t* committed_dev, int32_t* x_dev, const dcl_decode_config* cfg,
+                      int32_t* k_dev);
+
+/* ---- single-kernel entry points (the kernels of the step, for parity tests) ---- */
+
+/* y = x / sqrt(mean(x^2) + eps) * gain.  x_dev float [rows][d], gain_dev bf16 [d],
+ * y_dev bf16 [rows][d]; d a multiple of 4.  Async. */
+dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev, void* y_dev,
+                          int32_t rows, int32_t d, float eps);
+
+/* out = a @ w^T on the tcgen05 tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];
+ * mode 0: out bf16 [M][N]; mode 1: out float [M][N] += a @ w^T (residual add).
+ * K, N multiples of 64.  Async. */
+dcl_status dcl_op_linear(dcl_ctx* ctx, const void* a_dev, const void* w_dev, void* out_dev,
+                         int32_t M, int32_t N, int32_t K, int32_t mode);
+
+/* Non-causal attention softmax(q k^T / sqrt(hd)) v over all T positions of each of
+ * `batch` sequences.  qkv_dev bf16 [batch*T][(H+2G)*hd] (q | k | v column blocks, RoPE
+ * already applied), out_dev bf16 [batch*T][H*hd].  hd in {64, 128}.  Async. */
+dcl_status dcl_op_attention(dcl_ctx* ctx, const void* qkv_dev, void* out_dev, int32_t batch,
+                            int32_t T, int32_t H, int32_t G, int32_t hd);
+
+/* LM head + softmax confidence fused: for each row r of x_dev (bf16 [R][d]),
+ * z = x_r @ w^T (w_dev bf16 [V][d]); top1_dev[r] = argmax (lowest index on ties),
+ * p1_dev[r] = max softmax(z), p2_dev[r] = second largest probability.  Logits never
+ * reach memory.  d a multiple of 64.  Async. */
+dcl_status dcl_op_lmhead_top2(dcl_ctx* ctx, const void* x_dev, const void* w_dev, int32_t R,
+                              int32_t V, int32_t d, int32_t* top1_dev, float* p1_dev,
+                              float* p2_dev);
+
+/* Fill dst_dev (bf16, count elements) from the weight generator of
+ * dcl_init_random_weights for tensor id `tid` starting at element `start`.  Async. */
+dcl_status dcl_op_generate(dcl_ctx* ctx, void* dst_dev, uint64_t seed, int32_t tid, int64_t start,
+                           int64_t count, float std, float mean);
+
+/* ---- per-kernel timing of the step graph ---- */
+
+/* Kernel classes reported by dcl_profile_last_step. */
+typedef enum {
+  DCL_K_EMBED = 0,       /* remask + embedding gather */
+  DCL_K_RMSNORM = 1,
+  DCL_K_GEMM_QKV = 2,    /* QKV projection + RoPE epilogue */
+  DCL_K_ATTENTION = 3,
+  DCL_K_GEMM_O = 4,      /* output projection + residual */
+  DCL_K_GEMM_GATEUP = 5, /* gate/up projection + SwiGLU */
+  DCL_K_GEMM_DOWN = 6,   /* down projection + residual */
+  DCL_K_GEMM_LMHEAD = 7, /* LM head + softmax/top-2 partials */
+  DCL_K_COMBINE = 8,     /* merge of the LM-head partials */
+  DCL_K_DCV = 9          /* commit / draft / advance */
+} dcl_kernel_kind;
+
+/* enable = 1 re-captures the step graph with a pair of timing events (CUDA event record
+ * nodes on the context stream) around every kernel; 0 restores the plain graph.
+ * Takes effect at once if a prompt is set, else at the next dcl_set_prompt. */
+dcl_status dcl_set_profiling(dcl_ctx* ctx, int32_t enable);
+
+/* Per-kernel device durations (ms) of the most recent step run with profiling on, in
+ * launch order: ms[i], kind[i] for i < *n (at most cap).  Synchronises.
+ * Errors: STATE (profiling off or no step yet), CUDA. */
+dcl_status dcl_profile_last_step(dcl_ctx* ctx, float* ms, int32_t* kind, int32_t cap, int32_t* n);
+
+/* Last error message of this context (or of the last failed dcl_create when ctx is NULL). */
+const char* dcl_last_error(const dcl_ctx* ctx);
+
+/* Free everything the context owns.  NULL is a no-op. */
+void dcl_destroy(dcl_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DCLEAP_H */

@@ -9,10 +9,30 @@ the LLaDA/Dream family as configured: RMSNorm, rotate-half RoPE, multi-head (or
 grouped-query) attention over ALL positions, SwiGLU MLP, final RMSNorm, untied LM
 head, no biases.  Weights are read as given (bf16-exact values) and every
 operation runs in float64.
+
+Precision reading.  The paper evaluates bf16 checkpoints but never states where
+activations are rounded.  ``bf16_operands=False`` (default) is the pure definition:
+nothing is rounded.  ``bf16_operands=True`` is a bf16 model: every operand of a
+matrix product is stored in bf16 exactly where a bf16 model stores it - the RMSNorm
+outputs, q/k (after RoPE) and v, the attention output, the SwiGLU output and the
+final hidden state - while products accumulate, and norms, softmax and the residual
+stream are computed, in float64.  The rounding is value -> float32 -> bf16, both
+round-to-nearest-even.
 """
 from __future__ import annotations
 
 import numpy as np
+
+
+def to_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bf16 value (via float32; both steps round to nearest even)."""
+    b = np.ascontiguousarray(np.asarray(x, dtype=np.float64).astype(np.float32)).view(np.uint32)
+    r = ((b + np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)) << np.uint32(16)
+    return r.view(np.float32).astype(np.float64).reshape(np.shape(x))
+
+
+def _maybe_bf16(x, on):
+    return to_bf16(x) if on else x
 
 
 def rms_norm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
@@ -65,32 +85,41 @@ def _f64(a):
     return np.asarray(a, dtype=np.float64)
 
 
-def block(shape, lw: dict, h: np.ndarray, angles: np.ndarray) -> np.ndarray:
+def block(shape, lw: dict, h: np.ndarray, angles: np.ndarray, bf16_operands: bool = False) -> np.ndarray:
     """One transformer block on the residual stream h [T, d] (returns the new stream)."""
     T = h.shape[0]
     H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
-    xn = rms_norm(h, lw["attn_norm"], shape.rms_eps)
+    r = bf16_operands
+    xn = _maybe_bf16(rms_norm(h, lw["attn_norm"], shape.rms_eps), r)
     q = (xn @ _f64(lw["wq"]).T).reshape(T, H, hd)
     k = (xn @ _f64(lw["wk"]).T).reshape(T, G, hd)
-    v = (xn @ _f64(lw["wv"]).T).reshape(T, G, hd)
-    q = apply_rope(q, angles)
-    k = apply_rope(k, angles)
-    h = h + attention(q, k, v) @ _f64(lw["wo"]).T
-    xn = rms_norm(h, lw["mlp_norm"], shape.rms_eps)
-    a = silu(xn @ _f64(lw["w_gate"]).T) * (xn @ _f64(lw["w_up"]).T)
+    v = _maybe_bf16((xn @ _f64(lw["wv"]).T).reshape(T, G, hd), r)
+    q = _maybe_bf16(apply_rope(q, angles), r)
+    k = _maybe_bf16(apply_rope(k, angles), r)
+    h = h + _maybe_bf16(attention(q, k, v), r) @ _f64(lw["wo"]).T
+    xn = _maybe_bf16(rms_norm(h, lw["mlp_norm"], shape.rms_eps), r)
+    a = _maybe_bf16(silu(xn @ _f64(lw["w_gate"]).T) * (xn @ _f64(lw["w_up"]).T), r)
     return h + a @ _f64(lw["w_down"]).T
 
 
-def forward_hidden(shape, weights: dict, tokens: np.ndarray) -> np.ndarray:
-    """Final-normed hidden states [T, d] of one sequence (one full bidirectional pass)."""
+def forward_hidden(shape, weights: dict, tokens: np.ndarray, bf16_operands: bool = False,
+                   upto_layer: int = None) -> np.ndarray:
+    """Final-normed hidden states [T, d] of one sequence (one full bidirectional pass).
+
+    With ``upto_layer`` = l the un-normed residual stream after block l is returned
+    instead (l = -1: after the embedding)."""
     tokens = np.asarray(tokens)
     if tokens.min() < 0 or tokens.max() >= shape.vocab:
         raise ValueError("token id out of range")
     h = _f64(weights["embed"])[tokens]
+    if upto_layer == -1:
+        return h
     angles = rope_angles(len(tokens), shape.head_dim, shape.rope_theta)
-    for lw in weights["layers"]:
-        h = block(shape, lw, h, angles)
-    return rms_norm(h, weights["final_norm"], shape.rms_eps)
+    for li, lw in enumerate(weights["layers"]):
+        h = block(shape, lw, h, angles, bf16_operands)
+        if upto_layer == li:
+            return h
+    return _maybe_bf16(rms_norm(h, weights["final_norm"], shape.rms_eps), bf16_operands)
 
 
 def logits(weights: dict, hidden: np.ndarray) -> np.ndarray:
@@ -123,9 +152,9 @@ def confidence(z: np.ndarray):
     return ids.astype(np.int32), 1.0 / s, np.exp(z2 - m) / s
 
 
-def predict(shape, weights: dict, tokens: np.ndarray, rows=None):
+def predict(shape, weights: dict, tokens: np.ndarray, rows=None, bf16_operands: bool = False):
     """Forward + confidence: (ids, p1, p2) for positions ``rows`` (all positions by default)."""
-    hid = forward_hidden(shape, weights, tokens)
+    hid = forward_hidden(shape, weights, tokens, bf16_operands)
     if rows is not None:
         hid = hid[rows]
     return confidence(logits(weights, hid))

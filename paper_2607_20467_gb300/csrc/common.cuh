@@ -1,0 +1,118 @@
+// Shared device helpers and the internal (C++) interface between the library's
+// translation units.  Nothing here is part of the C ABI (include/dcleap.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dcl {
+
+// ---------------------------------------------------------------- device error word
+// Kernels never trap: they record the first fault here and return.  The host reads
+// the word at its sync points and turns it into a dcl_status.
+enum DevErr : int {
+  DERR_NONE = 0,
+  DERR_TOKEN_RANGE = 1,     // a token id outside [0, vocab) reached the embedding
+  DERR_WAIT_TIMEOUT = 2,    // a bounded mbarrier wait gave up (GEMM pipeline)
+  DERR_BAD_SHAPE = 3,       // a kernel was launched with a shape it does not support
+};
+
+__device__ __forceinline__ void report_error(int* err, int code) {
+  if (err) atomicCAS(err, 0, code);
+}
+
+// ---------------------------------------------------------------- small helpers
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ---------------------------------------------------------------- GEMM (gemm_tc.cu)
+// out = A[M][K] @ W[N][K]^T on tcgen05 tensor cores, with a fused epilogue.
+enum Epilogue : int {
+  EPI_BF16 = 0,      // out bf16 [M][ldo]
+  EPI_RESID_F32 = 1, // out float [M][ldo] += acc
+  EPI_QKV_ROPE = 2,  // out bf16 [M][ldo]; rotate-half RoPE on columns < rope_cols
+  EPI_SWIGLU = 3,    // W rows interleaved per 128: gate block then up block; out bf16
+                     // [M][ldo] column n = silu(gate_n) * up_n
+  EPI_LMHEAD = 4,    // per (row, 256-column block): float4 {max, sum exp(z-max),
+                     // argmax id (bits), second largest z}; columns >= vocab ignored
+};
+
+struct EpiParams {
+  void* out = nullptr;
+  int ldo = 0;
+  const float* rope_cos = nullptr;  // [T][head_dim/2]
+  const float* rope_sin = nullptr;
+  int rope_cols = 0;
+  int head_dim = 0;
+  int seq_T = 1;                    // rows per sequence (position = row % seq_T)
+  int vocab = 0;
+};
+
+struct GemmPlan {
+  CUtensorMap ta, tb;
+  int M = 0, N = 0, K = 0;
+  int bn = 256;
+  int epi = EPI_BF16;
+  EpiParams ep;
+  int grid = 0;
+  int n_tiles = 0;
+  size_t smem = 0;
+};
+
+// Encode the tensor maps and choose the tile width / grid.  A is [M][K] bf16 (row
+// pitch K), W is [N][K] bf16.  bn = 0 lets the planner choose 128 or 256.
+cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
+                      int epi, const EpiParams& ep, int num_sms, int bn, const char** why);
+cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
+int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
+
+// ---------------------------------------------------------------- attention (attention.cu)
+cudaError_t attention_launch(const __nv_bfloat16* qkv, __nv_bfloat16* out, int batch, int T,
+                             int H, int G, int hd, cudaStream_t stream);
+
+// ---------------------------------------------------------------- other kernels (kernels.cu)
+cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
+                                int mask_id, int vocab, const __nv_bfloat16* embed, int d,
+                                float* h, int* err, cudaStream_t stream);
+// rows_per_seq / seq_stride / row_offset map output row r to input row
+// (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq.
+cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows,
+                           int d, float eps, int rows_per_seq, int seq_stride, int row_offset,
+                           cudaStream_t stream);
+cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
+                                  float* p2, cudaStream_t stream);
+struct DcvParams {
+  float tau_commit, tau_draft;
+  int window, min_commit, contiguous_drafts;
+};
+// One step's acceptance on the generation rows: ids/c are [batch][M] (position N + i).
+cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
+                              const int32_t* ids, const float* c, int batch, int N, int M,
+                              const DcvParams& prm, int32_t* done_count, cudaStream_t stream);
+// Block acceptance from bf16 logits (dcl_accept).
+cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B,
+                                int P, int V, int32_t* ids, float* c1, float* c2,
+                                cudaStream_t stream);
+cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, const float* c1,
+                                 int32_t* x, int32_t* k, int B, int P, const DcvParams& prm,
+                                 cudaStream_t stream);
+// Counter-based weight generator (SplitMix64 + Irwin-Hall(4)), with an optional
+// row remap: element e of a [rows][cols] tensor goes to
+// dst[(e/cols) / blk * blk_stride + blk_off + (e/cols) % blk) * cols + e % cols]
+// (blk = 0 means contiguous).
+cudaError_t generate_launch(__nv_bfloat16* dst, uint64_t seed, int tid, int64_t start,
+                            int64_t count, float std, float mean, int64_t cols, int blk,
+                            int blk_stride, int blk_off, cudaStream_t stream);
+cudaError_t rope_table_build(float* cos_dev, float* sin_dev, int T, int hd, float theta,
+                             cudaStream_t stream);
+
+}  // namespace dcl

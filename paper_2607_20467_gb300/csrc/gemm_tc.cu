@@ -1,0 +1,601 @@
+// Persistent bf16 GEMM on the 5th-generation tensor cores (tcgen05) of sm_103a:
+//   out = A[M][K] @ W[N][K]^T   (both operands K-major, fp32 accumulation in TMEM)
+// with the step's epilogues fused (RoPE on Q/K, residual add, SwiGLU, LM-head softmax
+// partials).  These are the dense contractions of the denoise step's forward (the
+// single bidirectional pass of Sec. 3.3 step (ii)).
+//
+// Structure (one CTA per SM, 192 threads):
+//   warp 0 lane 0 : TMA producer.  Per 64-wide K block, one 128x64 A box and one
+//                   BNx64 W box (128-byte swizzle) land in a STAGES-deep smem ring,
+//                   completing a transaction-count mbarrier.
+//   warp 1        : allocates TMEM (2 x BN fp32 columns: double-buffered accumulator);
+//                   lane 0 issues tcgen05.mma (M=128, N=BN, K=16) x4 per K block and
+//                   tcgen05.commit to release smem stages / publish finished tiles.
+//   warps 2..5    : epilogue.  Warp w reads TMEM lanes 32*(w%4)..+31 (one output row
+//                   per thread) with tcgen05.ld and applies the fused epilogue while the
+//                   MMA warp accumulates the next tile into the other TMEM buffer.
+// Tiles are visited M-fastest so the CTAs working on one weight tile run together and
+// share it through L2.  Every mbarrier wait is bounded: on timeout the kernel records
+// DERR_WAIT_TIMEOUT, lets the other roles leave, waits (bounded) for its own copies
+// and MMAs in flight, frees TMEM and returns.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+
+namespace dcl {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // bf16 elements in one 128-byte swizzle row
+constexpr int A_STAGE_BYTES = BM * BK * 2;
+constexpr int NUM_THREADS = 192;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: far above any legitimate wait
+
+template <int BN>
+struct Cfg {
+  static constexpr int B_STAGE_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait for the phase of the given parity; false on timeout or abort.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(holder),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major tile written by TMA with 128-byte
+// swizzle: rows of 128 bytes, 8-row (1024-byte) swizzle atoms stacked along M/N.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+  d |= (uint64_t)1 << 16;                    // leading byte offset (unused for this layout)
+  d |= (uint64_t)(1024 >> 4) << 32;          // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;                    // descriptor version (tcgen05)
+  d |= (uint64_t)2 << 61;                    // 128-byte swizzle
+  return d;
+}
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both K-major.
+__host__ __device__ constexpr uint32_t make_idesc(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ float f32(uint32_t v) { return __uint_as_float(v); }
+
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    d4[i] = make_uint4(pack_bf16x2(v[8 * i + 0], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                       pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+}
+
+// ------------------------------------------------------------------ epilogues
+// taddr: TMEM address of (this warp's first lane, accumulator column 0); row: output row
+// of this thread; n_blk: tile column index.  All tcgen05.ld run warp-uniformly; only the
+// stores are guarded by row < M.
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk, int M, int N,
+                                              const EpiParams& ep) {
+  const int n0 = n_blk * BN;
+  const bool live = row < M;
+  if constexpr (EPI == EPI_BF16) {
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tmem_ld32(taddr + c, r);
+      tmem_ld_wait();
+      if (live && n0 + c < N) {
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+        store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)row * ep.ldo + n0 + c, v);
+      }
+    }
+  } else if constexpr (EPI == EPI_RESID_F32) {
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tmem_ld32(taddr + c, r);
+      tmem_ld_wait();
+      if (live && n0 + c < N) {
+        float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) +
+                                                (size_t)row * ep.ldo + n0 + c);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float4 o = dst[i];
+          o.x += f32(r[4 * i + 0]);
+          o.y += f32(r[4 * i + 1]);
+          o.z += f32(r[4 * i + 2]);
+          o.w += f32(r[4 * i + 3]);
+          dst[i] = o;
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_QKV_ROPE) {
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)row * ep.ldo + n0;
+    if (n0 < ep.rope_cols) {
+      const int hd = ep.head_dim, half = hd >> 1;
+      const int pos = live ? row % ep.seq_T : 0;
+      const float* cs = ep.rope_cos + (size_t)pos * half;
+      const float* sn = ep.rope_sin + (size_t)pos * half;
+#pragma unroll 1
+      for (int hb = 0; hb < BN; hb += hd) {
+#pragma unroll 1
+        for (int j0 = 0; j0 < half; j0 += 32) {
+          uint32_t lo[32], hi[32];
+          tmem_ld32(taddr + hb + j0, lo);
+          tmem_ld32(taddr + hb + half + j0, hi);
+          tmem_ld_wait();
+          if (live) {
+            float a[32], b[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float c = __ldg(cs + j0 + i), s = __ldg(sn + j0 + i);
+              const float x1 = f32(lo[i]), x2 = f32(hi[i]);
+              a[i] = x1 * c - x2 * s;
+              b[i] = x2 * c + x1 * s;
+            }
+            store_bf16x32(out + hb + j0, a);
+            store_bf16x32(out + hb + half + j0, b);
+          }
+        }
+      }
+    } else {
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        tmem_ld_wait();
+        if (live) {
+          float v[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+          store_bf16x32(out + c, v);
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    constexpr int H2 = BN / 2;
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)row * ep.ldo + n_blk * H2;
+#pragma unroll 1
+    for (int c = 0; c < H2; c += 32) {
+      uint32_t g[32], u[32];
+      tmem_ld32(taddr + c, g);
+      tmem_ld32(taddr + H2 + c, u);
+      tmem_ld_wait();
+      if (live) {
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float x = f32(g[i]);
+          v[i] = x / (1.0f + __expf(-x)) * f32(u[i]);
+        }
+        store_bf16x32(out + c, v);
+      }
+    }
+  } else if constexpr (EPI == EPI_LMHEAD) {
+    // Online softmax over this tile's columns: running max m (= top-1 value), sum of
+    // exp(z - m), argmax (lowest column on ties: columns arrive in increasing order and
+    // only a strictly larger value replaces the leader), and the second largest value.
+    float m = -INFINITY, s = 0.f, t2 = -INFINITY;
+    int id = -1;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tmem_ld32(taddr + c, r);
+      tmem_ld_wait();
+      const int col0 = n0 + c;
+      float v[32];
+      float cm = m;
+      int cid = id;
+      float c2 = t2;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        v[i] = (col0 + i < ep.vocab) ? f32(r[i]) : -INFINITY;
+        if (v[i] > cm) {
+          c2 = cm;
+          cm = v[i];
+          cid = col0 + i;
+        } else if (v[i] > c2) {
+          c2 = v[i];
+        }
+      }
+      if (cm > -INFINITY) {
+        const float mb = cm * kLog2e;
+        float acc = s * exp2f(m * kLog2e - mb);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], kLog2e, -mb));
+        s = acc;
+      }
+      m = cm;
+      id = cid;
+      t2 = c2;
+    }
+    if (live) {
+      const int nblk = (N + BN - 1) / BN;
+      float4* part = reinterpret_cast<float4*>(ep.out);
+      part[(size_t)row * nblk + n_blk] = make_float4(m, s, __int_as_float(id), t2);
+    }
+  }
+}
+
+// ------------------------------------------------------------------ the kernel
+template <int BN, int EPI>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
+                   int M, int N, int K, EpiParams ep, int* err) {
+  using C = Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+  const uint32_t sA = base;
+  const uint32_t sB = base + C::STAGES * A_STAGE_BYTES;
+  const uint32_t bars = sB + C::STAGES * C::B_STAGE_BYTES;
+  const uint32_t full0 = bars;                       // full[s]   = full0 + 8 s
+  const uint32_t empty0 = bars + 8 * C::STAGES;      // empty[s]  = empty0 + 8 s
+  const uint32_t tfull0 = bars + 16 * C::STAGES;     // tfull[ab] = tfull0 + 8 ab
+  const uint32_t tempty0 = tfull0 + 16;              // tempty[ab]
+  const uint32_t drain = tempty0 + 16;
+  const uint32_t holder = drain + 8;
+  volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_m = (M + BM - 1) / BM;
+  const int num_n = (N + BN - 1) / BN;
+  const int num_tiles = num_m * num_n;
+  const int num_kb = (K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(tfull0, 1);
+    mbar_init(tfull0 + 8, 1);
+    mbar_init(tempty0, 128);
+    mbar_init(tempty0 + 8, 128);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tma);
+    prefetch_tmap(&tmb);
+  }
+  if (warp == 1) tmem_alloc(holder, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *holder_ptr;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      long issued = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+        const int m_blk = t % num_m, n_blk = t / num_m;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full0 + 8 * stage, C::STAGE_BYTES);
+          tma_load_2d(sA + stage * A_STAGE_BYTES, &tma, kb * BK, m_blk * BM, full0 + 8 * stage);
+          tma_load_2d(sB + stage * C::B_STAGE_BYTES, &tmb, kb * BK, n_blk * BN, full0 + 8 * stage);
+          ++issued;
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+        // wait (bounded) until every copy this thread issued has landed
+        for (int s = 0; s < C::STAGES && s < issued; ++s) {
+          const long arms = (issued - 1 - s) / C::STAGES + 1;
+          volatile int no_abort = 0;
+          mbar_wait(full0 + 8 * s, (uint32_t)((arms - 1) & 1), &no_abort);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc = make_idesc(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int j = 0;
+      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++j) {
+        const int ab = j & 1;
+        const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+        if (!mbar_wait(tempty0 + 8 * ab, aph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = sw128_desc(sA + stage * A_STAGE_BYTES);
+          const uint64_t db = sw128_desc(sB + stage * C::B_STAGE_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)  // advance 16 elements = 32 bytes = 2 desc units
+            umma_bf16(d_tmem, da + 2 * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit(empty0 + 8 * stage);
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(tfull0 + 8 * ab);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+      }
+      // all MMAs issued by this thread complete before TMEM is released
+      umma_commit(drain);
+      volatile int no_abort = 0;
+      mbar_wait(drain, 0, &no_abort);
+    }
+  } else {
+    // ------------------------------------------------ epilogue warps 2..5
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    int j = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++j) {
+      const int ab = j & 1;
+      const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+      if (!mbar_wait(tfull0 + 8 * ab, aph, abort_flag)) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const int m_blk = t % num_m, n_blk = t / num_m;
+      const int row = m_blk * BM + q * 32 + lane;
+      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
+      epilogue_tile<BN, EPI>(taddr, row, n_blk, M, N, ep);
+      tc_fence_before();
+      mbar_arrive(tempty0 + 8 * ab);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+bool encode_kmajor(CUtensorMap* tm, const void* ptr, int rows, int k, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)k * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int EPI>
+cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
+  static bool attr_set = false;
+  auto kern = gemm_tc_kernel<BN, EPI>;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Cfg<BN>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  kern<<<p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
+  return cudaGetLastError();
+}
+
+double wave_efficiency(long tiles, int sms) {
+  const long waves = (tiles + sms - 1) / sms;
+  return (double)tiles / (double)(waves * sms);
+}
+
+}  // namespace
+
+int gemm_lmhead_blocks(int vocab) { return (vocab + 255) / 256; }
+
+cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N, int epi,
+                      const EpiParams& ep, int num_sms, int bn, const char** why) {
+  *why = nullptr;
+  if (M <= 0 || N <= 0 || K <= 0 || K % BK != 0 || (epi != EPI_LMHEAD && N % 32 != 0)) {
+    *why = "gemm: need M, N, K > 0, K % 64 == 0 and (except for the LM head) N % 32 == 0";
+    return cudaErrorInvalidValue;
+  }
+  if ((reinterpret_cast<uintptr_t>(A) & 15) || (reinterpret_cast<uintptr_t>(W) & 15)) {
+    *why = "gemm: operands must be 16-byte aligned";
+    return cudaErrorInvalidValue;
+  }
+  if (epi == EPI_SWIGLU || epi == EPI_LMHEAD) {
+    bn = 256;
+  } else if (bn == 0) {
+    const long m = (M + BM - 1) / BM;
+    const double e256 = wave_efficiency(m * ((N + 255) / 256), num_sms);
+    const double e128 = 0.9 * wave_efficiency(m * ((N + 127) / 128), num_sms);
+    bn = (e256 >= e128) ? 256 : 128;
+  }
+  if (bn != 128 && bn != 256) {
+    *why = "gemm: tile width must be 128 or 256";
+    return cudaErrorInvalidValue;
+  }
+  if (epi == EPI_SWIGLU && N % 256 != 0) {
+    *why = "gemm: SwiGLU needs 2*ffn a multiple of 256";
+    return cudaErrorInvalidValue;
+  }
+  if (epi == EPI_QKV_ROPE && (ep.rope_cols % bn != 0 || bn % ep.head_dim != 0 ||
+                              (ep.head_dim != 64 && ep.head_dim != 128))) {
+    *why = "gemm: RoPE epilogue needs tile-aligned q|k columns and head_dim 64/128";
+    return cudaErrorInvalidValue;
+  }
+  plan->M = M;
+  plan->N = N;
+  plan->K = K;
+  plan->bn = bn;
+  plan->epi = epi;
+  plan->ep = ep;
+  if (epi == EPI_LMHEAD) plan->ep.vocab = N;
+  if (!encode_kmajor(&plan->ta, A, M, K, BM) || !encode_kmajor(&plan->tb, W, N, K, bn)) {
+    *why = "gemm: cuTensorMapEncodeTiled failed";
+    return cudaErrorInvalidValue;
+  }
+  plan->n_tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn);
+  plan->grid = plan->n_tiles < num_sms ? plan->n_tiles : num_sms;
+  plan->smem = (bn == 256) ? Cfg<256>::SMEM : Cfg<128>::SMEM;
+  return cudaSuccess;
+}
+
+cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
+  if (p.bn == 256) {
+    switch (p.epi) {
+      case EPI_BF16: return launch_t<256, EPI_BF16>(p, err, stream);
+      case EPI_RESID_F32: return launch_t<256, EPI_RESID_F32>(p, err, stream);
+      case EPI_QKV_ROPE: return launch_t<256, EPI_QKV_ROPE>(p, err, stream);
+      case EPI_SWIGLU: return launch_t<256, EPI_SWIGLU>(p, err, stream);
+      case EPI_LMHEAD: return launch_t<256, EPI_LMHEAD>(p, err, stream);
+    }
+  } else {
+    switch (p.epi) {
+      case EPI_BF16: return launch_t<128, EPI_BF16>(p, err, stream);
+      case EPI_RESID_F32: return launch_t<128, EPI_RESID_F32>(p, err, stream);
+      case EPI_QKV_ROPE: return launch_t<128, EPI_QKV_ROPE>(p, err, stream);
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dcl

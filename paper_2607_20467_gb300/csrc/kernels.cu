@@ -1,0 +1,390 @@
+// Bandwidth- and latency-bound kernels of the denoise step:
+//   embed_remask   Eq. remasking (draft invalidation, Sec. 3.3 step (i)) fused with the
+//                  embedding gather that starts the forward
+//   rmsnorm        fp32 residual stream -> bf16 GEMM operand
+//   lmhead_combine per-row merge of the LM-head epilogue partials into the top-1 id,
+//                  top-1 probability and top-2 probability of Eq. 2's softmax
+//   dcv_commit     Eq. compute_k + commit + Eq. draft_update + advance (Sec. 3.3 steps
+//                  (iii)-(iv), Algorithm 1), one warp per sequence
+//   accept_*       the same acceptance on caller-provided bf16 logits
+//   generate       counter-based synthetic weight generator
+#include <math.h>
+
+#include "common.cuh"
+
+namespace dcl {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+// ------------------------------------------------------------------ embedding + remask
+__global__ void embed_remask_kernel(int32_t* __restrict__ x, const int32_t* __restrict__ p, int T,
+                                    int window, int mask_id, int vocab,
+                                    const __nv_bfloat16* __restrict__ embed, int d,
+                                    float* __restrict__ h, int* err) {
+  const int row = blockIdx.x;
+  const int b = row / T, t = row % T;
+  __shared__ int tok_s;
+  if (threadIdx.x == 0) {
+    const int pb = p[b];
+    int tok = x[row];
+    if (t >= pb && t - pb < window) {  // x_{p+i} <- MASK for i in [0, L)
+      tok = mask_id;
+      x[row] = mask_id;
+    }
+    if (tok < 0 || tok >= vocab) {
+      report_error(err, DERR_TOKEN_RANGE);
+      tok = mask_id;
+    }
+    tok_s = tok;
+  }
+  __syncthreads();
+  const uint4* src = reinterpret_cast<const uint4*>(embed + (size_t)tok_s * d);
+  float4* dst = reinterpret_cast<float4*>(h + (size_t)row * d);
+  for (int i = threadIdx.x; i < d / 8; i += blockDim.x) {
+    const uint4 v = __ldg(src + i);
+    dst[2 * i] = make_float4(bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y));
+    dst[2 * i + 1] = make_float4(bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w));
+  }
+}
+
+// ------------------------------------------------------------------ RMSNorm
+template <int THREADS>
+__global__ void __launch_bounds__(THREADS) rmsnorm_kernel(const float* __restrict__ x,
+                                                          const __nv_bfloat16* __restrict__ gain,
+                                                          __nv_bfloat16* __restrict__ y, int d,
+                                                          float eps, int rows_per_seq,
+                                                          int seq_stride, int row_offset) {
+  const int r = blockIdx.x;
+  const int in_row = (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
+  const int n4 = d / 4;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < n4; i += THREADS) {
+    const float4 v = xr[i];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  __shared__ float red[THREADS / 32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(kFull, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < THREADS / 32 ? red[threadIdx.x] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float inv = rsqrtf(red[0] / (float)d + eps);
+  const uint2* g2 = reinterpret_cast<const uint2*>(gain);
+  uint2* y2 = reinterpret_cast<uint2*>(y + (size_t)r * d);
+  for (int i = threadIdx.x; i < n4; i += THREADS) {
+    const float4 v = xr[i];
+    const uint2 g = __ldg(g2 + i);
+    y2[i] = make_uint2(pack_bf16x2(v.x * inv * bf16_lo(g.x), v.y * inv * bf16_hi(g.x)),
+                       pack_bf16x2(v.z * inv * bf16_lo(g.y), v.w * inv * bf16_hi(g.y)));
+  }
+}
+
+// ------------------------------------------------------------------ softmax partial merge
+// A partial is {max, sum exp(z - max), argmax id, second largest z} over some columns.
+struct Part {
+  float m, s, t2;
+  int id;
+};
+
+__device__ __forceinline__ void merge(Part& a, const Part& b) {
+  if (b.m == -INFINITY) return;
+  if (a.m == -INFINITY) {
+    a = b;
+    return;
+  }
+  const float m = fmaxf(a.m, b.m);
+  const float s = a.s * exp2f((a.m - m) * kLog2e) + b.s * exp2f((b.m - m) * kLog2e);
+  if (b.m > a.m || (b.m == a.m && b.id < a.id)) {
+    a.t2 = fmaxf(b.t2, a.m);
+    a.id = b.id;
+  } else {
+    a.t2 = fmaxf(a.t2, b.m);
+  }
+  a.m = m;
+  a.s = s;
+}
+
+__device__ __forceinline__ Part shfl_part(const Part& a, int off) {
+  Part b;
+  b.m = __shfl_xor_sync(kFull, a.m, off);
+  b.s = __shfl_xor_sync(kFull, a.s, off);
+  b.t2 = __shfl_xor_sync(kFull, a.t2, off);
+  b.id = __shfl_xor_sync(kFull, a.id, off);
+  return b;
+}
+
+__device__ __forceinline__ void write_conf(const Part& a, int32_t* top1, float* p1, float* p2, int r) {
+  top1[r] = a.id;
+  const float inv = 1.0f / a.s;  // p1 = exp(max - max) / sum
+  p1[r] = inv;
+  p2[r] = a.t2 == -INFINITY ? 0.f : exp2f((a.t2 - a.m) * kLog2e) * inv;
+}
+
+__global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows, int nblk,
+                                      int32_t* __restrict__ top1, float* __restrict__ p1,
+                                      float* __restrict__ p2) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
+  for (int i = lane; i < nblk; i += 32) {
+    const float4 v = part[(size_t)row * nblk + i];
+    merge(a, Part{v.x, v.y, v.w, __float_as_int(v.z)});
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) merge(a, shfl_part(a, o));
+  if (lane == 0) write_conf(a, top1, p1, p2, row);
+}
+
+// ------------------------------------------------------------------ DCV on one sequence
+// xrow / ids / c indexed by absolute position; window [pb, pb + min(L, T - pb)).
+// Runs on one full warp.  Returns K (valid on every lane).
+__device__ int dcv_row(int32_t* xrow, const int32_t* ids, const float* c, int pb, int T,
+                       const DcvParams& prm) {
+  const int lane = threadIdx.x & 31;
+  const int w_eff = min(prm.window, T - pb);
+  // Eq. compute_k: K = sum_i prod_{j<=i} 1(c_{p+j} > tau_commit) = length of the leading
+  // run of passing positions; each 32-wide chunk is one ballot.
+  int K = 0;
+  for (int base = 0; base < w_eff; base += 32) {
+    const int i = base + lane;
+    const bool ok = i < w_eff && c[pb + i] > prm.tau_commit;
+    const unsigned bal = __ballot_sync(kFull, ok);
+    if (bal == kFull) {
+      K += 32;
+      continue;
+    }
+    K += __ffs(~bal) - 1;
+    break;
+  }
+  K = min(max(K, prm.min_commit), w_eff);
+  for (int i = lane; i < K; i += 32) xrow[pb + i] = ids[pb + i];  // commit x[p:p+K]
+  // Eq. draft_update over the future region i >= p + L (p before the advance)
+  const int lo = pb + prm.window;
+  if (!prm.contiguous_drafts) {
+    for (int i = lo + lane; i < T; i += 32)
+      if (c[i] > prm.tau_draft) xrow[i] = ids[i];
+  } else {  // App. E variant: only the unbroken chain starting at p + L
+    for (int base = lo; base < T; base += 32) {
+      const int i = base + lane;
+      const bool ok = i < T && c[i] > prm.tau_draft;
+      const unsigned bal = __ballot_sync(kFull, ok);
+      const int run = (bal == kFull) ? 32 : __ffs(~bal) - 1;
+      if (lane < run) xrow[i] = ids[i];
+      if (run < 32) break;
+    }
+  }
+  return K;
+}
+
+__global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__ p,
+                                  int32_t* __restrict__ k_out, int32_t* __restrict__ steps,
+                                  const int32_t* __restrict__ ids, const float* __restrict__ c,
+                                  int N, int M, DcvParams prm, int32_t* done_count) {
+  const int b = blockIdx.x;
+  const int T = N + M;
+  const int pb = p[b];
+  if (pb >= T) {
+    if (threadIdx.x == 0) k_out[b] = 0;
+    return;
+  }
+  // shift the [M]-sized generation arrays so they are indexed by absolute position
+  const int K = dcv_row(x + (size_t)b * T, ids + (size_t)b * M - N, c + (size_t)b * M - N, pb, T, prm);
+  if (threadIdx.x == 0) {
+    k_out[b] = K;
+    p[b] = pb + K;
+    steps[b] += 1;
+    if (pb + K >= T) atomicAdd(done_count, 1);
+  }
+}
+
+// ------------------------------------------------------------------ block acceptance
+template <int THREADS>
+__global__ void __launch_bounds__(THREADS) accept_stats_kernel(
+    const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int P, int V,
+    int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2) {
+  const int pos = blockIdx.x;  // b * P + i
+  const int b = pos / P, i = pos % P;
+  if (i < committed[b]) return;  // committed positions are never read
+  const __nv_bfloat16* row = logits + (size_t)pos * V;
+  // per-thread online (max, sum, argmax, second) over a strided slice of the row
+  Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
+  auto take = [&](float v, int col) {
+    if (v > a.m) {
+      a.s = a.s * exp2f((a.m - v) * kLog2e) + 1.f;
+      a.t2 = a.m;
+      a.m = v;
+      a.id = col;
+    } else if (a.m != -INFINITY) {
+      if (v > a.t2) a.t2 = v;
+      a.s += exp2f((v - a.m) * kLog2e);
+    }
+  };
+  const bool vec = ((reinterpret_cast<uintptr_t>(row) & 15) == 0);
+  int done = 0;
+  if (vec) {
+    const uint4* r4 = reinterpret_cast<const uint4*>(row);
+    const int n8 = V / 8;
+    for (int j = threadIdx.x; j < n8; j += THREADS) {
+      const uint4 v = __ldcs(r4 + j);  // streamed once: do not keep in L2
+      const int col = j * 8;
+      take(bf16_lo(v.x), col + 0);
+      take(bf16_hi(v.x), col + 1);
+      take(bf16_lo(v.y), col + 2);
+      take(bf16_hi(v.y), col + 3);
+      take(bf16_lo(v.z), col + 4);
+      take(bf16_hi(v.z), col + 5);
+      take(bf16_lo(v.w), col + 6);
+      take(bf16_hi(v.w), col + 7);
+    }
+    done = n8 * 8;
+  }
+  const unsigned short* r2 = reinterpret_cast<const unsigned short*>(row);
+  for (int j = done + threadIdx.x; j < V; j += THREADS) take(__uint_as_float((uint32_t)r2[j] << 16), j);
+  // a thread's columns arrive in increasing order, so its argmax is its lowest maximal
+  // column; merge() breaks ties between threads by the lower id
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) merge(a, shfl_part(a, o));
+  __shared__ Part red[THREADS / 32];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = a;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    Part v = threadIdx.x < THREADS / 32 ? red[threadIdx.x] : Part{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) merge(v, shfl_part(v, o));
+    if (threadIdx.x == 0) write_conf(v, ids, c1, c2, pos);
+  }
+}
+
+__global__ void accept_commit_kernel(const int32_t* __restrict__ committed,
+                                     const int32_t* __restrict__ ids, const float* __restrict__ c1,
+                                     int32_t* __restrict__ x, int32_t* __restrict__ k, int P,
+                                     DcvParams prm) {
+  const int b = blockIdx.x;
+  const int pb = committed[b];
+  if (pb >= P || pb < 0) {
+    if (threadIdx.x == 0) k[b] = 0;
+    return;
+  }
+  const int K = dcv_row(x + (size_t)b * P, ids + (size_t)b * P, c1 + (size_t)b * P, pb, P, prm);
+  if (threadIdx.x == 0) k[b] = K;
+}
+
+// ------------------------------------------------------------------ weight generator
+__device__ __forceinline__ uint64_t splitmix64(uint64_t z) {
+  z += 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void generate_kernel(__nv_bfloat16* __restrict__ dst, uint64_t seed, int tid,
+                                int64_t start, int64_t count, float scale, float mean,
+                                int64_t cols, int blk, int blk_stride, int blk_off) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count; e += stride) {
+    const uint64_t idx = (uint64_t)(start + e);
+    const uint64_t h = splitmix64((seed << 48) | ((uint64_t)tid << 32) | idx);
+    const int s = (int)(h & 0xFFFF) + (int)((h >> 16) & 0xFFFF) + (int)((h >> 32) & 0xFFFF) +
+                  (int)(h >> 48);
+    float w = __fmul_rn((float)(s - 131070), scale);  // no fused multiply-add: exact IEEE ops
+    if (mean != 0.f) w = __fadd_rn(w, mean);
+    int64_t o = e;
+    if (blk > 0) {
+      const int64_t r = (int64_t)idx / cols, cidx = (int64_t)idx % cols;
+      o = ((r / blk) * blk_stride + blk_off + r % blk) * cols + cidx;
+    }
+    dst[o] = __float2bfloat16_rn(w);
+  }
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ launchers
+cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
+                                int mask_id, int vocab, const __nv_bfloat16* embed, int d, float* h,
+                                int* err, cudaStream_t stream) {
+  if (d % 8) return cudaErrorInvalidValue;
+  embed_remask_kernel<<<batch * T, 128, 0, stream>>>(x, p, T, window, mask_id, vocab, embed, d, h, err);
+  return cudaGetLastError();
+}
+
+cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows, int d,
+                           float eps, int rows_per_seq, int seq_stride, int row_offset,
+                           cudaStream_t stream) {
+  if (d % 4 || rows <= 0) return cudaErrorInvalidValue;
+  rmsnorm_kernel<256><<<rows, 256, 0, stream>>>(x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
+  return cudaGetLastError();
+}
+
+cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
+                                  float* p2, cudaStream_t stream) {
+  const int threads = 256;
+  const int blocks = (rows * 32 + threads - 1) / threads;
+  lmhead_combine_kernel<<<blocks, threads, 0, stream>>>(part, rows, nblk, top1, p1, p2);
+  return cudaGetLastError();
+}
+
+cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
+                              const int32_t* ids, const float* c, int batch, int N, int M,
+                              const DcvParams& prm, int32_t* done_count, cudaStream_t stream) {
+  dcv_commit_kernel<<<batch, 32, 0, stream>>>(x, p, k_out, steps, ids, c, N, M, prm, done_count);
+  return cudaGetLastError();
+}
+
+cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
+                                int V, int32_t* ids, float* c1, float* c2, cudaStream_t stream) {
+  accept_stats_kernel<512><<<B * P, 512, 0, stream>>>(logits, committed, P, V, ids, c1, c2);
+  return cudaGetLastError();
+}
+
+cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, const float* c1,
+                                 int32_t* x, int32_t* k, int B, int P, const DcvParams& prm,
+                                 cudaStream_t stream) {
+  accept_commit_kernel<<<B, 32, 0, stream>>>(committed, ids, c1, x, k, P, prm);
+  return cudaGetLastError();
+}
+
+cudaError_t generate_launch(__nv_bfloat16* dst, uint64_t seed, int tid, int64_t start, int64_t count,
+                            float std, float mean, int64_t cols, int blk, int blk_stride, int blk_off,
+                            cudaStream_t stream) {
+  if (count <= 0) return cudaSuccess;
+  const double sigma4 = sqrt(4.0 * (65536.0 * 65536.0 - 1.0) / 12.0);
+  const float scale = (float)((double)std / sigma4);
+  int64_t blocks = (count + 255) / 256;
+  if (blocks > 152 * 32) blocks = 152 * 32;
+  generate_kernel<<<(int)blocks, 256, 0, stream>>>(dst, seed, tid, start, count, scale, mean, cols, blk,
+                                                   blk_stride, blk_off);
+  return cudaGetLastError();
+}
+
+cudaError_t rope_table_build(float* cos_dev, float* sin_dev, int T, int hd, float theta,
+                             cudaStream_t stream) {
+  const int half = hd / 2;
+  float* hc = nullptr;
+  cudaError_t e = cudaMallocHost(&hc, sizeof(float) * 2 * (size_t)T * half);
+  if (e != cudaSuccess) return e;
+  for (int t = 0; t < T; ++t)
+    for (int j = 0; j < half; ++j) {
+      const double ang = (double)t * pow((double)theta, -2.0 * j / hd);
+      hc[(size_t)t * half + j] = (float)cos(ang);
+      hc[(size_t)T * half + (size_t)t * half + j] = (float)sin(ang);
+    }
+  e = cudaMemcpyAsync(cos_dev, hc, sizeof(float) * (size_t)T * half, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(sin_dev, hc + (size_t)T * half, sizeof(float) * (size_t)T * half,
+                        cudaMemcpyHostToDevice, stream);
+  cudaError_t s = cudaStreamSynchronize(stream);
+  cudaFreeHost(hc);
+  return e != cudaSuccess ? e : s;
+}
+
+}  // namespace dcl

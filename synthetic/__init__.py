@@ -118,7 +118,8 @@ def weight_values(seed: int, tid: int, start: int, count: int, std: float,
     m16 = np.uint64(0xFFFF)
     s = ((h & m16) + ((h >> np.uint64(16)) & m16) + ((h >> np.uint64(32)) & m16)
          + (h >> np.uint64(48))).astype(np.int64)
-    w = (s - GEN_MEAN4).astype(np.float32) * np.float32(std / GEN_SIGMA4)
+    std32 = float(np.float32(std))        # the C ABI receives std as a float
+    w = (s - GEN_MEAN4).astype(np.float32) * np.float32(std32 / GEN_SIGMA4)
     if mean != 0.0:
         w = w + np.float32(mean)
     return round_bf16(w)
@@ -163,8 +164,10 @@ def model_weights(shape: ModelShape, seed: int, std: float = 0.02,
         if kind in TensorKind.NORMS:
             v = weight_values(seed, tensor_id(kind, layer), 0, n, norm_gain_std, 1.0)
         else:
-            s = std * (lm_head_scale if kind == TensorKind.LM_HEAD else 1.0)
-            v = weight_values(seed, tensor_id(kind, layer), 0, n, s)
+            s = np.float32(std)
+            if kind == TensorKind.LM_HEAD:
+                s = s * np.float32(lm_head_scale)   # fp32 product, as on the device
+            v = weight_values(seed, tensor_id(kind, layer), 0, n, float(s))
         return v.reshape(dims[kind])
 
     names = {TensorKind.ATTN_NORM: "attn_norm", TensorKind.WQ: "wq", TensorKind.WK: "wk",

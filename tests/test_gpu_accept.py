@@ -1,0 +1,77 @@
+"""Acceptance pass from bf16 logits (dcl_accept) against the oracle: bit-exact K,
+committed ids and drafts on the same logits.
+
+Both sides take each decision ``c > tau`` in float32, but they reach c by different
+roundings (fp32 sum on the GPU, fp64 in the oracle), so positions whose oracle
+confidence lies within 1e-4 of a threshold have their top logit nudged until none
+does; the integer outputs are then exact by construction.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synthetic as syn
+from oracle import accept, decode, model
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ops():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2607_20467_gb300 as dcl
+    ctx = dcl.Context(None, 1, 1)
+    yield ctx
+    ctx.close()
+
+
+def _guarded(seed, B, P, V, taus):
+    d = syn.accept_inputs(seed, B, P, V, V - 1)
+    bits = d["logits_bf16"]
+    for _ in range(50):
+        z = syn.bf16_to_f32(bits).astype(np.float64)
+        bad = []
+        for b in range(B):
+            for i in range(int(d["committed"][b]), P):
+                _, c1, _ = model.confidence(z[b, i][None])
+                if min(abs(c1[0] - t) for t in taus) < 1e-4:
+                    bad.append((b, i))
+        if not bad:
+            return d, syn.bf16_to_f32(bits)
+        for b, i in bad:  # raise the top logit by a few bf16 steps
+            top = int(np.argmax(z[b, i]))
+            bits[b, i, top] = syn.bf16_bits(np.array([z[b, i, top] + 0.25], np.float32))[0]
+    raise RuntimeError("could not clear the guard band")
+
+
+@pytest.mark.parametrize("B,P,V,L,contig", [(8, 32, 4096, 16, 0), (16, 32, 1000, 32, 0), (6, 40, 3001, 7, 1),
+                                            (64, 32, 126464, 16, 0), (64, 32, 126464, 32, 1)])
+def test_accept_bit_exact(ops, B, P, V, L, contig):
+    import paper_2607_20467_gb300 as dcl
+    tc, td = 0.7, 0.9
+    d, z = _guarded(B * 131 + P + L, B, P, V, (tc, td))
+    logits = torch.from_numpy(d["logits_bf16"].view(np.int16)).cuda().view(torch.bfloat16)
+    committed = torch.from_numpy(d["committed"]).cuda()
+    x = torch.from_numpy(d["x"].copy()).cuda()
+    k = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    cfg = dcl.decode_config(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P,
+                            contiguous_drafts=contig)
+    ops.accept(logits, committed, x, cfg, k)
+    torch.cuda.synchronize()
+    ocfg = decode.DecodeConfig(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P,
+                               contiguous_drafts=bool(contig))
+    K, x_out, _, _, _ = accept.accept(z, d["committed"], d["x"], ocfg, L)
+    assert (k.cpu().numpy() == K).all()
+    assert (x.cpu().numpy() == x_out).all()
+
+
+def test_accept_rejects_bad_arguments(ops):
+    import paper_2607_20467_gb300 as dcl
+    cfg = dcl.decode_config(gen_len=32)
+    t = torch.zeros(4, dtype=torch.int32, device="cuda")
+    st = dcl.lib().dcl_accept(ops.ptr, None, 1, 32, 100, t.data_ptr(), t.data_ptr(), cfg, t.data_ptr())
+    assert st == dcl.DCL_ERR_INVALID_ARG
+    st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 5000, 100, t.data_ptr(), t.data_ptr(), cfg,
+                              t.data_ptr())
+    assert st == dcl.DCL_ERR_INVALID_ARG

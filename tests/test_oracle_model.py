@@ -141,10 +141,21 @@ def test_silu_matches_library():
 
 # --------------------------------------------------------------- whole forward
 
-def _torch_forward(shape, w, tokens):
+def test_to_bf16_matches_torch_rounding():
+    rng = np.random.default_rng(9)
+    x = np.concatenate([rng.normal(0, 1, 10000), rng.normal(0, 1e4, 1000),
+                        # exact halfway cases between bf16 neighbours (ties to even)
+                        (np.arange(1, 200, dtype=np.float64) * 2 + 1) * 2 ** -8 + 1.0])
+    ref = torch.tensor(x).float().bfloat16().double().numpy()
+    assert (model.to_bf16(x) == ref).all()
+
+
+def _torch_forward(shape, w, tokens, bf16=False):
     """Independent fp64 restatement with torch library ops (F.linear, F.rms_norm, SDPA, F.silu)
-    and RoPE as a complex multiplication."""
+    and RoPE as a complex multiplication; bf16=True casts matrix-product operands with
+    torch's own bf16 conversion at the points a bf16 model stores them."""
     t = lambda a: torch.tensor(np.asarray(a, np.float64))
+    c = (lambda a: a.float().bfloat16().double()) if bf16 else (lambda a: a)
     T = len(tokens)
     H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     h = t(w["embed"])[torch.tensor(tokens, dtype=torch.long)]
@@ -156,17 +167,17 @@ def _torch_forward(shape, w, tokens):
         zc = torch.complex(x[..., :hd // 2], x[..., hd // 2:]) * rot[:, None, :]
         return torch.cat([zc.real, zc.imag], dim=-1)
     for lw in w["layers"]:
-        xn = F.rms_norm(h, (shape.d_model,), t(lw["attn_norm"]), eps=shape.rms_eps)
-        q = rope(F.linear(xn, t(lw["wq"])).view(T, H, hd))
-        k = rope(F.linear(xn, t(lw["wk"])).view(T, G, hd)).repeat_interleave(H // G, dim=1)
-        v = F.linear(xn, t(lw["wv"])).view(T, G, hd).repeat_interleave(H // G, dim=1)
+        xn = c(F.rms_norm(h, (shape.d_model,), t(lw["attn_norm"]), eps=shape.rms_eps))
+        q = c(rope(F.linear(xn, t(lw["wq"])).view(T, H, hd)))
+        k = c(rope(F.linear(xn, t(lw["wk"])).view(T, G, hd))).repeat_interleave(H // G, dim=1)
+        v = c(F.linear(xn, t(lw["wv"])).view(T, G, hd)).repeat_interleave(H // G, dim=1)
         a = F.scaled_dot_product_attention(q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1),
                                            is_causal=False).transpose(0, 1).reshape(T, H * hd)
-        h = h + F.linear(a, t(lw["wo"]))
-        xn = F.rms_norm(h, (shape.d_model,), t(lw["mlp_norm"]), eps=shape.rms_eps)
-        h = h + F.linear(F.silu(F.linear(xn, t(lw["w_gate"]))) * F.linear(xn, t(lw["w_up"])),
+        h = h + F.linear(c(a), t(lw["wo"]))
+        xn = c(F.rms_norm(h, (shape.d_model,), t(lw["mlp_norm"]), eps=shape.rms_eps))
+        h = h + F.linear(c(F.silu(F.linear(xn, t(lw["w_gate"]))) * F.linear(xn, t(lw["w_up"]))),
                          t(lw["w_down"]))
-    h = F.rms_norm(h, (shape.d_model,), t(w["final_norm"]), eps=shape.rms_eps)
+    h = c(F.rms_norm(h, (shape.d_model,), t(w["final_norm"]), eps=shape.rms_eps))
     return F.linear(h, t(w["lm_head"])).numpy()
 
 
@@ -178,6 +189,30 @@ def test_tiny_forward_matches_torch_restatement():
     z = model.logits(w, model.forward_hidden(TINY, w, tokens))
     ref = _torch_forward(TINY, w, tokens)
     assert np.abs(z - ref).max() <= 1e-9 * np.abs(ref).max()
+
+
+def test_tiny_forward_bf16_operands_matches_torch_restatement():
+    w = syn.model_weights(TINY, 0, lm_head_scale=40.0, norm_gain_std=0.1)
+    tokens = np.concatenate([syn.prompt_ids(5, 1, 32, TINY.mask_id)[0],
+                             np.full(64, TINY.mask_id, np.int32)])
+    z = model.logits(w, model.forward_hidden(TINY, w, tokens, bf16_operands=True))
+    ref = _torch_forward(TINY, w, tokens, bf16=True)
+    # identical rounding points; only fp64 summation order differs (it may move a value
+    # across a bf16 rounding boundary, so allow a few bf16 ulps in rare elements)
+    assert np.abs(z - ref).max() <= 1e-4 * np.abs(ref).max()
+    # and the rounding is real: the pure forward differs
+    z0 = model.logits(w, model.forward_hidden(TINY, w, tokens))
+    assert np.abs(z0 - z).max() > 1e-3
+
+
+def test_upto_layer_returns_residual_stream():
+    w = syn.model_weights(TINY, 1)
+    tokens = syn.prompt_ids(2, 1, 20, TINY.mask_id)[0]
+    h_emb = model.forward_hidden(TINY, w, tokens, upto_layer=-1)
+    assert np.array_equal(h_emb, np.asarray(w["embed"], np.float64)[tokens])
+    h0 = model.forward_hidden(TINY, w, tokens, upto_layer=0)
+    ang = model.rope_angles(20, TINY.head_dim, TINY.rope_theta)
+    assert np.array_equal(h0, model.block(TINY, w["layers"][0], h_emb, ang))
 
 
 def test_gqa_forward_matches_torch_restatement():
