@@ -185,6 +185,30 @@ dcl_status dcl_accept(dcl_ctx* ctx, const void* logits_dev, int32_t B, int32_t P
                       const int32_t* committed_dev, int32_t* x_dev, const dcl_decode_config* cfg,
                       int32_t* k_dev);
 
+/* ---- allocation-free acceptance ---- */
+
+/* Largest B*P that dcl_accept_noalloc accepts: the size of its static scratch. */
+#define DCL_NOALLOC_MAX_POSITIONS 32768
+
+/* The paper has no counterpart of this call; it exists for callers that cannot allocate
+ * device memory - code running inside another framework's memory pool, or under a
+ * real-time budget where cudaMalloc may stall or is forbidden - and so cannot create a
+ * dcl_ctx either.  It computes exactly what dcl_accept computes (same arguments, same
+ * kernels) on `cuda_stream` (NULL = the legacy default stream), without a context and
+ * without any allocation: its scratch (12 bytes per position) is a file-scope device
+ * array of DCL_NOALLOC_MAX_POSITIONS positions (384 KB) that every GPU loading this
+ * library holds until the process exits.
+ *   - B*P above DCL_NOALLOC_MAX_POSITIONS is rejected with DCL_ERR_INVALID_ARG.
+ *   - The first call on a device looks up the array's device address (once per device,
+ *     with that device current); make that first call before any stream capture.
+ *   - All calls share the one array and it keeps the last call's contents; a call
+ *     writes every scratch entry it reads, so nothing needs clearing, but calls whose
+ *     work overlaps on the GPU (e.g. on two streams) race on it.
+ *   - Errors: INVALID_ARG, CUDA; the message is available from dcl_last_error(NULL). */
+dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int32_t P, int32_t V,
+                              const int32_t* committed_dev, int32_t* x_dev,
+                              const dcl_decode_config* cfg, int32_t* k_dev, void* cuda_stream);
+
 /* ---- single-kernel entry points (the kernels of the step, for parity tests) ---- */
 
 /* y = x / sqrt(mean(x^2) + eps) * gain.  x_dev float [rows][d], gain_dev bf16 [d],

@@ -73,6 +73,7 @@ SIGNATURES = {
     "dcl_forward_debug": (_I, [_P, _P, _P, _P, _P]),
     "dcl_debug_hidden": (_I, [_P, _I, _P]),
     "dcl_accept": (_I, [_P, _P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P]),
+    "dcl_accept_noalloc": (_I, [_P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P, _P]),
     "dcl_op_rmsnorm": (_I, [_P, _P, _P, _P, _I, _I, _F]),
     "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I]),
     "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I]),

@@ -115,4 +115,7 @@ cudaError_t generate_launch(__nv_bfloat16* dst, uint64_t seed, int tid, int64_t 
 cudaError_t rope_table_build(float* cos_dev, float* sin_dev, int T, int hd, float theta,
                              cudaStream_t stream);
 
+// Message returned by dcl_last_error(NULL) for calls that have no context.
+void set_thread_error(const char* msg);
+
 }  // namespace dcl

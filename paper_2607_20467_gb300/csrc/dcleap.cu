@@ -349,6 +349,8 @@ dcl_status reset_done_count(dcl_ctx* c, const int32_t* p_host) {
 
 }  // namespace
 
+void dcl::set_thread_error(const char* msg) { g_create_error = msg ? msg : ""; }
+
 // ==================================================================== C ABI
 extern "C" {
 
