@@ -45,6 +45,10 @@ WORKLOADS = {
     # the same architecture, long generation: prompt 512, gen 1024, batch 1
     "llada8b-long": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
                          seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
+    # the LLaDA-8B shape cut to 2 layers (~3 GB on the device): the same GEMM, attention and
+    # LM-head launches as the full model, small enough for ncu captures with replay
+    "llada8b-2l": dict(shape="llada8b-2l", batch=1, n_prompt=256, gen=256, block=32, window=128,
+                       seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
     # 2-layer test model (latency-bound)
     "tiny": dict(shape="tiny", batch=1, n_prompt=32, gen=64, block=32, window=32,
                  seed=0, lm_scale=40.0, tau_c=0.70, tau_d=0.98),
@@ -108,7 +112,7 @@ class ClockSampler:
         try:
             self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                   "-lms", "200"]
+                   "-lms", "100"]
             if self.uuid:
                 cmd += ["-i", self.uuid]
             self.proc = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
@@ -433,19 +437,26 @@ def run_ours(args):
 
 
 def _traffic_from_profiles(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if present."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    """DRAM bytes per launch of `kernel` from the committed ncu summary (profiles/traffic.txt),
+    or None when the GEMM source has changed since the counters were taken."""
+    import hashlib
     try:
-        with open(path) as f:
-            return json.load(f).get(kernel)
+        with open(os.path.join(ROOT, "paper_2607_20467_gb300", "csrc", "gemm_tc.cu"), "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()[:16]
+        with open(os.path.join(ROOT, "profiles", "traffic.txt")) as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) >= 3 and parts[0] == kernel and not line.startswith("#"):
+                    return int(parts[1]) if parts[2] == sha else None
     except (OSError, ValueError):
-        return None
+        pass
+    return None
 
 
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="llada8b")

@@ -58,6 +58,8 @@ SHAPES = {
     "tiny": ModelShape(2, 256, 4, 4, 64, 1024, 4096, 4095, 10000.0),
     # LLaDA-8B-shaped: 32 layers, d 4096, 32x128 MHA, ffn 12288, vocab 126464
     "llada8b": ModelShape(32, 4096, 32, 32, 128, 12288, 126464, 126463, 500000.0),
+    # the LLaDA-8B shape with 2 layers (profiling captures of the same kernels)
+    "llada8b-2l": ModelShape(2, 4096, 32, 32, 128, 12288, 126464, 126463, 500000.0),
     # Dream-7B-shaped: 28 layers, d 3584, 28 query / 4 kv heads x128, ffn 18944, vocab 152064
     "dream7b": ModelShape(28, 3584, 28, 4, 128, 18944, 152064, 152063, 1000000.0),
 }
