@@ -216,11 +216,17 @@ dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int32_t P, int3
 dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev, void* y_dev,
                           int32_t rows, int32_t d, float eps);
 
-/* out = a @ w^T on the tcgen05 tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];
+/* Tile choices of the GEMM entry points: 0 lets the library choose (as in the step),
+ * 128 / 256 force a one-CTA 128 x 128 / 128 x 256 tile, DCL_TILE_PAIR a CTA-pair
+ * (tcgen05 cta_group::2) 256 x 256 tile. */
+#define DCL_TILE_PAIR 2
+
+/* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05
+ * tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];
  * mode 0: out bf16 [M][N]; mode 1: out float [M][N] += a @ w^T (residual add).
- * K, N multiples of 64.  Async. */
+ * K a multiple of 64, N of 32.  Synchronises (reports device-side faults). */
 dcl_status dcl_op_linear(dcl_ctx* ctx, const void* a_dev, const void* w_dev, void* out_dev,
-                         int32_t M, int32_t N, int32_t K, int32_t mode);
+                         int32_t M, int32_t N, int32_t K, int32_t mode, int32_t tile);
 
 /* Non-causal attention softmax(q k^T / sqrt(hd)) v over all T positions of each of
  * `batch` sequences.  qkv_dev bf16 [batch*T][(H+2G)*hd] (q | k | v column blocks, RoPE
@@ -228,13 +234,14 @@ dcl_status dcl_op_linear(dcl_ctx* ctx, const void* a_dev, const void* w_dev, voi
 dcl_status dcl_op_attention(dcl_ctx* ctx, const void* qkv_dev, void* out_dev, int32_t batch,
                             int32_t T, int32_t H, int32_t G, int32_t hd);
 
-/* LM head + softmax confidence fused: for each row r of x_dev (bf16 [R][d]),
- * z = x_r @ w^T (w_dev bf16 [V][d]); top1_dev[r] = argmax (lowest index on ties),
- * p1_dev[r] = max softmax(z), p2_dev[r] = second largest probability.  Logits never
- * reach memory.  d a multiple of 64.  Async. */
+/* LM head + softmax confidence fused (Eq. 2; top-1 of Eq. threshold_pd; top-2 of
+ * Sec. 2.2): for each row r of x_dev (bf16 [R][d]), z = x_r @ w^T (w_dev bf16 [V][d]);
+ * top1_dev[r] = argmax (lowest index on ties), p1_dev[r] = max softmax(z), p2_dev[r] =
+ * second largest probability.  Logits never reach memory.  d a multiple of 64;
+ * tile 0, 256 or DCL_TILE_PAIR.  Synchronises. */
 dcl_status dcl_op_lmhead_top2(dcl_ctx* ctx, const void* x_dev, const void* w_dev, int32_t R,
                               int32_t V, int32_t d, int32_t* top1_dev, float* p1_dev,
-                              float* p2_dev);
+                              float* p2_dev, int32_t tile);
 
 /* Fill dst_dev (bf16, count elements) from the weight generator of
  * dcl_init_random_weights for tensor id `tid` starting at element `start`.  Async. */

@@ -20,6 +20,7 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libdcleap.so")
 
+DCL_TILE_PAIR = 2
 DCL_OK, DCL_ERR_INVALID_ARG, DCL_ERR_STATE, DCL_ERR_OOM, DCL_ERR_CUDA, DCL_ERR_TIMEOUT, \
     DCL_ERR_UNSUPPORTED = range(7)
 STATUS_NAMES = ["OK", "INVALID_ARG", "STATE", "OOM", "CUDA", "TIMEOUT", "UNSUPPORTED"]
@@ -75,9 +76,9 @@ SIGNATURES = {
     "dcl_accept": (_I, [_P, _P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P]),
     "dcl_accept_noalloc": (_I, [_P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P, _P]),
     "dcl_op_rmsnorm": (_I, [_P, _P, _P, _P, _I, _I, _F]),
-    "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I]),
+    "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I]),
     "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I]),
-    "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P]),
+    "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _I]),
     "dcl_op_generate": (_I, [_P, _P, ctypes.c_uint64, _I, ctypes.c_int64, ctypes.c_int64, _F, _F]),
     "dcl_set_profiling": (_I, [_P, _I]),
     "dcl_profile_last_step": (_I, [_P, _P, _P, _I, _P]),
@@ -254,19 +255,19 @@ class Context:
         rows, d = x.shape
         self._check(self._L.dcl_op_rmsnorm(self.ptr, _ptr(x), _ptr(gain), _ptr(y), rows, d, eps))
 
-    def op_linear(self, a, w, out, mode=0):
+    def op_linear(self, a, w, out, mode=0, tile=0):
         M, K = a.shape
         N = w.shape[0]
-        self._check(self._L.dcl_op_linear(self.ptr, _ptr(a), _ptr(w), _ptr(out), M, N, K, mode))
+        self._check(self._L.dcl_op_linear(self.ptr, _ptr(a), _ptr(w), _ptr(out), M, N, K, mode, tile))
 
     def op_attention(self, qkv, out, batch, T, H, G, hd):
         self._check(self._L.dcl_op_attention(self.ptr, _ptr(qkv), _ptr(out), batch, T, H, G, hd))
 
-    def op_lmhead_top2(self, x, w, top1, p1, p2):
+    def op_lmhead_top2(self, x, w, top1, p1, p2, tile=0):
         R, d = x.shape
         V = w.shape[0]
         self._check(self._L.dcl_op_lmhead_top2(self.ptr, _ptr(x), _ptr(w), R, V, d, _ptr(top1),
-                                               _ptr(p1), _ptr(p2)))
+                                               _ptr(p1), _ptr(p2), tile))
 
     def op_generate(self, dst, seed, tid, start, count, std, mean=0.0):
         self._check(self._L.dcl_op_generate(self.ptr, _ptr(dst), seed, tid, start, count, std, mean))

@@ -60,7 +60,8 @@ struct EpiParams {
 struct GemmPlan {
   CUtensorMap ta, tb;
   int M = 0, N = 0, K = 0;
-  int bn = 256;
+  int bn = 256;          // output columns per tile
+  int cg = 1;            // 1: one CTA per 128 x bn tile; 2: a CTA pair per 256 x 256 tile
   int epi = EPI_BF16;
   EpiParams ep;
   int grid = 0;
@@ -68,10 +69,12 @@ struct GemmPlan {
   size_t smem = 0;
 };
 
-// Encode the tensor maps and choose the tile width / grid.  A is [M][K] bf16 (row
-// pitch K), W is [N][K] bf16.  bn = 0 lets the planner choose 128 or 256.
+// Encode the tensor maps and choose the tile / grid.  A is [M][K] bf16 (row pitch K),
+// W is [N][K] bf16.  tile: 0 lets the planner choose; 128 or 256 force a one-CTA tile of
+// that width; kTilePair forces the CTA-pair 256 x 256 tile.
+constexpr int kTilePair = 2;
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
-                      int epi, const EpiParams& ep, int num_sms, int bn, const char** why);
+                      int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
 

@@ -281,7 +281,7 @@ dcl_status build_plans(dcl_ctx* c) {
     e2.out = c->act;
     e2.ldo = m.ffn_dim;
     if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms,
-                  256, &why))
+                  0, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "gate/up plan: %s", why ? why : "?");
     if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms,
                   0, &why))
@@ -290,7 +290,7 @@ dcl_status build_plans(dcl_ctx* c) {
   EpiParams el;
   el.out = c->part;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,
-                c->num_sms, 256, &why))
+                c->num_sms, 0, &why))
     return fail(c, DCL_ERR_UNSUPPORTED, "LM-head plan: %s", why ? why : "?");
   return DCL_OK;
 }
@@ -771,15 +771,16 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* c, const float* x_dev, const void* gain_dev, 
 }
 
 dcl_status dcl_op_linear(dcl_ctx* c, const void* a_dev, const void* w_dev, void* out_dev, int32_t M, int32_t N,
-                         int32_t K, int32_t mode) {
+                         int32_t K, int32_t mode, int32_t tile) {
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!a_dev || !w_dev || !out_dev || (mode != 0 && mode != 1)) return fail(c, DCL_ERR_INVALID_ARG, "bad linear args");
+  if (tile != 0 && tile != 128 && tile != 256 && tile != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
   GemmPlan pl;
   EpiParams ep;
   ep.out = out_dev;
   ep.ldo = N;
   const char* why = nullptr;
-  if (gemm_plan(&pl, a_dev, M, K, w_dev, N, mode == 0 ? EPI_BF16 : EPI_RESID_F32, ep, c->num_sms, 0, &why))
+  if (gemm_plan(&pl, a_dev, M, K, w_dev, N, mode == 0 ? EPI_BF16 : EPI_RESID_F32, ep, c->num_sms, tile, &why))
     return fail(c, DCL_ERR_INVALID_ARG, "%s", why ? why : "bad GEMM shape");
   CUDA_TRY(c, gemm_launch(pl, c->derr, c->stream));
   return check_device(c);
@@ -796,10 +797,11 @@ dcl_status dcl_op_attention(dcl_ctx* c, const void* qkv_dev, void* out_dev, int3
 }
 
 dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, int32_t R, int32_t V, int32_t d,
-                              int32_t* top1_dev, float* p1_dev, float* p2_dev) {
+                              int32_t* top1_dev, float* p1_dev, float* p2_dev, int32_t tile) {
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!x_dev || !w_dev || !top1_dev || !p1_dev || !p2_dev || R <= 0 || V <= 1)
     return fail(c, DCL_ERR_INVALID_ARG, "bad lmhead args");
+  if (tile != 0 && tile != 256 && tile != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
   const int nblk = gemm_lmhead_blocks(V);
   float4* part = static_cast<float4*>(dev_alloc(c, sizeof(float4) * (size_t)R * nblk));
   if (!part) return fail(c, DCL_ERR_OOM, "partials allocation failed");
@@ -807,7 +809,7 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
   EpiParams ep;
   ep.out = part;
   const char* why = nullptr;
-  if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, 256, &why))
+  if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, tile, &why))
     return fail(c, DCL_ERR_INVALID_ARG, "%s", why ? why : "bad LM-head shape");
   CUDA_TRY(c, gemm_launch(pl, c->derr, c->stream));
   CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, c->stream));

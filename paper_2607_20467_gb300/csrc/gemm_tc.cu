@@ -481,6 +481,223 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ------------------------------------------------------------------ 2-CTA variant
+// A CTA pair (cluster of 2) computes a 256 x 256 tile with tcgen05.mma.cta_group::2:
+// each CTA stages its own 128 rows of A and its own 128-row half of the weight tile
+// (32 KB per K block instead of 48 KB, so a 6-deep ring fits), the even CTA issues the
+// M = 256 MMAs for both, and each CTA's TMEM receives its 128 rows x 256 columns.
+constexpr int B2_STAGE_BYTES = 128 * BK * 2;
+constexpr int STAGE2_BYTES = A_STAGE_BYTES + B2_STAGE_BYTES;
+constexpr int STAGES2 = 6;
+constexpr size_t SMEM2 = 1024 + (size_t)STAGES2 * STAGE2_BYTES + 256;
+constexpr int TMEM2_COLS = 512;
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* tm, int x, int y,
+                                                 uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(holder), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// arrive (once) on the mbarrier at this offset in every CTA of cta_mask
+__device__ __forceinline__ void umma_commit_pair(uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          bar),
+      "h"(cta_mask)
+      : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+template <int EPI>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, int M,
+                    int N, int K, EpiParams ep, int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+  const uint32_t sA = base;
+  const uint32_t sB = base + STAGES2 * A_STAGE_BYTES;
+  const uint32_t bars = sB + STAGES2 * B2_STAGE_BYTES;
+  const uint32_t full0 = bars;
+  const uint32_t empty0 = bars + 8 * STAGES2;
+  const uint32_t tfull0 = bars + 16 * STAGES2;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain = tempty0 + 16;
+  const uint32_t holder = drain + 8;
+  volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
+  const int cluster = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+  const int num_m = (M + 255) / 256;
+  const int num_n = (N + 255) / 256;
+  const int num_tiles = num_m * num_n;
+  const int num_kb = (K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES2; ++s) {
+      mbar_init(full0 + 8 * s, 1);   // leader's producer arrives; both CTAs' copies complete_tx
+      mbar_init(empty0 + 8 * s, 1);  // the leader's MMA commit (multicast)
+    }
+    mbar_init(tfull0, 1);
+    mbar_init(tfull0 + 8, 1);
+    mbar_init(tempty0, 8);  // 4 epilogue warps x 2 CTAs (used in the leader)
+    mbar_init(tempty0 + 8, 8);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tma);
+    prefetch_tmap(&tmb);
+  }
+  if (warp == 1) tmem_alloc_pair(holder, TMEM2_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // the peer's barriers exist before any remote arrive / multicast
+  tc_fence_after();
+  const uint32_t tmem_base = *holder_ptr;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer (both CTAs)
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int t = cluster; t < num_tiles && ok; t += n_clusters) {
+        const int m_blk = t % num_m, n_blk = t / num_m;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t full_leader = mapa_shared(full0 + 8 * stage, 0);
+          if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, 2 * STAGE2_BYTES);
+          tma_load_2d_pair(sA + stage * A_STAGE_BYTES, &tma, kb * BK, m_blk * 256 + (int)rank * 128, full_leader);
+          tma_load_2d_pair(sB + stage * B2_STAGE_BYTES, &tmb, kb * BK, n_blk * 256 + (int)rank * 128, full_leader);
+          if (++stage == STAGES2) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ------------------------------------------------ MMA issuer (leader CTA only)
+      constexpr uint32_t idesc = make_idesc(256, 256);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int j = 0;
+      for (int t = cluster; t < num_tiles && ok; t += n_clusters, ++j) {
+        const int ab = j & 1;
+        const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+        if (!mbar_wait(tempty0 + 8 * ab, aph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * 256);
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = sw128_desc(sA + stage * A_STAGE_BYTES);
+          const uint64_t db = sw128_desc(sB + stage * B2_STAGE_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit_pair(empty0 + 8 * stage, 0x3);
+          if (++stage == STAGES2) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit_pair(tfull0 + 8 * ab, 0x3);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+      }
+      umma_commit_pair(drain, 0x1);
+      volatile int no_abort = 0;
+      mbar_wait(drain, 0, &no_abort);
+    }
+  } else {
+    // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
+    const int q = warp & 3;
+    int j = 0;
+    for (int t = cluster; t < num_tiles; t += n_clusters, ++j) {
+      const int ab = j & 1;
+      const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+      if (!mbar_wait(tfull0 + 8 * ab, aph, abort_flag)) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const int m_blk = t % num_m, n_blk = t / num_m;
+      const int row = m_blk * 256 + (int)rank * 128 + q * 32 + lane;
+      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
+      epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(tempty0 + 8 * ab, 0));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  __syncwarp();
+  cluster_sync_all();  // no CTA leaves while its pair may still touch its smem or TMEM
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, TMEM2_COLS);
+  }
+}
+
 // ------------------------------------------------------------------ host side
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -521,6 +738,19 @@ cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int EPI>
+cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
+  static bool attr_set = false;
+  auto kern = gemm_tc2_kernel<EPI>;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
+  return cudaGetLastError();
+}
+
 double wave_efficiency(long tiles, int sms) {
   const long waves = (tiles + sms - 1) / sms;
   return (double)tiles / (double)(waves * sms);
@@ -531,7 +761,7 @@ double wave_efficiency(long tiles, int sms) {
 int gemm_lmhead_blocks(int vocab) { return (vocab + 255) / 256; }
 
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N, int epi,
-                      const EpiParams& ep, int num_sms, int bn, const char** why) {
+                      const EpiParams& ep, int num_sms, int tile, const char** why) {
   *why = nullptr;
   if (M <= 0 || N <= 0 || K <= 0 || K % BK != 0 || (epi != EPI_LMHEAD && N % 32 != 0)) {
     *why = "gemm: need M, N, K > 0, K % 64 == 0 and (except for the LM head) N % 32 == 0";
@@ -541,13 +771,29 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     *why = "gemm: operands must be 16-byte aligned";
     return cudaErrorInvalidValue;
   }
-  if (epi == EPI_SWIGLU || epi == EPI_LMHEAD) {
+  // Estimated efficiency = wave fill x a feed factor (how busy the tensor pipe stays while
+  // the tile runs; the pair tile halves each SM's weight traffic).
+  int bn = tile, cg = 1;
+  if (tile == kTilePair) {
     bn = 256;
-  } else if (bn == 0) {
-    const long m = (M + BM - 1) / BM;
-    const double e256 = wave_efficiency(m * ((N + 255) / 256), num_sms);
-    const double e128 = 0.9 * wave_efficiency(m * ((N + 127) / 128), num_sms);
-    bn = (e256 >= e128) ? 256 : 128;
+    cg = 2;
+  } else if (tile == 0) {
+    const long m1 = (M + BM - 1) / BM, m2 = (M + 255) / 256;
+    const double e256 = 0.62 * wave_efficiency(m1 * ((N + 255) / 256), num_sms);
+    const double e128 = (epi == EPI_SWIGLU || epi == EPI_LMHEAD)
+                            ? 0.0
+                            : 0.55 * wave_efficiency(m1 * ((N + 127) / 128), num_sms);
+    const double e2 = (num_sms >= 2 && M > BM) ? 0.85 * wave_efficiency(m2 * ((N + 255) / 256), num_sms / 2) : 0.0;
+    if (e2 >= e256 && e2 >= e128) {
+      bn = 256;
+      cg = 2;
+    } else {
+      bn = (e256 >= e128) ? 256 : 128;
+    }
+  }
+  if ((epi == EPI_SWIGLU || epi == EPI_LMHEAD) && bn != 256) {
+    *why = "gemm: SwiGLU and LM-head epilogues need 256-column tiles";
+    return cudaErrorInvalidValue;
   }
   if (bn != 128 && bn != 256) {
     *why = "gemm: tile width must be 128 or 256";
@@ -566,20 +812,39 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   plan->N = N;
   plan->K = K;
   plan->bn = bn;
+  plan->cg = cg;
   plan->epi = epi;
   plan->ep = ep;
   if (epi == EPI_LMHEAD) plan->ep.vocab = N;
-  if (!encode_kmajor(&plan->ta, A, M, K, BM) || !encode_kmajor(&plan->tb, W, N, K, bn)) {
+  // each CTA loads 128 rows of A; of W a one-CTA tile loads bn rows, a pair CTA 128
+  if (!encode_kmajor(&plan->ta, A, M, K, BM) || !encode_kmajor(&plan->tb, W, N, K, cg == 2 ? 128 : bn)) {
     *why = "gemm: cuTensorMapEncodeTiled failed";
     return cudaErrorInvalidValue;
   }
-  plan->n_tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn);
-  plan->grid = plan->n_tiles < num_sms ? plan->n_tiles : num_sms;
-  plan->smem = (bn == 256) ? Cfg<256>::SMEM : Cfg<128>::SMEM;
+  if (cg == 2) {
+    plan->n_tiles = ((M + 255) / 256) * ((N + 255) / 256);
+    const int pairs = num_sms / 2;
+    plan->grid = 2 * (plan->n_tiles < pairs ? plan->n_tiles : pairs);
+    plan->smem = SMEM2;
+  } else {
+    plan->n_tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn);
+    plan->grid = plan->n_tiles < num_sms ? plan->n_tiles : num_sms;
+    plan->smem = (bn == 256) ? Cfg<256>::SMEM : Cfg<128>::SMEM;
+  }
   return cudaSuccess;
 }
 
 cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
+  if (p.cg == 2) {
+    switch (p.epi) {
+      case EPI_BF16: return launch_t2<EPI_BF16>(p, err, stream);
+      case EPI_RESID_F32: return launch_t2<EPI_RESID_F32>(p, err, stream);
+      case EPI_QKV_ROPE: return launch_t2<EPI_QKV_ROPE>(p, err, stream);
+      case EPI_SWIGLU: return launch_t2<EPI_SWIGLU>(p, err, stream);
+      case EPI_LMHEAD: return launch_t2<EPI_LMHEAD>(p, err, stream);
+    }
+    return cudaErrorInvalidValue;
+  }
   if (p.bn == 256) {
     switch (p.epi) {
       case EPI_BF16: return launch_t<256, EPI_BF16>(p, err, stream);

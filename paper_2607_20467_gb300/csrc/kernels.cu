@@ -87,6 +87,47 @@ __global__ void __launch_bounds__(THREADS) rmsnorm_kernel(const float* __restric
   }
 }
 
+// Single pass: ROWS rows per CTA, 128 threads per row, each thread keeping its
+// VPT float4 of the row in registers between the sum of squares and the scaling.
+template <int VPT, int ROWS>
+__global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
+    const float* __restrict__ x, const __nv_bfloat16* __restrict__ gain, __nv_bfloat16* __restrict__ y,
+    int rows, int d, float eps, int rows_per_seq, int seq_stride, int row_offset) {
+  const int sub = threadIdx.x >> 7, t = threadIdx.x & 127;
+  const int r = blockIdx.x * ROWS + sub;
+  const bool live = r < rows;
+  const int in_row = (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
+  const int n4 = d / 4;
+  float4 v[VPT];
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int j = t + 128 * i;
+    v[i] = (live && j < n4) ? xr[j] : make_float4(0.f, 0.f, 0.f, 0.f);
+    ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(kFull, ss, o);
+  __shared__ float red[ROWS][4];
+  if ((t & 31) == 0) red[sub][t >> 5] = ss;
+  __syncthreads();
+  const float tot = red[sub][0] + red[sub][1] + red[sub][2] + red[sub][3];
+  const float inv = rsqrtf(tot / (float)d + eps);
+  if (!live) return;
+  const uint2* g2 = reinterpret_cast<const uint2*>(gain);
+  uint2* y2 = reinterpret_cast<uint2*>(y + (size_t)r * d);
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int j = t + 128 * i;
+    if (j < n4) {
+      const uint2 g = __ldg(g2 + j);
+      y2[j] = make_uint2(pack_bf16x2(v[i].x * inv * bf16_lo(g.x), v[i].y * inv * bf16_hi(g.x)),
+                         pack_bf16x2(v[i].z * inv * bf16_lo(g.y), v[i].w * inv * bf16_hi(g.y)));
+    }
+  }
+}
+
 // ------------------------------------------------------------------ softmax partial merge
 // A partial is {max, sum exp(z - max), argmax id, second largest z} over some columns.
 struct Part {
@@ -321,7 +362,17 @@ cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloa
                            float eps, int rows_per_seq, int seq_stride, int row_offset,
                            cudaStream_t stream) {
   if (d % 4 || rows <= 0) return cudaErrorInvalidValue;
-  rmsnorm_kernel<256><<<rows, 256, 0, stream>>>(x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
+  const int vpt = (d / 4 + 127) / 128;  // float4 per thread with 128 threads per row
+  const int grid2 = (rows + 1) / 2;
+  switch (vpt) {
+    case 1: rmsnorm_reg_kernel<1, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+    case 2: rmsnorm_reg_kernel<2, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+    case 4: case 3: rmsnorm_reg_kernel<4, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+    case 5: case 6: case 7: case 8:
+      rmsnorm_reg_kernel<8, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+    default:
+      rmsnorm_kernel<256><<<rows, 256, 0, stream>>>(x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
+  }
   return cudaGetLastError();
 }
 

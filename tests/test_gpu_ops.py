@@ -62,14 +62,18 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
+TILES = [0, 128, 256, 2]  # auto, one-CTA 128 / 256 columns, CTA pair 256 x 256
+
+
+@pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("M,N,K", [(96, 768, 256), (128, 256, 64), (300, 512, 1024), (1, 128, 64),
                                    (257, 384, 192), (512, 4096, 4096), (200, 1024, 12288)])
-def test_linear_bf16(ops, M, N, K):
+def test_linear_bf16(ops, M, N, K, tile):
     rng = np.random.default_rng(M + N + K)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
     out = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
-    ops.op_linear(_bf16(a), _bf16(w), out, mode=0)
+    ops.op_linear(_bf16(a), _bf16(w), out, mode=0, tile=tile)
     torch.cuda.synchronize()
     ref = a.astype(np.float64) @ w.astype(np.float64).T
     got = _f64(out)
@@ -78,14 +82,15 @@ def test_linear_bf16(ops, M, N, K):
     assert (err <= 2 ** -8 * np.abs(ref) + 1e-3 * np.sqrt((ref ** 2).mean())).all()
 
 
+@pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("M,N,K", [(96, 256, 256), (512, 4096, 4096), (70, 3584, 3584)])
-def test_linear_residual(ops, M, N, K):
+def test_linear_residual(ops, M, N, K, tile):
     rng = np.random.default_rng(7 * M + N)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
     h0 = rng.normal(0, 2, (M, N)).astype(np.float32)
     h = torch.from_numpy(h0).cuda()
-    ops.op_linear(_bf16(a), _bf16(w), h, mode=1)
+    ops.op_linear(_bf16(a), _bf16(w), h, mode=1, tile=tile)
     torch.cuda.synchronize()
     ref = h0.astype(np.float64) + a.astype(np.float64) @ w.astype(np.float64).T
     assert np.abs(h.cpu().numpy() - ref).max() <= 1e-4 * np.sqrt((ref ** 2).mean()) * 10
@@ -115,9 +120,10 @@ def test_attention_non_causal(ops, B, T, H, G, hd):
 
 
 # ------------------------------------------------------------------ LM head + confidence
+@pytest.mark.parametrize("tile", [0, 256, 2])
 @pytest.mark.parametrize("R,V,d,sz", [(37, 4096, 256, 12.0), (5, 1000, 128, 6.0), (130, 4096, 64, 20.0),
-                                      (64, 126464, 4096, 15.0)])
-def test_lmhead_top2(ops, R, V, d, sz):
+                                      (300, 4096, 256, 12.0), (64, 126464, 4096, 15.0)])
+def test_lmhead_top2(ops, R, V, d, sz, tile):
     rng = np.random.default_rng(R * V + d)
     x = syn.round_bf16(rng.normal(0, 1, (R, d)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, sz / np.sqrt(d), (V, d)).astype(np.float32))
@@ -130,7 +136,7 @@ def test_lmhead_top2(ops, R, V, d, sz):
     top1 = torch.zeros(R, dtype=torch.int32, device="cuda")
     p1 = torch.zeros(R, dtype=torch.float32, device="cuda")
     p2 = torch.zeros(R, dtype=torch.float32, device="cuda")
-    ops.op_lmhead_top2(_bf16(x), _bf16(w), top1, p1, p2)
+    ops.op_lmhead_top2(_bf16(x), _bf16(w), top1, p1, p2, tile=tile)
     torch.cuda.synchronize()
     rows = np.arange(R) if R <= 64 else rng.choice(R, 32, replace=False)
     z = x[rows].astype(np.float64) @ w.astype(np.float64).T
