@@ -218,7 +218,8 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
 
 /* Tile choices of the GEMM entry points: 0 lets the library choose (as in the step),
  * 128 / 256 force a one-CTA 128 x 128 / 128 x 256 tile, DCL_TILE_PAIR a CTA-pair
- * (tcgen05 cta_group::2) 256 x 256 tile. */
+ * (tcgen05 cta_group::2) 256 x 256 tile, DCL_TILE_PAIR | (S << 8) that tile with the K
+ * dimension split S ways (partial sums combined in split order, deterministically). */
 #define DCL_TILE_PAIR 2
 
 /* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05

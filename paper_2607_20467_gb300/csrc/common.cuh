@@ -67,12 +67,17 @@ struct GemmPlan {
   int grid = 0;
   int n_tiles = 0;
   size_t smem = 0;
+  int splits = 1;          // split-K factor (pair tiles only)
+  size_t flags_needed = 0; // ints of zero-initialised split counters the launch needs
+  size_t ws_needed = 0;    // floats of workspace for split-K partials
+  int* flags = nullptr;    // set by the caller when flags_needed > 0
+  float* ws = nullptr;     // set by the caller when ws_needed > 0
 };
 
 // Encode the tensor maps and choose the tile / grid.  A is [M][K] bf16 (row pitch K),
 // W is [N][K] bf16.  tile: 0 lets the planner choose; 128 or 256 force a one-CTA tile of
 // that width; kTilePair forces the CTA-pair 256 x 256 tile.
-constexpr int kTilePair = 2;
+constexpr int kTilePair = 2;  // tile = kTilePair | (S << 8) forces S splits (S = 0: chosen)
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
                       int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);

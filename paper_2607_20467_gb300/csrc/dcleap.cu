@@ -4,6 +4,7 @@
 #include <chrono>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -58,6 +59,10 @@ struct dcl_ctx {
   int* derr = nullptr;
   float *rope_cos = nullptr, *rope_sin = nullptr;
   float* snap = nullptr;  // residual stream after the embedding and after each layer (debug)
+  int* gemm_flags = nullptr;  // split-K counters of the step's GEMMs (zero between launches)
+  size_t gemm_flags_n = 0;
+  float* gemm_ws = nullptr;   // split-K partials of the step's GEMMs
+  size_t gemm_ws_n = 0;
   size_t snap_rows = 0;
 
   // accept scratch (dcl_accept)
@@ -130,6 +135,20 @@ void dev_free_all(dcl_ctx* c) {
   c->owned.clear();
 }
 
+void dev_free_one(dcl_ctx* c, void* ptr) {
+  if (!ptr) return;
+  for (size_t i = 0; i < c->owned.size(); ++i) {
+    if (c->owned[i] == ptr) {
+      c->owned.erase(c->owned.begin() + i);
+      if (c->custom_alloc)
+        c->alloc.free(ptr, c->alloc.user);
+      else
+        cudaFree(ptr);
+      return;
+    }
+  }
+}
+
 // Read and clear the device error word; map it to a status.
 dcl_status check_device(dcl_ctx* c) {
   int e = 0;
@@ -138,6 +157,8 @@ dcl_status check_device(dcl_ctx* c) {
   if (e != DERR_NONE) {
     const int zero = 0;
     cudaMemcpy(c->derr, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    // an aborted split-K launch may leave its counters set: clear them for the next one
+    if (c->gemm_flags) cudaMemset(c->gemm_flags, 0, sizeof(int) * c->gemm_flags_n);
     if (e == DERR_WAIT_TIMEOUT)
       return fail(c, DCL_ERR_TIMEOUT, "a GEMM pipeline wait timed out on the device (kernel returned)");
     if (e == DERR_TOKEN_RANGE) return fail(c, DCL_ERR_INVALID_ARG, "a token id outside [0, vocab) reached the embedding");
@@ -253,12 +274,34 @@ dcl_status build_graph(dcl_ctx* c) {
   return DCL_OK;
 }
 
+// Tile of one of the step's GEMMs ("qkv", "o", "gateup", "down", "lmhead") forced by the
+// environment variable DCL_GEMM_TILES, e.g. "o=128,down=pair:2" (128 / 256 = one-CTA tile
+// width, pair[:S] = CTA-pair tile with S K-splits); 0 = let the planner choose.
+int tile_override(const char* name) {
+  const char* env = getenv("DCL_GEMM_TILES");
+  if (!env) return 0;
+  const size_t n = strlen(name);
+  for (const char* s = env; *s;) {
+    const char* e = strchr(s, ',');
+    const size_t len = e ? (size_t)(e - s) : strlen(s);
+    if (len > n && strncmp(s, name, n) == 0 && s[n] == '=') {
+      const char* v = s + n + 1;
+      if (strncmp(v, "pair", 4) == 0) return kTilePair | ((v[4] == ':' ? atoi(v + 5) : 0) << 8);
+      return atoi(v);
+    }
+    s += len + (e ? 1 : 0);
+  }
+  return 0;
+}
+
 dcl_status build_plans(dcl_ctx* c) {
   const dcl_model_config& m = c->cfg;
   const int R = c->B * c->T, d = m.d_model, hd = m.head_dim;
   const int nqkv = (m.n_heads + 2 * m.n_kv_heads) * hd;
   c->plans.assign(4 * m.n_layers + 1, GemmPlan{});
   const char* why = nullptr;
+  const int t_qkv = tile_override("qkv"), t_o = tile_override("o"), t_gu = tile_override("gateup"),
+            t_down = tile_override("down"), t_lm = tile_override("lmhead");
   for (int l = 0; l < m.n_layers; ++l) {
     const Layer& L = c->layers[l];
     EpiParams e0;
@@ -269,30 +312,83 @@ dcl_status build_plans(dcl_ctx* c) {
     e0.rope_cols = (m.n_heads + m.n_kv_heads) * hd;
     e0.head_dim = hd;
     e0.seq_T = c->T;
-    if (gemm_plan(&c->plans[4 * l], c->xn, R, d, L.wqkv, nqkv, EPI_QKV_ROPE, e0, c->num_sms, 0, &why))
+    if (gemm_plan(&c->plans[4 * l], c->xn, R, d, L.wqkv, nqkv, EPI_QKV_ROPE, e0, c->num_sms, t_qkv, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "QKV plan: %s", why ? why : "?");
     EpiParams e1;
     e1.out = c->h;
     e1.ldo = d;
     if (gemm_plan(&c->plans[4 * l + 1], c->attn, R, m.n_heads * hd, L.wo, d, EPI_RESID_F32, e1,
-                  c->num_sms, 0, &why))
+                  c->num_sms, t_o, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "O plan: %s", why ? why : "?");
     EpiParams e2;
     e2.out = c->act;
     e2.ldo = m.ffn_dim;
     if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms,
-                  0, &why))
+                  t_gu, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "gate/up plan: %s", why ? why : "?");
     if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms,
-                  0, &why))
+                  t_down, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "down plan: %s", why ? why : "?");
   }
   EpiParams el;
   el.out = c->part;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,
-                c->num_sms, 0, &why))
+                c->num_sms, t_lm, &why))
     return fail(c, DCL_ERR_UNSUPPORTED, "LM-head plan: %s", why ? why : "?");
+  // split-K counters and partials, shared by the step's GEMMs (they run one after another)
+  size_t need_f = 0, need_w = 0;
+  for (const GemmPlan& p : c->plans) {
+    need_f = p.flags_needed > need_f ? p.flags_needed : need_f;
+    need_w = p.ws_needed > need_w ? p.ws_needed : need_w;
+  }
+  if (need_f > c->gemm_flags_n || need_w > c->gemm_ws_n) {
+    CUDA_TRY(c, cudaStreamSynchronize(c->stream));  // no launch may still use the old buffers
+    if (c->gexec) {
+      cudaGraphExecDestroy(c->gexec);
+      c->gexec = nullptr;
+    }
+  }
+  if (need_f > c->gemm_flags_n) {
+    dev_free_one(c, c->gemm_flags);
+    c->gemm_flags = static_cast<int*>(dev_alloc(c, sizeof(int) * need_f));
+    if (!c->gemm_flags) return fail(c, DCL_ERR_OOM, "split-K counter allocation failed");
+    CUDA_TRY(c, cudaMemset(c->gemm_flags, 0, sizeof(int) * need_f));
+    c->gemm_flags_n = need_f;
+  }
+  if (need_w > c->gemm_ws_n) {
+    dev_free_one(c, c->gemm_ws);
+    c->gemm_ws = static_cast<float*>(dev_alloc(c, sizeof(float) * need_w));
+    if (!c->gemm_ws) return fail(c, DCL_ERR_OOM, "split-K workspace allocation failed");
+    c->gemm_ws_n = need_w;
+  }
+  for (GemmPlan& p : c->plans) {
+    p.flags = c->gemm_flags;
+    p.ws = c->gemm_ws;
+  }
   return DCL_OK;
+}
+
+// Scratch for a one-off GEMM launch (the single-kernel entry points): allocated here,
+// released by release_scratch after the launch has completed.
+dcl_status attach_scratch(dcl_ctx* c, GemmPlan* p) {
+  if (p->flags_needed) {
+    p->flags = static_cast<int*>(dev_alloc(c, sizeof(int) * p->flags_needed));
+    if (!p->flags) return fail(c, DCL_ERR_OOM, "split-K counter allocation failed");
+    CUDA_TRY(c, cudaMemsetAsync(p->flags, 0, sizeof(int) * p->flags_needed, c->stream));
+  }
+  if (p->ws_needed) {
+    p->ws = static_cast<float*>(dev_alloc(c, sizeof(float) * p->ws_needed));
+    if (!p->ws) return fail(c, DCL_ERR_OOM, "split-K workspace allocation failed");
+  }
+  return DCL_OK;
+}
+
+void release_scratch(dcl_ctx* c, GemmPlan* p) {
+  cudaStreamSynchronize(c->stream);
+  dev_free_one(c, p->flags);
+  dev_free_one(c, p->ws);
+  p->flags = nullptr;
+  p->ws = nullptr;
 }
 
 // weight destination for (kind, layer): pointer, rows, and the gate/up interleave offset
@@ -722,7 +818,11 @@ dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, fl
     const char* why = nullptr;
     if (gemm_plan(&pl, c->xg, (int)G, c->cfg.d_model, c->lm_head, c->cfg.vocab, EPI_BF16, ep, c->num_sms, 0, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "logits plan: %s", why ? why : "?");
-    CUDA_TRY(c, gemm_launch(pl, c->derr, c->stream));
+    dcl_status s = attach_scratch(c, &pl);
+    if (s != DCL_OK) return s;
+    const cudaError_t e = gemm_launch(pl, c->derr, c->stream);
+    release_scratch(c, &pl);
+    if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "logits GEMM: %s", cudaGetErrorString(e));
   }
   return check_device(c);
 }
@@ -774,7 +874,8 @@ dcl_status dcl_op_linear(dcl_ctx* c, const void* a_dev, const void* w_dev, void*
                          int32_t K, int32_t mode, int32_t tile) {
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!a_dev || !w_dev || !out_dev || (mode != 0 && mode != 1)) return fail(c, DCL_ERR_INVALID_ARG, "bad linear args");
-  if (tile != 0 && tile != 128 && tile != 256 && tile != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
+  if (tile != 0 && tile != 128 && tile != 256 && (tile & 0xff) != kTilePair)
+    return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
   GemmPlan pl;
   EpiParams ep;
   ep.out = out_dev;
@@ -782,7 +883,11 @@ dcl_status dcl_op_linear(dcl_ctx* c, const void* a_dev, const void* w_dev, void*
   const char* why = nullptr;
   if (gemm_plan(&pl, a_dev, M, K, w_dev, N, mode == 0 ? EPI_BF16 : EPI_RESID_F32, ep, c->num_sms, tile, &why))
     return fail(c, DCL_ERR_INVALID_ARG, "%s", why ? why : "bad GEMM shape");
-  CUDA_TRY(c, gemm_launch(pl, c->derr, c->stream));
+  dcl_status s = attach_scratch(c, &pl);
+  if (s != DCL_OK) return s;
+  const cudaError_t e = gemm_launch(pl, c->derr, c->stream);
+  release_scratch(c, &pl);
+  if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "GEMM launch: %s", cudaGetErrorString(e));
   return check_device(c);
 }
 
@@ -801,7 +906,7 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!x_dev || !w_dev || !top1_dev || !p1_dev || !p2_dev || R <= 0 || V <= 1)
     return fail(c, DCL_ERR_INVALID_ARG, "bad lmhead args");
-  if (tile != 0 && tile != 256 && tile != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
+  if (tile != 0 && tile != 256 && (tile & 0xff) != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
   const int nblk = gemm_lmhead_blocks(V);
   float4* part = static_cast<float4*>(dev_alloc(c, sizeof(float4) * (size_t)R * nblk));
   if (!part) return fail(c, DCL_ERR_OOM, "partials allocation failed");
@@ -811,17 +916,14 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
   const char* why = nullptr;
   if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, tile, &why))
     return fail(c, DCL_ERR_INVALID_ARG, "%s", why ? why : "bad LM-head shape");
-  CUDA_TRY(c, gemm_launch(pl, c->derr, c->stream));
+  dcl_status s = attach_scratch(c, &pl);
+  if (s != DCL_OK) return s;
+  const cudaError_t e = gemm_launch(pl, c->derr, c->stream);
+  release_scratch(c, &pl);
+  if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "LM-head GEMM: %s", cudaGetErrorString(e));
   CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, c->stream));
-  dcl_status s = check_device(c);
-  // release the partials at once (they were appended last)
-  if (!c->owned.empty() && c->owned.back() == part) {
-    c->owned.pop_back();
-    if (c->custom_alloc)
-      c->alloc.free(part, c->alloc.user);
-    else
-      cudaFree(part);
-  }
+  s = check_device(c);
+  dev_free_one(c, part);
   return s;
 }
 

@@ -57,14 +57,16 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// One try: the thread sleeps in hardware until the phase completes or ~1 ms passes
+// (suspend-time hint), instead of spinning on the shared-memory pipe.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}\n"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(1000000u)
       : "memory");
   return ok != 0;
 }
@@ -79,10 +81,8 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) return false;
-    }
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
   }
 }
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y,
@@ -93,6 +93,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm,
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// Bring a box of the tensor into L2 ahead of its load (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* tm, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+#ifndef DCL_PF_AHEAD
+#define DCL_PF_AHEAD 0
+#endif
+constexpr int kPrefetchAhead = DCL_PF_AHEAD;  // K blocks of weights requested into L2 ahead
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
 }
@@ -171,43 +182,79 @@ __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v
 }
 
 // ------------------------------------------------------------------ epilogues
+// Earlier split-K partials of this thread's row: fp32 tiles stored column-major
+// [256 columns][128 rows] per (tile, CTA half); n = 0 for an unsplit tile.
+struct Parts {
+  const float* base = nullptr;  // partial of split 0
+  size_t stride = 0;            // floats from one split's partial to the next
+  int n = 0;                    // number of earlier splits
+  int row = 0;                  // this thread's row within its 128-row half
+};
+
+// Accumulator columns [col, col + 32) of this thread's row, added to the earlier partials
+// in split order: ((p0 + p1) + ...) + own, so the sum is the same on every run.
+__device__ __forceinline__ void load_cols(uint32_t taddr, int col, float (&v)[32], const Parts& ps) {
+  uint32_t r[32];
+  tmem_ld32(taddr + col, r);
+  tmem_ld_wait();
+  if (ps.n == 0) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float* q = ps.base + (size_t)(col + i) * 128 + ps.row;
+      float a = __ldcg(q);
+      for (int sp = 1; sp < ps.n; ++sp) a += __ldcg(q + sp * ps.stride);
+      v[i] = a + f32(r[i]);
+    }
+  }
+}
+
+// Write this thread's accumulator row as a split-K partial (column-major, see Parts).
+template <int BN>
+__device__ __forceinline__ void store_partial(uint32_t taddr, float* dst, int row) {
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    uint32_t r[32];
+    tmem_ld32(taddr + c, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 32; ++i) __stcg(dst + (size_t)(c + i) * 128 + row, f32(r[i]));
+  }
+}
+
 // taddr: TMEM address of (this warp's first lane, accumulator column 0); row: output row
 // of this thread; n_blk: tile column index.  All tcgen05.ld run warp-uniformly; only the
 // stores are guarded by row < M.
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk, int M, int N,
-                                              const EpiParams& ep) {
+                                              const EpiParams& ep, const Parts& ps) {
   const int n0 = n_blk * BN;
   const bool live = row < M;
   if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(taddr + c, r);
-      tmem_ld_wait();
-      if (live && n0 + c < N) {
-        float v[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+      float v[32];
+      load_cols(taddr, c, v, ps);
+      if (live && n0 + c < N)
         store_bf16x32(reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)row * ep.ldo + n0 + c, v);
-      }
     }
   } else if constexpr (EPI == EPI_RESID_F32) {
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(taddr + c, r);
-      tmem_ld_wait();
+      float v[32];
+      load_cols(taddr, c, v, ps);
       if (live && n0 + c < N) {
         float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(ep.out) +
                                                 (size_t)row * ep.ldo + n0 + c);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           float4 o = dst[i];
-          o.x += f32(r[4 * i + 0]);
-          o.y += f32(r[4 * i + 1]);
-          o.z += f32(r[4 * i + 2]);
-          o.w += f32(r[4 * i + 3]);
+          o.x += v[4 * i + 0];
+          o.y += v[4 * i + 1];
+          o.z += v[4 * i + 2];
+          o.w += v[4 * i + 3];
           dst[i] = o;
         }
       }
@@ -223,18 +270,16 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
       for (int hb = 0; hb < BN; hb += hd) {
 #pragma unroll 1
         for (int j0 = 0; j0 < half; j0 += 32) {
-          uint32_t lo[32], hi[32];
-          tmem_ld32(taddr + hb + j0, lo);
-          tmem_ld32(taddr + hb + half + j0, hi);
-          tmem_ld_wait();
+          float lo[32], hi[32];
+          load_cols(taddr, hb + j0, lo, ps);
+          load_cols(taddr, hb + half + j0, hi, ps);
           if (live) {
             float a[32], b[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const float c = __ldg(cs + j0 + i), s = __ldg(sn + j0 + i);
-              const float x1 = f32(lo[i]), x2 = f32(hi[i]);
-              a[i] = x1 * c - x2 * s;
-              b[i] = x2 * c + x1 * s;
+              a[i] = lo[i] * c - hi[i] * s;
+              b[i] = hi[i] * c + lo[i] * s;
             }
             store_bf16x32(out + hb + j0, a);
             store_bf16x32(out + hb + half + j0, b);
@@ -244,15 +289,9 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
     } else {
 #pragma unroll 1
       for (int c = 0; c < BN; c += 32) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c, r);
-        tmem_ld_wait();
-        if (live) {
-          float v[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
-          store_bf16x32(out + c, v);
-        }
+        float v[32];
+        load_cols(taddr, c, v, ps);
+        if (live) store_bf16x32(out + c, v);
       }
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
@@ -260,17 +299,13 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(ep.out) + (size_t)row * ep.ldo + n_blk * H2;
 #pragma unroll 1
     for (int c = 0; c < H2; c += 32) {
-      uint32_t g[32], u[32];
-      tmem_ld32(taddr + c, g);
-      tmem_ld32(taddr + H2 + c, u);
-      tmem_ld_wait();
+      float g[32], u[32];
+      load_cols(taddr, c, g, ps);
+      load_cols(taddr, H2 + c, u, ps);
       if (live) {
         float v[32];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float x = f32(g[i]);
-          v[i] = x / (1.0f + __expf(-x)) * f32(u[i]);
-        }
+        for (int i = 0; i < 32; ++i) v[i] = g[i] / (1.0f + __expf(-g[i])) * u[i];
         store_bf16x32(out + c, v);
       }
     }
@@ -282,17 +317,15 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
     int id = -1;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(taddr + c, r);
-      tmem_ld_wait();
-      const int col0 = n0 + c;
       float v[32];
+      load_cols(taddr, c, v, ps);
+      const int col0 = n0 + c;
       float cm = m;
       int cid = id;
       float c2 = t2;
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        v[i] = (col0 + i < ep.vocab) ? f32(r[i]) : -INFINITY;
+        if (col0 + i >= ep.vocab) v[i] = -INFINITY;
         if (v[i] > cm) {
           c2 = cm;
           cm = v[i];
@@ -378,7 +411,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
         const int m_blk = t % num_m, n_blk = t / num_m;
+        for (int kb = 0; kb < num_kb && kb < kPrefetchAhead; ++kb)
+          tma_prefetch_l2(&tmb, kb * BK, n_blk * BN);
         for (int kb = 0; kb < num_kb; ++kb) {
+          if (kb + kPrefetchAhead < num_kb) tma_prefetch_l2(&tmb, (kb + kPrefetchAhead) * BK, n_blk * BN);
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
             ok = false;
             break;
@@ -426,7 +462,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ok = false;
             break;
           }
-          tc_fence_after();
           const uint64_t da = sw128_desc(sA + stage * A_STAGE_BYTES);
           const uint64_t db = sw128_desc(sB + stage * C::B_STAGE_BYTES);
 #pragma unroll
@@ -466,7 +501,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int m_blk = t % num_m, n_blk = t / num_m;
       const int row = m_blk * BM + q * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
-      epilogue_tile<BN, EPI>(taddr, row, n_blk, M, N, ep);
+      epilogue_tile<BN, EPI>(taddr, row, n_blk, M, N, ep, Parts{});
       tc_fence_before();
       mbar_arrive(tempty0 + 8 * ab);
     }
@@ -484,11 +519,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // ------------------------------------------------------------------ 2-CTA variant
 // A CTA pair (cluster of 2) computes a 256 x 256 tile with tcgen05.mma.cta_group::2:
 // each CTA stages its own 128 rows of A and its own 128-row half of the weight tile
-// (32 KB per K block instead of 48 KB, so a 6-deep ring fits), the even CTA issues the
-// M = 256 MMAs for both, and each CTA's TMEM receives its 128 rows x 256 columns.
-constexpr int B2_STAGE_BYTES = 128 * BK * 2;
-constexpr int STAGE2_BYTES = A_STAGE_BYTES + B2_STAGE_BYTES;
-constexpr int STAGES2 = 6;
+// (32 KB per 64-wide K block instead of 48 KB), the even CTA issues the M = 256 MMAs for
+// both, and each CTA's TMEM receives its 128 rows x 256 columns.  A ring stage holds KA2
+// K blocks (KA2 x 4 MMAs per stage barrier round trip).
+#ifndef DCL_PAIR_KA
+#define DCL_PAIR_KA 1
+#endif
+constexpr int KA2 = DCL_PAIR_KA;
+constexpr int A2_STAGE_BYTES = KA2 * A_STAGE_BYTES;
+constexpr int B2_BLOCK_BYTES = 128 * BK * 2;
+constexpr int B2_STAGE_BYTES = KA2 * B2_BLOCK_BYTES;
+constexpr int STAGE2_BYTES = A2_STAGE_BYTES + B2_STAGE_BYTES;
+constexpr int STAGES2 = (7 * 32768) / STAGE2_BYTES;
 constexpr size_t SMEM2 = 1024 + (size_t)STAGES2 * STAGE2_BYTES + 256;
 constexpr int TMEM2_COLS = 512;
 
@@ -542,16 +584,44 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
+__device__ __forceinline__ void epilogue_bar() {  // the 128 epilogue threads (warps 2..5)
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+// Bounded wait until the split-K counter at f reaches target; false on timeout or abort.
+__device__ __noinline__ bool wait_flag_geq(const int* f, int target, volatile int* abort_flag) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+  if (v >= target) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(100);
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+    if (v >= target) return true;
+    if ((it & 15u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) return false;
+    }
+  }
+}
+
+// Work items w = split * tiles + tile (split-major), each a contiguous range of K blocks.
+// Split-K results are combined in split order, so every run gives the same bits:
+//   residual epilogue: split s adds its accumulator to h after split s-1 has (a per-tile
+//     counter, released by each split and reset by the last);
+//   other epilogues: splits < S-1 store fp32 partials, the last split waits for all of
+//     them, sums them in order with its own accumulator and runs the epilogue.
+// Split 0 never waits and each CTA pair takes items in increasing order with every CTA
+// resident (grid <= SMs, one CTA per SM), so the waits always end.
 template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, int M,
-                    int N, int K, EpiParams ep, int* err) {
+                    int N, int K, EpiParams ep, int splits, int* flags, float* ws, int* err) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
   const uint32_t sA = base;
-  const uint32_t sB = base + STAGES2 * A_STAGE_BYTES;
+  const uint32_t sB = base + STAGES2 * A2_STAGE_BYTES;
   const uint32_t bars = sB + STAGES2 * B2_STAGE_BYTES;
   const uint32_t full0 = bars;
   const uint32_t empty0 = bars + 8 * STAGES2;
@@ -568,7 +638,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   const int num_m = (M + 255) / 256;
   const int num_n = (N + 255) / 256;
   const int num_tiles = num_m * num_n;
-  const int num_kb = (K + BK - 1) / BK;
+  const int num_items = num_tiles * splits;
+  const int num_ku = (K + BK * KA2 - 1) / (BK * KA2);  // ring stages of KA2 K blocks each
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
@@ -598,17 +669,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int t = cluster; t < num_tiles && ok; t += n_clusters) {
+      for (int w = cluster; w < num_items && ok; w += n_clusters) {
+        const int sp = w / num_tiles, t = w % num_tiles;
         const int m_blk = t % num_m, n_blk = t / num_m;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        const int kb0 = (int)((long)sp * num_ku / splits) * KA2;
+        const int kb1 = (int)((long)(sp + 1) * num_ku / splits) * KA2;
+        const int wrow = n_blk * 256 + (int)rank * 128;  // this CTA's half of the weight tile
+        for (int kb = kb0; kb < kb1 && kb < kb0 + kPrefetchAhead; ++kb) tma_prefetch_l2(&tmb, kb * BK, wrow);
+        for (int kb = kb0; kb < kb1; kb += KA2) {
+          for (int a = 0; a < KA2; ++a)
+            if (kb + a + kPrefetchAhead < kb1) tma_prefetch_l2(&tmb, (kb + a + kPrefetchAhead) * BK, wrow);
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
             ok = false;
             break;
           }
           const uint32_t full_leader = mapa_shared(full0 + 8 * stage, 0);
           if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, 2 * STAGE2_BYTES);
-          tma_load_2d_pair(sA + stage * A_STAGE_BYTES, &tma, kb * BK, m_blk * 256 + (int)rank * 128, full_leader);
-          tma_load_2d_pair(sB + stage * B2_STAGE_BYTES, &tmb, kb * BK, n_blk * 256 + (int)rank * 128, full_leader);
+          for (int a = 0; a < KA2; ++a) {
+            tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, &tma, (kb + a) * BK,
+                             m_blk * 256 + (int)rank * 128, full_leader);
+            tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, &tmb, (kb + a) * BK, wrow,
+                             full_leader);
+          }
           if (++stage == STAGES2) {
             stage = 0;
             phase ^= 1u;
@@ -628,7 +710,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       bool ok = true;
       int j = 0;
-      for (int t = cluster; t < num_tiles && ok; t += n_clusters, ++j) {
+      for (int w = cluster; w < num_items && ok; w += n_clusters, ++j) {
+        const int sp = w / num_tiles;
+        const int kb0 = (int)((long)sp * num_ku / splits) * KA2;
+        const int kb1 = (int)((long)(sp + 1) * num_ku / splits) * KA2;
         const int ab = j & 1;
         const uint32_t aph = (uint32_t)(j >> 1) & 1u;
         if (!mbar_wait(tempty0 + 8 * ab, aph ^ 1u, abort_flag)) {
@@ -637,17 +722,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * 256);
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = kb0; kb < kb1; kb += KA2) {
           if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) {
             ok = false;
             break;
           }
-          tc_fence_after();
-          const uint64_t da = sw128_desc(sA + stage * A_STAGE_BYTES);
-          const uint64_t db = sw128_desc(sB + stage * B2_STAGE_BYTES);
+          // (no tcgen05 fence here: the stage was written by TMA, whose completion the
+          // mbarrier itself publishes to the tensor core's async proxy)
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          for (int a = 0; a < KA2; ++a) {
+            const uint64_t da = sw128_desc(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES);
+            const uint64_t db = sw128_desc(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, idesc, (kb > kb0 || a > 0 || k > 0) ? 1u : 0u);
+          }
           umma_commit_pair(empty0 + 8 * stage, 0x3);
           if (++stage == STAGES2) {
             stage = 0;
@@ -668,8 +757,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   } else {
     // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
     const int q = warp & 3;
+    const int et = (warp - 2) * 32 + lane;  // 0..127
+    const int row_local = q * 32 + lane;
+    const size_t part_floats = (size_t)256 * 128;                 // one CTA half of a tile
+    const size_t split_stride = (size_t)num_tiles * 2 * part_floats;
     int j = 0;
-    for (int t = cluster; t < num_tiles; t += n_clusters, ++j) {
+    for (int w = cluster; w < num_items; w += n_clusters, ++j) {
+      const int sp = w / num_tiles, t = w % num_tiles;
       const int ab = j & 1;
       const uint32_t aph = (uint32_t)(j >> 1) & 1u;
       if (!mbar_wait(tfull0 + 8 * ab, aph, abort_flag)) {
@@ -679,9 +773,51 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       }
       tc_fence_after();
       const int m_blk = t % num_m, n_blk = t / num_m;
-      const int row = m_blk * 256 + (int)rank * 128 + q * 32 + lane;
+      const int row = m_blk * 256 + (int)rank * 128 + row_local;
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
-      epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep);
+      if (splits == 1) {
+        epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, Parts{});
+      } else {
+        int* flag = flags + t * 2 + rank;
+        if constexpr (EPI == EPI_RESID_F32) {
+          if (et == 0 && !wait_flag_geq(flag, sp, abort_flag)) {
+            *abort_flag = 1;
+            report_error(err, DERR_WAIT_TIMEOUT);
+          }
+          epilogue_bar();
+          if (!*abort_flag) epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, Parts{});
+          epilogue_bar();
+          if (et == 0) {
+            __threadfence();
+            atomicExch(flag, sp + 1 == splits ? 0 : sp + 1);
+          }
+        } else {
+          float* part0 = ws + ((size_t)t * 2 + rank) * part_floats;
+          if (sp < splits - 1) {
+            store_partial<256>(taddr, part0 + sp * split_stride, row_local);
+            epilogue_bar();
+            if (et == 0) {
+              __threadfence();
+              atomicAdd(flag, 1);
+            }
+          } else {
+            if (et == 0 && !wait_flag_geq(flag, splits - 1, abort_flag)) {
+              *abort_flag = 1;
+              report_error(err, DERR_WAIT_TIMEOUT);
+            }
+            epilogue_bar();
+            __threadfence();
+            Parts ps;
+            ps.base = part0;
+            ps.stride = split_stride;
+            ps.n = splits - 1;
+            ps.row = row_local;
+            if (!*abort_flag) epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, ps);
+            epilogue_bar();
+            if (et == 0) atomicExch(flag, 0);
+          }
+        }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(mapa_shared(tempty0 + 8 * ab, 0));
@@ -747,7 +883,7 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
+  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, p.splits, p.flags, p.ws, err);
   return cudaGetLastError();
 }
 
@@ -771,25 +907,39 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     *why = "gemm: operands must be 16-byte aligned";
     return cudaErrorInvalidValue;
   }
-  // Estimated efficiency = wave fill x a feed factor (how busy the tensor pipe stays while
-  // the tile runs; the pair tile halves each SM's weight traffic).
-  int bn = tile, cg = 1;
-  if (tile == kTilePair) {
+  // Tile choice (measured on the LLaDA-8B step's shapes): the CTA-pair tile keeps the
+  // tensor pipe busiest and is used whenever M spans more than one 128-row tile; a
+  // residual GEMM with too few pair tiles to fill the GPU (N = d_model) instead uses
+  // one-CTA 128 x 128 tiles when K is short, or the pair tile with K split in two when K
+  // is long; small M uses one-CTA tiles, 256 or 128 wide by wave fill.
+  const bool pair_forced = (tile & 0xff) == kTilePair;
+  int bn = pair_forced ? kTilePair : tile, cg = 1, splits = 1;
+  const int forced_splits = pair_forced ? (tile >> 8) : 0;
+  const long nkb = (K + BK - 1) / BK;
+  const long m1 = (M + BM - 1) / BM, m2 = (M + 255) / 256;
+  const long pair_tiles = m2 * ((N + 255) / 256);
+  const bool wide_only = (epi == EPI_SWIGLU || epi == EPI_LMHEAD);
+  if (bn == kTilePair) {
     bn = 256;
     cg = 2;
-  } else if (tile == 0) {
-    const long m1 = (M + BM - 1) / BM, m2 = (M + 255) / 256;
-    const double e256 = 0.62 * wave_efficiency(m1 * ((N + 255) / 256), num_sms);
-    const double e128 = (epi == EPI_SWIGLU || epi == EPI_LMHEAD)
-                            ? 0.0
-                            : 0.55 * wave_efficiency(m1 * ((N + 127) / 128), num_sms);
-    const double e2 = (num_sms >= 2 && M > BM) ? 0.85 * wave_efficiency(m2 * ((N + 255) / 256), num_sms / 2) : 0.0;
-    if (e2 >= e256 && e2 >= e128) {
+    splits = forced_splits > 0 ? forced_splits : 1;
+  } else if (bn == 0) {
+    const bool sparse = 4 * pair_tiles < 3 * (num_sms / 2);
+    if (M > BM && num_sms >= 2 && !(epi == EPI_RESID_F32 && sparse && nkb < 128)) {
       bn = 256;
       cg = 2;
+      splits = (epi == EPI_RESID_F32 && sparse && nkb >= 128) ? 2 : 1;
+    } else if (wide_only) {
+      bn = 256;
     } else {
+      const double e256 = wave_efficiency(m1 * ((N + 255) / 256), num_sms);
+      const double e128 = 0.9 * wave_efficiency(m1 * ((N + 127) / 128), num_sms);
       bn = (e256 >= e128) ? 256 : 128;
     }
+  }
+  if (splits < 1 || splits > nkb) {
+    *why = "gemm: split count must be in [1, K/64]";
+    return cudaErrorInvalidValue;
   }
   if ((epi == EPI_SWIGLU || epi == EPI_LMHEAD) && bn != 256) {
     *why = "gemm: SwiGLU and LM-head epilogues need 256-column tiles";
@@ -821,11 +971,21 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     *why = "gemm: cuTensorMapEncodeTiled failed";
     return cudaErrorInvalidValue;
   }
+  plan->splits = splits;
+  plan->flags_needed = 0;
+  plan->ws_needed = 0;
+  plan->flags = nullptr;
+  plan->ws = nullptr;
   if (cg == 2) {
     plan->n_tiles = ((M + 255) / 256) * ((N + 255) / 256);
     const int pairs = num_sms / 2;
-    plan->grid = 2 * (plan->n_tiles < pairs ? plan->n_tiles : pairs);
+    const int items = plan->n_tiles * splits;
+    plan->grid = 2 * (items < pairs ? items : pairs);
     plan->smem = SMEM2;
+    if (splits > 1) {
+      plan->flags_needed = (size_t)plan->n_tiles * 2;
+      if (epi != EPI_RESID_F32) plan->ws_needed = (size_t)(splits - 1) * plan->n_tiles * 2 * 256 * 128;
+    }
   } else {
     plan->n_tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     plan->grid = plan->n_tiles < num_sms ? plan->n_tiles : num_sms;
@@ -835,6 +995,7 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
 }
 
 cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
+  if ((p.flags_needed && !p.flags) || (p.ws_needed && !p.ws)) return cudaErrorInvalidValue;
   if (p.cg == 2) {
     switch (p.epi) {
       case EPI_BF16: return launch_t2<EPI_BF16>(p, err, stream);

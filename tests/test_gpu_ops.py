@@ -62,13 +62,20 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
-TILES = [0, 128, 256, 2]  # auto, one-CTA 128 / 256 columns, CTA pair 256 x 256
+# auto, one-CTA 128 / 256 columns, CTA pair 256 x 256, CTA pair with 2 / 3 K splits
+TILES = [0, 128, 256, 2, 2 | (2 << 8), 2 | (3 << 8)]
+
+
+def _splits(tile):
+    return (tile >> 8) if (tile & 0xff) == 2 else 1
 
 
 @pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("M,N,K", [(96, 768, 256), (128, 256, 64), (300, 512, 1024), (1, 128, 64),
                                    (257, 384, 192), (512, 4096, 4096), (200, 1024, 12288)])
 def test_linear_bf16(ops, M, N, K, tile):
+    if K // 64 < _splits(tile):
+        pytest.skip("fewer K blocks than splits")
     rng = np.random.default_rng(M + N + K)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
@@ -85,6 +92,8 @@ def test_linear_bf16(ops, M, N, K, tile):
 @pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("M,N,K", [(96, 256, 256), (512, 4096, 4096), (70, 3584, 3584)])
 def test_linear_residual(ops, M, N, K, tile):
+    if K // 64 < _splits(tile):
+        pytest.skip("fewer K blocks than splits")
     rng = np.random.default_rng(7 * M + N)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
@@ -94,6 +103,25 @@ def test_linear_residual(ops, M, N, K, tile):
     torch.cuda.synchronize()
     ref = h0.astype(np.float64) + a.astype(np.float64) @ w.astype(np.float64).T
     assert np.abs(h.cpu().numpy() - ref).max() <= 1e-4 * np.sqrt((ref ** 2).mean()) * 10
+
+
+@pytest.mark.parametrize("tile,mode", [(2 | (3 << 8), 1), (2 | (2 << 8), 0), (0, 1)])
+def test_linear_split_k_is_deterministic(ops, tile, mode):
+    """Split-K partial sums are combined in split order: two runs give the same bits."""
+    rng = np.random.default_rng(5)
+    M, N, K = 512, 4096, 12288
+    a = _bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
+    w = _bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
+    outs = []
+    for _ in range(2):
+        if mode == 1:
+            o = torch.ones(M, N, device="cuda")
+        else:
+            o = torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+        ops.op_linear(a, w, o, mode=mode, tile=tile)
+        outs.append(o)
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1])
 
 
 # ------------------------------------------------------------------ attention
