@@ -218,9 +218,15 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
 
 /* Tile choices of the GEMM entry points: 0 lets the library choose (as in the step),
  * 128 / 256 force a one-CTA 128 x 128 / 128 x 256 tile, DCL_TILE_PAIR a CTA-pair
- * (tcgen05 cta_group::2) 256 x 256 tile, DCL_TILE_PAIR | (S << 8) that tile with the K
- * dimension split S ways (partial sums combined in split order, deterministically). */
+ * (tcgen05 cta_group::2) 256 x 256 tile with the library's choice of K splitting,
+ * DCL_TILE_PAIR | (S << 8) that tile with the K dimension split S ways (S = 1: unsplit),
+ * DCL_TILE_PAIR | DCL_TILE_STREAMK that tile with the stream-K schedule (the tiles of a
+ * partly filled last round of the persistent grid are shared out by K ranges over all
+ * CTA pairs; rejected with DCL_ERR_INVALID_ARG when the last round is full or holds
+ * fewer K blocks than there are CTA pairs).  Partial sums are always combined in K order,
+ * so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
+#define DCL_TILE_STREAMK (1 << 16)
 
 /* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05
  * tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];

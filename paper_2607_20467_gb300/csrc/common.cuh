@@ -59,6 +59,8 @@ struct EpiParams {
 
 struct GemmPlan {
   CUtensorMap ta, tb;
+  CUtensorMap tc;        // pair tiles: the output (bf16 / fp32 boxes of 32 rows x 128 bytes)
+  CUtensorMap tw;        // pair tiles with partials: the fp32 workspace [rows][256]
   int M = 0, N = 0, K = 0;
   int bn = 256;          // output columns per tile
   int cg = 1;            // 1: one CTA per 128 x bn tile; 2: a CTA pair per 256 x 256 tile
@@ -68,18 +70,27 @@ struct GemmPlan {
   int n_tiles = 0;
   size_t smem = 0;
   int splits = 1;          // split-K factor (pair tiles only)
+  int streamk = 0;         // 1: left-over pair tiles shared out by K (stream-K)
+  int ws_slots = 0;        // stream-K partial slots per left-over tile
   size_t flags_needed = 0; // ints of zero-initialised split counters the launch needs
   size_t ws_needed = 0;    // floats of workspace for split-K partials
-  int* flags = nullptr;    // set by the caller when flags_needed > 0
-  float* ws = nullptr;     // set by the caller when ws_needed > 0
+  int* flags = nullptr;    // set through gemm_bind_scratch when flags_needed > 0
+  float* ws = nullptr;     // set through gemm_bind_scratch when ws_needed > 0
 };
 
 // Encode the tensor maps and choose the tile / grid.  A is [M][K] bf16 (row pitch K),
 // W is [N][K] bf16.  tile: 0 lets the planner choose; 128 or 256 force a one-CTA tile of
-// that width; kTilePair forces the CTA-pair 256 x 256 tile.
-constexpr int kTilePair = 2;  // tile = kTilePair | (S << 8) forces S splits (S = 0: chosen)
+// that width; kTilePair forces the CTA-pair 256 x 256 tile, kTilePair | (S << 8) that
+// tile with S K splits (S = 0: the planner chooses, S = 1: unsplit),
+// kTilePair | kTileStreamK the pair tile with the stream-K schedule.
+constexpr int kTilePair = 2;
+constexpr int kTileStreamK = 1 << 16;
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
                       int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
+// Attach the zero-initialised counters (>= flags_needed ints) and the workspace
+// (>= ws_needed floats, 16-byte aligned) a plan needs; they may be shared by plans that
+// run one after another on one stream.
+cudaError_t gemm_bind_scratch(GemmPlan* plan, int* flags, float* ws);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
 

@@ -276,7 +276,8 @@ dcl_status build_graph(dcl_ctx* c) {
 
 // Tile of one of the step's GEMMs ("qkv", "o", "gateup", "down", "lmhead") forced by the
 // environment variable DCL_GEMM_TILES, e.g. "o=128,down=pair:2" (128 / 256 = one-CTA tile
-// width, pair[:S] = CTA-pair tile with S K-splits); 0 = let the planner choose.
+// width, pair[:S] = CTA-pair tile with S K-splits, pair:sk = CTA-pair tile with the
+// stream-K schedule); 0 = let the planner choose.
 int tile_override(const char* name) {
   const char* env = getenv("DCL_GEMM_TILES");
   if (!env) return 0;
@@ -286,6 +287,7 @@ int tile_override(const char* name) {
     const size_t len = e ? (size_t)(e - s) : strlen(s);
     if (len > n && strncmp(s, name, n) == 0 && s[n] == '=') {
       const char* v = s + n + 1;
+      if (strncmp(v, "pair:sk", 7) == 0) return kTilePair | kTileStreamK;
       if (strncmp(v, "pair", 4) == 0) return kTilePair | ((v[4] == ':' ? atoi(v + 5) : 0) << 8);
       return atoi(v);
     }
@@ -361,15 +363,16 @@ dcl_status build_plans(dcl_ctx* c) {
     if (!c->gemm_ws) return fail(c, DCL_ERR_OOM, "split-K workspace allocation failed");
     c->gemm_ws_n = need_w;
   }
-  for (GemmPlan& p : c->plans) {
-    p.flags = c->gemm_flags;
-    p.ws = c->gemm_ws;
-  }
+  for (GemmPlan& p : c->plans)
+    if (gemm_bind_scratch(&p, c->gemm_flags, c->gemm_ws) != cudaSuccess)
+      return fail(c, DCL_ERR_CUDA, "GEMM scratch binding failed");
   return DCL_OK;
 }
 
 // Scratch for a one-off GEMM launch (the single-kernel entry points): allocated here,
 // released by release_scratch after the launch has completed.
+void release_scratch(dcl_ctx* c, GemmPlan* p);
+
 dcl_status attach_scratch(dcl_ctx* c, GemmPlan* p) {
   if (p->flags_needed) {
     p->flags = static_cast<int*>(dev_alloc(c, sizeof(int) * p->flags_needed));
@@ -378,7 +381,15 @@ dcl_status attach_scratch(dcl_ctx* c, GemmPlan* p) {
   }
   if (p->ws_needed) {
     p->ws = static_cast<float*>(dev_alloc(c, sizeof(float) * p->ws_needed));
-    if (!p->ws) return fail(c, DCL_ERR_OOM, "split-K workspace allocation failed");
+    if (!p->ws) {
+      dev_free_one(c, p->flags);
+      p->flags = nullptr;
+      return fail(c, DCL_ERR_OOM, "split-K workspace allocation failed");
+    }
+  }
+  if (gemm_bind_scratch(p, p->flags, p->ws) != cudaSuccess) {
+    release_scratch(c, p);
+    return fail(c, DCL_ERR_CUDA, "GEMM scratch binding failed");
   }
   return DCL_OK;
 }
@@ -914,13 +925,21 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
   EpiParams ep;
   ep.out = part;
   const char* why = nullptr;
-  if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, tile, &why))
+  if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, tile, &why)) {
+    dev_free_one(c, part);
     return fail(c, DCL_ERR_INVALID_ARG, "%s", why ? why : "bad LM-head shape");
+  }
   dcl_status s = attach_scratch(c, &pl);
-  if (s != DCL_OK) return s;
+  if (s != DCL_OK) {
+    dev_free_one(c, part);
+    return s;
+  }
   const cudaError_t e = gemm_launch(pl, c->derr, c->stream);
   release_scratch(c, &pl);
-  if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "LM-head GEMM: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) {
+    dev_free_one(c, part);
+    return fail(c, DCL_ERR_CUDA, "LM-head GEMM: %s", cudaGetErrorString(e));
+  }
   CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, c->stream));
   s = check_device(c);
   dev_free_one(c, part);

@@ -19,6 +19,7 @@
 // DERR_WAIT_TIMEOUT, lets the other roles leave, waits (bounded) for its own copies
 // and MMAs in flight, frees TMEM and returns.
 #include <cudaTypedefs.h>
+#include <string.h>
 
 #include "common.cuh"
 
@@ -182,46 +183,16 @@ __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v
 }
 
 // ------------------------------------------------------------------ epilogues
-// Earlier split-K partials of this thread's row: fp32 tiles stored column-major
-// [256 columns][128 rows] per (tile, CTA half); n = 0 for an unsplit tile.
-struct Parts {
-  const float* base = nullptr;  // partial of split 0
-  size_t stride = 0;            // floats from one split's partial to the next
-  int n = 0;                    // number of earlier splits
-  int row = 0;                  // this thread's row within its 128-row half
-};
+// (one-CTA tiles; the CTA-pair kernel has its own, staged through shared memory)
+struct Parts {};  // no earlier partial sums: one-CTA tiles are never split
 
-// Accumulator columns [col, col + 32) of this thread's row, added to the earlier partials
-// in split order: ((p0 + p1) + ...) + own, so the sum is the same on every run.
-__device__ __forceinline__ void load_cols(uint32_t taddr, int col, float (&v)[32], const Parts& ps) {
+// Accumulator columns [col, col + 32) of this thread's row.
+__device__ __forceinline__ void load_cols(uint32_t taddr, int col, float (&v)[32], const Parts&) {
   uint32_t r[32];
   tmem_ld32(taddr + col, r);
   tmem_ld_wait();
-  if (ps.n == 0) {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
-  } else {
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const float* q = ps.base + (size_t)(col + i) * 128 + ps.row;
-      float a = __ldcg(q);
-      for (int sp = 1; sp < ps.n; ++sp) a += __ldcg(q + sp * ps.stride);
-      v[i] = a + f32(r[i]);
-    }
-  }
-}
-
-// Write this thread's accumulator row as a split-K partial (column-major, see Parts).
-template <int BN>
-__device__ __forceinline__ void store_partial(uint32_t taddr, float* dst, int row) {
-#pragma unroll 1
-  for (int c = 0; c < BN; c += 32) {
-    uint32_t r[32];
-    tmem_ld32(taddr + c, r);
-    tmem_ld_wait();
-#pragma unroll
-    for (int i = 0; i < 32; ++i) __stcg(dst + (size_t)(c + i) * 128 + row, f32(r[i]));
-  }
+  for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
 }
 
 // taddr: TMEM address of (this warp's first lane, accumulator column 0); row: output row
@@ -522,6 +493,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // (32 KB per 64-wide K block instead of 48 KB), the even CTA issues the M = 256 MMAs for
 // both, and each CTA's TMEM receives its 128 rows x 256 columns.  A ring stage holds KA2
 // K blocks (KA2 x 4 MMAs per stage barrier round trip).
+//
+// The epilogue leaves through TMA: each epilogue warp owns 32 output rows and two 4 KB
+// staging boxes (32 rows x 128 bytes, 128-byte swizzle, so that one row per thread is
+// written without bank conflicts); a box is stored (bf16 / fp32 outputs) or added into
+// the fp32 residual stream (cp.reduce.async.bulk .add) by one lane while the warp fills
+// the other box.  Whole 128-byte row segments reach L2 instead of 16-byte pieces of 32
+// different rows.
 #ifndef DCL_PAIR_KA
 #define DCL_PAIR_KA 1
 #endif
@@ -530,8 +508,16 @@ constexpr int A2_STAGE_BYTES = KA2 * A_STAGE_BYTES;
 constexpr int B2_BLOCK_BYTES = 128 * BK * 2;
 constexpr int B2_STAGE_BYTES = KA2 * B2_BLOCK_BYTES;
 constexpr int STAGE2_BYTES = A2_STAGE_BYTES + B2_STAGE_BYTES;
-constexpr int STAGES2 = (7 * 32768) / STAGE2_BYTES;
-constexpr size_t SMEM2 = 1024 + (size_t)STAGES2 * STAGE2_BYTES + 256;
+constexpr int STAGES2 = (6 * 32768) / STAGE2_BYTES;
+constexpr int RING2_BYTES = STAGES2 * STAGE2_BYTES;
+constexpr int BOX_BYTES = 32 * 128;                 // one staging box: 32 rows x 128 bytes
+constexpr int STG2_BYTES = 4 * 2 * BOX_BYTES;       // 4 epilogue warps x 2 boxes
+constexpr int FIX_BOXES = RING2_BYTES / (4 * BOX_BYTES);  // stream-K fix-up boxes per warp
+constexpr int BARS2_BYTES = 640;
+static_assert(16 * STAGES2 + 48 + 8 * 4 * FIX_BOXES <= BARS2_BYTES, "barrier area");
+static_assert(FIX_BOXES >= 2, "fix-up needs two boxes per warp");
+constexpr size_t SMEM2 = 1024 + (size_t)RING2_BYTES + STG2_BYTES + BARS2_BYTES;
+static_assert(SMEM2 <= 232448, "shared memory per CTA");
 constexpr int TMEM2_COLS = 512;
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
@@ -583,11 +569,314 @@ __device__ __forceinline__ void umma_commit_pair(uint32_t bar, uint16_t cta_mask
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
+// 32 consecutive fp32 columns of this thread's TMEM lane, written from registers.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]),
+      "f"(v[9]), "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]),
+      "f"(v[17]), "f"(v[18]), "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]),
+      "f"(v[25]), "f"(v[26]), "f"(v[27]), "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// ---- bulk tensor stores and fences
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
+// global[box] += shared[box] (fp32 adds performed at L2; one writer per element here)
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* tm, uint32_t src, int x, int y) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {  // the smem sources of all but N groups were read
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {  // every group has completed its writes
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+// Order this thread's earlier generic-proxy accesses before its later async-proxy ones.
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+__device__ __forceinline__ float4 ld_shared_v4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr)
+               : "memory");
+  return v;
+}
+// Byte offset of 16-byte chunk k of row r in a 1024-byte-aligned box of 128-byte rows
+// written / read by TMA with 128-byte swizzle.
+__device__ __forceinline__ uint32_t swz(int r, int k) { return (uint32_t)(r * 128 + ((k ^ (r & 7)) << 4)); }
+
+// This lane's row of a staging box: 32 fp32 values, or 32 bf16 values into half h
+// (columns 32h .. 32h + 31) of a 64-column bf16 box.
+__device__ __forceinline__ void stage_f32(uint32_t box, int lane, const float (&v)[32]) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    st_shared_v4(box + swz(lane, k), __float_as_uint(v[4 * k]), __float_as_uint(v[4 * k + 1]),
+                 __float_as_uint(v[4 * k + 2]), __float_as_uint(v[4 * k + 3]));
+}
+__device__ __forceinline__ void stage_bf16(uint32_t box, int lane, int h, const float (&v)[32]) {
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    st_shared_v4(box + swz(lane, 4 * h + k), pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+                 pack_bf16x2(v[8 * k + 4], v[8 * k + 5]), pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
+}
+
+// One epilogue warp's output stream: its 32-row band and its two staging boxes.
+struct Stage {
+  uint32_t box0;   // shared address of this warp's first box (the second follows)
+  int lane;
+  int row0;        // first output row of the band
+  bool live;       // row0 < M (a band wholly below M is not stored)
+  int n;           // boxes issued so far (selects the box)
+  // a free box: the one issued two boxes ago has been read
+  __device__ __forceinline__ uint32_t acquire() {
+    if (lane == 0) bulk_wait_read<1>();
+    __syncwarp();
+    return box0 + (uint32_t)(n & 1) * BOX_BYTES;
+  }
+  // issue the box just filled: a store (or reduce-add) of it at column x of the band
+  __device__ __forceinline__ void issue(const CUtensorMap* tm, uint32_t box, int x, int y, bool reduce) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (live) {
+        if (reduce)
+          tma_reduce_add_2d(tm, box, x, y);
+        else
+          tma_store_2d(tm, box, x, y);
+      }
+      bulk_commit();
+    }
+    ++n;
+  }
+  // every store issued so far has completed and is ordered before later generic
+  // accesses of this warp (before a release that publishes it)
+  __device__ __forceinline__ void drain() {
+    if (lane == 0) {
+      bulk_wait_all();
+      fence_proxy_async_global();
+    }
+    __syncwarp();
+  }
+};
+
+// Accumulator (plus earlier partials) of this warp's 32 rows x 32 columns at col.
+struct Src {
+  uint32_t taddr;        // this warp's TMEM lanes, accumulator column 0
+  bool has_sum = false;  // TMEM at tsum holds the summed earlier stream-K partials
+  uint32_t tsum = 0;     // (TMEM address 0 is a valid address)
+  const float* part = nullptr;  // split-K: earlier splits' partials, row-major [rows][256]
+  size_t part_stride = 0;       // floats between consecutive splits' partials
+  int nparts = 0;
+  int row = 0;                  // this thread's row within the CTA's 128-row half
+};
+__device__ __forceinline__ void src_cols(const Src& s, int col, float (&v)[32]) {
+  uint32_t r[32];
+  tmem_ld32(s.taddr + col, r);
+  if (s.has_sum) {
+    uint32_t q[32];
+    tmem_ld32(s.tsum + col, q);
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = f32(q[i]) + f32(r[i]);
+  } else if (s.nparts > 0) {
+    tmem_ld_wait();
+    const float4* q = reinterpret_cast<const float4*>(s.part + (size_t)s.row * 256 + col);
+    float a[32];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float4 t = __ldcg(q + k);
+      a[4 * k] = t.x, a[4 * k + 1] = t.y, a[4 * k + 2] = t.z, a[4 * k + 3] = t.w;
+    }
+    for (int sp = 1; sp < s.nparts; ++sp) {
+      const float4* qs = reinterpret_cast<const float4*>(s.part + sp * s.part_stride + (size_t)s.row * 256 + col);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float4 t = __ldcg(qs + k);
+        a[4 * k] += t.x, a[4 * k + 1] += t.y, a[4 * k + 2] += t.z, a[4 * k + 3] += t.w;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = a[i] + f32(r[i]);
+  } else {
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+  }
+}
+
+// Accumulator columns [c, c + 64) of the band as one bf16 box at output column x.
+__device__ __forceinline__ void store_bf16_box(const Src& s, Stage& o, const CUtensorMap* tmc, int c, int x) {
+  const uint32_t b = o.acquire();
+#pragma unroll 1
+  for (int h = 0; h < 2; ++h) {
+    float v[32];
+    src_cols(s, c + 32 * h, v);
+    stage_bf16(b, o.lane, h, v);
+  }
+  o.issue(tmc, b, x, o.row0, false);
+}
+
+// The fused epilogues of a 256 x 256 pair tile, for one warp's 32-row band of one CTA
+// half.  All tcgen05.ld run warp-uniformly.
+template <int EPI>
+__device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUtensorMap* tmc, int row, int n_blk,
+                                              int M, int N, const EpiParams& ep) {
+  const int n0 = n_blk * 256;
+  if constexpr (EPI == EPI_BF16) {
+#pragma unroll 1
+    for (int c = 0; c < 256 && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
+  } else if constexpr (EPI == EPI_RESID_F32) {
+#pragma unroll 1
+    for (int c = 0; c < 256; c += 32) {
+      float v[32];
+      src_cols(s, c, v);
+      if (n0 + c >= N) break;
+      const uint32_t b = o.acquire();
+      stage_f32(b, o.lane, v);
+      o.issue(tmc, b, n0 + c, o.row0, true);
+    }
+  } else if constexpr (EPI == EPI_QKV_ROPE) {
+    if (n0 < ep.rope_cols) {
+      const int hd = ep.head_dim, half = hd >> 1;
+      const int pos = row < M ? row % ep.seq_T : 0;
+      const float* cs = ep.rope_cos + (size_t)pos * half;
+      const float* sn = ep.rope_sin + (size_t)pos * half;
+#pragma unroll 1
+      for (int hb = 0; hb < 256; hb += hd) {
+        // rotate-half pairs (j, j + half): hd 128 fills a box with rotated columns
+        // [hb, hb + 64) and one with [hb + 64, hb + 128); hd 64 fills one box [hb, hb + 64)
+        uint32_t b0, b1;
+        if (hd == 128) {  // both boxes free
+          if (o.lane == 0) bulk_wait_read<0>();
+          __syncwarp();
+          b0 = o.box0 + (uint32_t)(o.n & 1) * BOX_BYTES;
+          b1 = o.box0 + (uint32_t)((o.n + 1) & 1) * BOX_BYTES;
+        } else {
+          b0 = b1 = o.acquire();
+        }
+#pragma unroll 1
+        for (int j0 = 0; j0 < half; j0 += 32) {
+          float lo[32], hi[32];
+          src_cols(s, hb + j0, lo);
+          src_cols(s, hb + half + j0, hi);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float c = __ldg(cs + j0 + i), sv = __ldg(sn + j0 + i);
+            const float x = lo[i], y = hi[i];
+            lo[i] = x * c - y * sv;
+            hi[i] = y * c + x * sv;
+          }
+          if (hd == 128) {
+            stage_bf16(b0, o.lane, j0 >> 5, lo);
+            stage_bf16(b1, o.lane, j0 >> 5, hi);
+          } else {
+            stage_bf16(b0, o.lane, 0, lo);
+            stage_bf16(b0, o.lane, 1, hi);
+          }
+        }
+        o.issue(tmc, b0, n0 + hb, o.row0, false);
+        if (hd == 128) o.issue(tmc, b1, n0 + hb + 64, o.row0, false);
+      }
+    } else {
+#pragma unroll 1
+      for (int c = 0; c < 256 && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    // columns [0, 128) of the tile are gate rows, [128, 256) the matching up rows
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 64) {
+      const uint32_t b = o.acquire();
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        float g[32], u[32];
+        src_cols(s, c + 32 * h, g);
+        src_cols(s, 128 + c + 32 * h, u);
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = g[i] / (1.0f + __expf(-g[i])) * u[i];
+        stage_bf16(b, o.lane, h, v);
+      }
+      o.issue(tmc, b, n_blk * 128 + c, o.row0, false);
+    }
+  } else if constexpr (EPI == EPI_LMHEAD) {
+    // Online softmax over this tile's columns (see epilogue_tile); one float4 per row.
+    float m = -INFINITY, sum = 0.f, t2 = -INFINITY;
+    int id = -1;
+#pragma unroll 1
+    for (int c = 0; c < 256; c += 32) {
+      float v[32];
+      src_cols(s, c, v);
+      const int col0 = n0 + c;
+      float cm = m;
+      int cid = id;
+      float c2 = t2;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        if (col0 + i >= ep.vocab) v[i] = -INFINITY;
+        if (v[i] > cm) {
+          c2 = cm;
+          cm = v[i];
+          cid = col0 + i;
+        } else if (v[i] > c2) {
+          c2 = v[i];
+        }
+      }
+      if (cm > -INFINITY) {
+        const float mb = cm * kLog2e;
+        float acc = sum * exp2f(m * kLog2e - mb);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], kLog2e, -mb));
+        sum = acc;
+      }
+      m = cm;
+      id = cid;
+      t2 = c2;
+    }
+    if (row < M) {
+      const int nblk = (N + 255) / 256;
+      float4* part = reinterpret_cast<float4*>(ep.out);
+      part[(size_t)row * nblk + n_blk] = make_float4(m, sum, __int_as_float(id), t2);
+    }
+  }
+}
+
+// This warp's 32 rows x 256 columns of the accumulator, stored as an fp32 partial
+// (rows y0 .. y0 + 31 of the workspace, [rows][256]).
+__device__ __forceinline__ void store_partial_pair(const Src& s, Stage& o, const CUtensorMap* tmw, int y0) {
+  const bool live = o.live;
+  o.live = true;  // partials are stored for every band
+#pragma unroll 1
+  for (int c = 0; c < 256; c += 32) {
+    float v[32];
+    src_cols(s, c, v);
+    const uint32_t b = o.acquire();
+    stage_f32(b, o.lane, v);
+    o.issue(tmw, b, c, y0, false);
+  }
+  o.live = live;
+}
 
 __device__ __forceinline__ void epilogue_bar() {  // the 128 epilogue threads (warps 2..5)
   asm volatile("bar.sync 1, 128;" ::: "memory");
 }
-// Bounded wait until the split-K counter at f reaches target; false on timeout or abort.
+// Bounded wait until the counter at f reaches target; false on timeout or abort.
 __device__ __noinline__ bool wait_flag_geq(const int* f, int target, volatile int* abort_flag) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
@@ -604,42 +893,186 @@ __device__ __noinline__ bool wait_flag_geq(const int* f, int target, volatile in
   }
 }
 
-// Work items w = split * tiles + tile (split-major), each a contiguous range of K blocks.
-// Split-K results are combined in split order, so every run gives the same bits:
-//   residual epilogue: split s adds its accumulator to h after split s-1 has (a per-tile
-//     counter, released by each split and reset by the last);
-//   other epilogues: splits < S-1 store fp32 partials, the last split waits for all of
-//     them, sums them in order with its own accumulator and runs the epilogue.
-// Split 0 never waits and each CTA pair takes items in increasing order with every CTA
-// resident (grid <= SMs, one CTA per SM), so the waits always end.
+// Stream-K fix-up, per epilogue warp.  A tile's last K segment is its CTA pair's last
+// work item, so when it is reached the operand ring is idle in both CTAs and the second
+// TMEM accumulator is free.  Each warp streams the n earlier partials of its 32 rows
+// through FIX_BOXES boxes of its quarter of the ring (TMA loads of 32 rows x 32 fp32,
+// 128-byte swizzle; column-chunk-major, partial-minor), sums each element in K order
+// p0 + p1 + ... and writes the sum to TMEM at tsum, for the epilogue to add its own
+// accumulator last.  Returns false (with *abort_flag set) if a box did not arrive in time;
+// the result is warp-uniform.
+__device__ __noinline__ bool fixup_to_tmem(const CUtensorMap* tmw, int y0, int slot_rows, int n, uint32_t ring,
+                                           uint32_t bar0, uint32_t tsum, int lane, volatile int* abort_flag,
+                                           int* err) {
+  const int total = 8 * n;
+  if (lane == 0) {
+    fence_proxy_async_global();  // the partials were published to this CTA (acquire + barrier)
+    for (int p = 0; p < total && p < FIX_BOXES; ++p) {
+      mbar_arrive_expect_tx(bar0 + 8 * p, BOX_BYTES);
+      tma_load_2d(ring + p * BOX_BYTES, tmw, (p / n) * 32, y0 + (p % n) * slot_rows, bar0 + 8 * p);
+    }
+  }
+  bool ok = true;
+#pragma unroll 1
+  for (int j = 0; j < 8; ++j) {
+    float a[32];
+#pragma unroll 1
+    for (int sl = 0; sl < n; ++sl) {
+      const int p = j * n + sl, b = p % FIX_BOXES;
+      if (ok && !mbar_wait(bar0 + 8 * b, (uint32_t)(p / FIX_BOXES) & 1u, abort_flag)) ok = false;
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok) {
+        const uint32_t box = ring + b * BOX_BYTES;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const float4 t = ld_shared_v4(box + swz(lane, k));
+          if (sl == 0) {
+            a[4 * k] = t.x, a[4 * k + 1] = t.y, a[4 * k + 2] = t.z, a[4 * k + 3] = t.w;
+          } else {
+            a[4 * k] += t.x, a[4 * k + 1] += t.y, a[4 * k + 2] += t.z, a[4 * k + 3] += t.w;
+          }
+        }
+      }
+      fence_proxy_async_smem();  // this lane's reads of box b before its refill
+      __syncwarp();
+      const int nxt = p + FIX_BOXES;
+      if (lane == 0 && ok && nxt < total) {
+        mbar_arrive_expect_tx(bar0 + 8 * b, BOX_BYTES);
+        tma_load_2d(ring + b * BOX_BYTES, tmw, (nxt / n) * 32, y0 + (nxt % n) * slot_rows, bar0 + 8 * b);
+      }
+    }
+    if (ok) tmem_st32(tsum + j * 32, a);
+  }
+  tmem_st_wait();
+  if (!ok) {
+    *abort_flag = 1;
+    report_error(err, DERR_WAIT_TIMEOUT);
+  }
+  return ok;
+}
+
+// ---- work items of a CTA pair ------------------------------------------------------
+// A work item is a tile and a range [ku0, ku1) of its K units (KA2 K blocks each).
+//   plain    : pair c takes tiles c, c + C, ...  (C pairs)
+//   split-K  : items w = split * tiles + tile (split-major), pair c takes w = c, c + C, ...
+//   stream-K : the first (tiles / C) * C tiles as plain rounds; the R left-over tiles'
+//              R * U K units are then cut into C equal contiguous ranges, one per pair.
+//              A range covers the tail of one tile and/or the head of the next; the pair
+//              processes the head first (it only writes a partial) and the tail second
+//              (the tile's last segment: it waits for the other segments' partials, sums
+//              them in K order and runs the epilogue), so no pair waits on a pair that is
+//              itself waiting.
+enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3 };
+struct Sched {
+  int tiles, ku, C, splits, streamk;
+};
+struct Item {
+  int t, ku0, ku1, kind;
+  int sp;     // IT_SPLIT: split index
+  int rel;    // IT_PART / IT_LAST: stream-K tile index (0..R-1)
+  int slot;   // IT_PART: partial slot; IT_LAST: number of earlier segments
+};
+
+__device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& it) {
+  if (s.splits > 1) {
+    const long w = (long)c + (long)idx * s.C;
+    if (w >= (long)s.tiles * s.splits) return false;
+    it.sp = (int)(w / s.tiles);
+    it.t = (int)(w % s.tiles);
+    it.ku0 = (int)((long)it.sp * s.ku / s.splits);
+    it.ku1 = (int)((long)(it.sp + 1) * s.ku / s.splits);
+    it.kind = IT_SPLIT;
+    return true;
+  }
+  const int rounds = s.streamk ? s.tiles / s.C : (s.tiles + s.C - 1) / s.C;
+  if (idx < rounds) {
+    it.t = c + idx * s.C;
+    if (it.t >= s.tiles) return false;
+    it.ku0 = 0;
+    it.ku1 = s.ku;
+    it.kind = IT_PLAIN;
+    return true;
+  }
+  if (!s.streamk) return false;
+  const int first = rounds * s.C;
+  const long RU = (long)(s.tiles - first) * s.ku;
+  const long lo = (long)c * RU / s.C, hi = (long)(c + 1) * RU / s.C;
+  if (hi <= lo) return false;
+  const int ta = (int)(lo / s.ku), tb = (int)((hi - 1) / s.ku);
+  const int k = idx - rounds;
+  int rel, k0, k1;
+  if (ta == tb) {
+    if (k > 0) return false;
+    rel = ta;
+    k0 = (int)(lo - (long)ta * s.ku);
+    k1 = (int)(hi - (long)ta * s.ku);
+  } else if (k == 0) {  // head of the later tile first
+    rel = tb;
+    k0 = 0;
+    k1 = (int)(hi - (long)tb * s.ku);
+  } else if (k == 1) {  // then the tail of the earlier tile
+    rel = ta;
+    k0 = (int)(lo - (long)ta * s.ku);
+    k1 = s.ku;
+  } else {
+    return false;
+  }
+  const int c_first = (int)((((long)rel * s.ku + 1) * s.C - 1) / RU);  // owner of the tile's first unit
+  it.t = first + rel;
+  it.rel = rel;
+  it.ku0 = k0;
+  it.ku1 = k1;
+  it.kind = (k1 == s.ku) ? IT_LAST : IT_PART;
+  it.slot = c - c_first;
+  return true;
+}
+
+// Work items are taken in the order above by the producer, the MMA issuer and the
+// epilogue alike.  Combination rules, all bit-reproducible:
+//   split-K, residual epilogue: split s adds its accumulator to h after split s-1 has
+//     (a per-tile counter, released by each split and reset by the last);
+//   split-K, other epilogues: splits < S-1 store fp32 partials, the last split waits for
+//     all of them, sums them in order with its own accumulator and runs the epilogue;
+//   stream-K: as split-K's second rule, per left-over tile, the sum formed in TMEM.
+// Partials are fp32 [rows][256] in the workspace: row ((tile * S + slot) * 2 + rank) * 128
+// + r holds row r of CTA `rank`'s half of the tile (S slots per tile).  Items that are
+// waited on never wait themselves before they publish, and every CTA is resident (grid <=
+// SMs, one CTA per SM), so every wait ends.
 template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, int M,
-                    int N, int K, EpiParams ep, int splits, int* flags, float* ws, int* err) {
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
+                    const __grid_constant__ CUtensorMap tmc, const __grid_constant__ CUtensorMap tmw, int M,
+                    int N, int K, EpiParams ep, int splits, int streamk, int ws_slots, int* flags, float* ws,
+                    int* err) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
   const uint32_t sA = base;
   const uint32_t sB = base + STAGES2 * A2_STAGE_BYTES;
-  const uint32_t bars = sB + STAGES2 * B2_STAGE_BYTES;
+  const uint32_t stg = base + RING2_BYTES;
+  const uint32_t bars = stg + STG2_BYTES;
   const uint32_t full0 = bars;
   const uint32_t empty0 = bars + 8 * STAGES2;
   const uint32_t tfull0 = bars + 16 * STAGES2;
   const uint32_t tempty0 = tfull0 + 16;
   const uint32_t drain = tempty0 + 16;
   const uint32_t holder = drain + 8;
+  const uint32_t fix0 = holder + 8;  // 4 x FIX_BOXES stream-K fix-up barriers
   volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
-  const int cluster = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+  const int cluster = blockIdx.x >> 1;
   const int num_m = (M + 255) / 256;
   const int num_n = (N + 255) / 256;
-  const int num_tiles = num_m * num_n;
-  const int num_items = num_tiles * splits;
-  const int num_ku = (K + BK * KA2 - 1) / (BK * KA2);  // ring stages of KA2 K blocks each
+  Sched sc;
+  sc.tiles = num_m * num_n;
+  sc.ku = (K + BK * KA2 - 1) / (BK * KA2);
+  sc.C = gridDim.x >> 1;
+  sc.splits = splits;
+  sc.streamk = streamk;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
@@ -651,6 +1084,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     mbar_init(tempty0, 8);  // 4 epilogue warps x 2 CTAs (used in the leader)
     mbar_init(tempty0 + 8, 8);
     mbar_init(drain, 1);
+    for (int b = 0; b < 4 * FIX_BOXES; ++b) mbar_init(fix0 + 8 * b, 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tma);
@@ -669,11 +1103,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int w = cluster; w < num_items && ok; w += n_clusters) {
-        const int sp = w / num_tiles, t = w % num_tiles;
-        const int m_blk = t % num_m, n_blk = t / num_m;
-        const int kb0 = (int)((long)sp * num_ku / splits) * KA2;
-        const int kb1 = (int)((long)(sp + 1) * num_ku / splits) * KA2;
+      Item it;
+      for (int idx = 0; ok && next_item(idx, sc, cluster, it); ++idx) {
+        const int m_blk = it.t % num_m, n_blk = it.t / num_m;
+        const int kb0 = it.ku0 * KA2, kb1 = it.ku1 * KA2;
         const int wrow = n_blk * 256 + (int)rank * 128;  // this CTA's half of the weight tile
         for (int kb = kb0; kb < kb1 && kb < kb0 + kPrefetchAhead; ++kb) tma_prefetch_l2(&tmb, kb * BK, wrow);
         for (int kb = kb0; kb < kb1; kb += KA2) {
@@ -709,13 +1142,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      int j = 0;
-      for (int w = cluster; w < num_items && ok; w += n_clusters, ++j) {
-        const int sp = w / num_tiles;
-        const int kb0 = (int)((long)sp * num_ku / splits) * KA2;
-        const int kb1 = (int)((long)(sp + 1) * num_ku / splits) * KA2;
-        const int ab = j & 1;
-        const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+      Item it;
+      for (int idx = 0; ok && next_item(idx, sc, cluster, it); ++idx) {
+        const int kb0 = it.ku0 * KA2, kb1 = it.ku1 * KA2;
+        const int ab = idx & 1;
+        const uint32_t aph = (uint32_t)(idx >> 1) & 1u;
         if (!mbar_wait(tempty0 + 8 * ab, aph ^ 1u, abort_flag)) {
           ok = false;
           break;
@@ -756,28 +1187,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ------------------------------------------------ epilogue warps 2..5 (both CTAs)
-    const int q = warp & 3;
+    const int q = warp & 3;                 // TMEM lane quarter = 32-row band of this warp
     const int et = (warp - 2) * 32 + lane;  // 0..127
     const int row_local = q * 32 + lane;
-    const size_t part_floats = (size_t)256 * 128;                 // one CTA half of a tile
-    const size_t split_stride = (size_t)num_tiles * 2 * part_floats;
-    int j = 0;
-    for (int w = cluster; w < num_items; w += n_clusters, ++j) {
-      const int sp = w / num_tiles, t = w % num_tiles;
-      const int ab = j & 1;
-      const uint32_t aph = (uint32_t)(j >> 1) & 1u;
+    Stage o;
+    o.box0 = stg + (uint32_t)(q * 2 * BOX_BYTES);
+    o.lane = lane;
+    o.n = 0;
+    Item it;
+    for (int idx = 0; next_item(idx, sc, cluster, it); ++idx) {
+      const int ab = idx & 1;
+      const uint32_t aph = (uint32_t)(idx >> 1) & 1u;
       if (!mbar_wait(tfull0 + 8 * ab, aph, abort_flag)) {
         *abort_flag = 1;
         report_error(err, DERR_WAIT_TIMEOUT);
         break;
       }
       tc_fence_after();
+      const int t = it.t;
       const int m_blk = t % num_m, n_blk = t / num_m;
       const int row = m_blk * 256 + (int)rank * 128 + row_local;
-      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
-      if (splits == 1) {
-        epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, Parts{});
-      } else {
+      o.row0 = m_blk * 256 + (int)rank * 128 + q * 32;
+      o.live = o.row0 < M;
+      Src s;
+      s.taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
+      s.row = row_local;
+      if (it.kind == IT_PLAIN) {
+        epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+      } else if (it.kind == IT_SPLIT) {
+        const int sp = it.sp;
         int* flag = flags + t * 2 + rank;
         if constexpr (EPI == EPI_RESID_F32) {
           if (et == 0 && !wait_flag_geq(flag, sp, abort_flag)) {
@@ -785,43 +1223,75 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             report_error(err, DERR_WAIT_TIMEOUT);
           }
           epilogue_bar();
-          if (!*abort_flag) epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, Parts{});
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+          o.drain();
           epilogue_bar();
           if (et == 0) {
             __threadfence();
             atomicExch(flag, sp + 1 == splits ? 0 : sp + 1);
           }
         } else {
-          float* part0 = ws + ((size_t)t * 2 + rank) * part_floats;
-          if (sp < splits - 1) {
-            store_partial<256>(taddr, part0 + sp * split_stride, row_local);
+          const int S1 = splits - 1;
+          if (sp < S1) {
+            store_partial_pair(s, o, &tmw, ((t * S1 + sp) * 2 + (int)rank) * 128 + q * 32);
+            o.drain();
             epilogue_bar();
             if (et == 0) {
               __threadfence();
               atomicAdd(flag, 1);
             }
           } else {
-            if (et == 0 && !wait_flag_geq(flag, splits - 1, abort_flag)) {
+            if (et == 0 && !wait_flag_geq(flag, S1, abort_flag)) {
               *abort_flag = 1;
               report_error(err, DERR_WAIT_TIMEOUT);
             }
             epilogue_bar();
             __threadfence();
-            Parts ps;
-            ps.base = part0;
-            ps.stride = split_stride;
-            ps.n = splits - 1;
-            ps.row = row_local;
-            if (!*abort_flag) epilogue_tile<256, EPI>(taddr, row, n_blk, M, N, ep, ps);
+            s.part = ws + ((size_t)t * S1 * 2 + rank) * 128 * 256;
+            s.part_stride = (size_t)2 * 128 * 256;
+            s.nparts = S1;
+            if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
             epilogue_bar();
             if (et == 0) atomicExch(flag, 0);
           }
+        }
+      } else {
+        // stream-K segment of left-over tile it.rel
+        int* flag = flags + it.rel * 2 + rank;
+        const int y_slot0 = ((it.rel * ws_slots) * 2 + (int)rank) * 128 + q * 32;
+        if (it.kind == IT_PART) {
+          store_partial_pair(s, o, &tmw, y_slot0 + it.slot * 256);
+          o.drain();
+          epilogue_bar();
+          if (et == 0) {
+            __threadfence();
+            atomicAdd(flag, 1);
+          }
+        } else {
+          if (et == 0 && it.slot > 0 && !wait_flag_geq(flag, it.slot, abort_flag)) {
+            *abort_flag = 1;
+            report_error(err, DERR_WAIT_TIMEOUT);
+          }
+          epilogue_bar();
+          if (it.slot > 0 && !*abort_flag) {
+            const uint32_t tsum = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)((ab ^ 1) * 256);
+            if (fixup_to_tmem(&tmw, y_slot0, 256, it.slot, base + (uint32_t)(q * (RING2_BYTES / 4)),
+                              fix0 + (uint32_t)(q * 8 * FIX_BOXES), tsum, lane, abort_flag, err)) {
+              s.has_sum = true;
+              s.tsum = tsum;
+            }
+          }
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+          epilogue_bar();
+          if (et == 0) atomicExch(flag, 0);
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(mapa_shared(tempty0 + 8 * ab, 0));
     }
+    if (lane == 0) bulk_wait_all();  // the staging boxes outlive every store reading them
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -860,6 +1330,19 @@ bool encode_kmajor(CUtensorMap* tm, const void* ptr, int rows, int k, int box_ro
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Row-major [rows][cols] output / workspace seen in boxes of 32 rows x 128 bytes with
+// 128-byte swizzle (the pair epilogue's staging layout).
+bool encode_rows(CUtensorMap* tm, void* ptr, CUtensorMapDataType dt, int esize, long rows, long cols, long ld) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * esize};
+  cuuint32_t box[2] = {(cuuint32_t)(128 / esize), 32};
+  cuuint32_t es[2] = {1, 1};
+  return fn(tm, dt, 2, ptr, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN, int EPI>
 cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
   static bool attr_set = false;
@@ -883,7 +1366,8 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, p.splits, p.flags, p.ws, err);
+  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.tc, p.tw, p.M, p.N, p.K, p.ep, p.splits, p.streamk,
+                                                p.ws_slots, p.flags, p.ws, err);
   return cudaGetLastError();
 }
 
@@ -909,26 +1393,43 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   }
   // Tile choice (measured on the LLaDA-8B step's shapes): the CTA-pair tile keeps the
   // tensor pipe busiest and is used whenever M spans more than one 128-row tile; a
-  // residual GEMM with too few pair tiles to fill the GPU (N = d_model) instead uses
-  // one-CTA 128 x 128 tiles when K is short, or the pair tile with K split in two when K
-  // is long; small M uses one-CTA tiles, 256 or 128 wide by wave fill.
+  // residual GEMM whose pair tiles fill less than 3/4 of the GPU and whose K is long
+  // splits K in two; small M uses one-CTA tiles, 256 or 128 wide by wave fill.  Stream-K
+  // is available on request (kTileStreamK): with a fix-up that reads (segments - 1) fp32
+  // partials of 256 KB per tile it lost to the plain schedule on those shapes.
   const bool pair_forced = (tile & 0xff) == kTilePair;
-  int bn = pair_forced ? kTilePair : tile, cg = 1, splits = 1;
-  const int forced_splits = pair_forced ? (tile >> 8) : 0;
+  const bool sk_forced = pair_forced && (tile & kTileStreamK);
+  int bn = pair_forced ? kTilePair : (tile & 0xff), cg = 1, splits = 1, streamk = 0;
+  const int forced_splits = pair_forced ? ((tile >> 8) & 0xff) : 0;
   const long nkb = (K + BK - 1) / BK;
-  const long m1 = (M + BM - 1) / BM, m2 = (M + 255) / 256;
-  const long pair_tiles = m2 * ((N + 255) / 256);
+  const long m1 = (M + BM - 1) / BM;
   const bool wide_only = (epi == EPI_SWIGLU || epi == EPI_LMHEAD);
+  const int pairs = num_sms / 2;
+  const long units = (K + BK * KA2 - 1) / (BK * KA2);
+  const long pair_tiles = (long)((M + 255) / 256) * ((N + 255) / 256);
+  const long left = pairs > 0 ? pair_tiles % pairs : 0;
+  if (pair_forced && pairs < 1) {
+    *why = "gemm: the CTA-pair tile needs two SMs";
+    return cudaErrorInvalidValue;
+  }
   if (bn == kTilePair) {
     bn = 256;
     cg = 2;
     splits = forced_splits > 0 ? forced_splits : 1;
+    if (sk_forced) {
+      if (forced_splits > 1 || left == 0 || left * units < pairs) {
+        *why = "gemm: stream-K needs one split and a partial last round of at least one K unit per pair";
+        return cudaErrorInvalidValue;
+      }
+      streamk = 1;
+    } else if (forced_splits == 0) {
+      splits = (epi == EPI_RESID_F32 && 4 * pair_tiles < 3L * pairs && nkb >= 128) ? 2 : 1;
+    }
   } else if (bn == 0) {
-    const bool sparse = 4 * pair_tiles < 3 * (num_sms / 2);
-    if (M > BM && num_sms >= 2 && !(epi == EPI_RESID_F32 && sparse && nkb < 128)) {
+    if (M > BM && pairs >= 1) {
       bn = 256;
       cg = 2;
-      splits = (epi == EPI_RESID_F32 && sparse && nkb >= 128) ? 2 : 1;
+      splits = (epi == EPI_RESID_F32 && 4 * pair_tiles < 3L * pairs && nkb >= 128) ? 2 : 1;
     } else if (wide_only) {
       bn = 256;
     } else {
@@ -972,24 +1473,67 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     return cudaErrorInvalidValue;
   }
   plan->splits = splits;
+  plan->streamk = streamk;
+  plan->ws_slots = 0;
   plan->flags_needed = 0;
   plan->ws_needed = 0;
   plan->flags = nullptr;
   plan->ws = nullptr;
+  memset(&plan->tc, 0, sizeof(plan->tc));
+  memset(&plan->tw, 0, sizeof(plan->tw));
+  if (cg == 2 && epi != EPI_LMHEAD) {
+    const bool f32 = (epi == EPI_RESID_F32);
+    const int es = f32 ? 4 : 2;
+    const long cols = (epi == EPI_SWIGLU) ? N / 2 : N;
+    if ((reinterpret_cast<uintptr_t>(ep.out) & 15) || ((long)ep.ldo * es) % 16 != 0 || ep.ldo < cols) {
+      *why = "gemm: the output must be 16-byte aligned with a row pitch of a multiple of 16 bytes";
+      return cudaErrorInvalidValue;
+    }
+    if (!encode_rows(&plan->tc, ep.out, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, es,
+                     M, cols, ep.ldo)) {
+      *why = "gemm: cuTensorMapEncodeTiled failed (output)";
+      return cudaErrorInvalidValue;
+    }
+  }
   if (cg == 2) {
-    plan->n_tiles = ((M + 255) / 256) * ((N + 255) / 256);
-    const int pairs = num_sms / 2;
-    const int items = plan->n_tiles * splits;
-    plan->grid = 2 * (items < pairs ? items : pairs);
+    plan->n_tiles = (int)pair_tiles;
+    const long items = streamk ? pairs : pair_tiles * splits;
+    plan->grid = 2 * (int)(items < pairs ? items : pairs);
     plan->smem = SMEM2;
     if (splits > 1) {
       plan->flags_needed = (size_t)plan->n_tiles * 2;
       if (epi != EPI_RESID_F32) plan->ws_needed = (size_t)(splits - 1) * plan->n_tiles * 2 * 256 * 128;
     }
+    if (streamk) {
+      // left-over tile r's K units [r*U, (r+1)*U) are owned by pairs
+      // owner(r*U) .. owner((r+1)*U - 1), owner(u) = ((u + 1) * C - 1) / (R * U); all
+      // but the last write a partial slot
+      const long RU = left * units;
+      long slots = 1;
+      for (long r = 0; r < left; ++r) {
+        const long c0 = ((r * units + 1) * pairs - 1) / RU;
+        const long c1 = (((r + 1) * units) * pairs - 1) / RU;
+        slots = (c1 - c0) > slots ? (c1 - c0) : slots;
+      }
+      plan->ws_slots = (int)slots;
+      plan->flags_needed = (size_t)left * 2;
+      plan->ws_needed = (size_t)left * slots * 2 * 256 * 128;
+    }
   } else {
     plan->n_tiles = ((M + BM - 1) / BM) * ((N + bn - 1) / bn);
     plan->grid = plan->n_tiles < num_sms ? plan->n_tiles : num_sms;
     plan->smem = (bn == 256) ? Cfg<256>::SMEM : Cfg<128>::SMEM;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t gemm_bind_scratch(GemmPlan* p, int* flags, float* ws) {
+  p->flags = flags;
+  p->ws = ws;
+  if (p->cg == 2 && p->ws_needed) {
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 15)) return cudaErrorInvalidValue;
+    if (!encode_rows(&p->tw, ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (long)(p->ws_needed / 256), 256, 256))
+      return cudaErrorInvalidValue;
   }
   return cudaSuccess;
 }

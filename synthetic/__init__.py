@@ -18,14 +18,16 @@ take their inputs from it:
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
 import dataclasses
 import math
+import os
 
 import numpy as np
 
 __all__ = [
     "ModelShape", "SHAPES", "TensorKind", "tensor_id", "splitmix64",
-    "weight_values", "bf16_bits", "bf16_to_f32", "round_bf16",
+    "weight_values", "embed_rows", "bf16_bits", "bf16_to_f32", "round_bf16",
     "model_weights", "prompt_ids", "accept_inputs", "GEN_SIGMA4",
 ]
 
@@ -114,17 +116,58 @@ def weight_values(seed: int, tid: int, start: int, count: int, std: float,
     """
     if not (0 <= seed < 65536 and 0 <= tid < 65536 and start >= 0 and start + count <= 2 ** 32):
         raise ValueError("generator counter out of range")
-    idx = np.arange(start, start + count, dtype=np.uint64)
-    key = (np.uint64(seed) << np.uint64(48)) | (np.uint64(tid) << np.uint64(32)) | idx
-    h = splitmix64(key)
-    m16 = np.uint64(0xFFFF)
-    s = ((h & m16) + ((h >> np.uint64(16)) & m16) + ((h >> np.uint64(32)) & m16)
-         + (h >> np.uint64(48))).astype(np.int64)
+    out = np.empty(count, np.float32)
+    threads = min(16, os.cpu_count() or 1)
+    if count < (1 << 22) or threads == 1:
+        _weight_chunks(seed, tid, start, count, std, mean, out)
+    else:  # elementwise and counter-based: independent sub-ranges, numpy releases the GIL
+        step = -(-count // threads)
+
+        def job(i):
+            a, b = i * step, min(count, (i + 1) * step)
+            if a < b:
+                _weight_chunks(seed, tid, start + a, b - a, std, mean, out[a:b])
+
+        with cf.ThreadPoolExecutor(threads) as ex:
+            list(ex.map(job, range(threads)))
+    return out
+
+
+def _weight_chunks(seed, tid, start, count, std, mean, out):
+    """weight_values written into out (float32 [count]), in cache-sized chunks with
+    in-place integer steps."""
+    hi = (np.uint64(seed) << np.uint64(48)) | (np.uint64(tid) << np.uint64(32))
     std32 = float(np.float32(std))        # the C ABI receives std as a float
-    w = (s - GEN_MEAN4).astype(np.float32) * np.float32(std32 / GEN_SIGMA4)
-    if mean != 0.0:
-        w = w + np.float32(mean)
-    return round_bf16(w)
+    scale = np.float32(std32 / GEN_SIGMA4)
+    m16 = np.uint64(0xFFFF)
+    chunk = 1 << 16
+    for c0 in range(0, count, chunk):
+        n = min(chunk, count - c0)
+        z = np.arange(start + c0, start + c0 + n, dtype=np.uint64)
+        z |= hi                                       # key = seed << 48 | tid << 32 | index
+        t = np.empty_like(z)
+        with np.errstate(over="ignore"):              # SplitMix64, as splitmix64() above
+            z += _GOLDEN
+            np.right_shift(z, np.uint64(30), out=t)
+            z ^= t
+            z *= _M1
+            np.right_shift(z, np.uint64(27), out=t)
+            z ^= t
+            z *= _M2
+            np.right_shift(z, np.uint64(31), out=t)
+            z ^= t
+        s = z & m16                                   # sum of the four 16-bit fields
+        for sh in (16, 32):
+            np.right_shift(z, np.uint64(sh), out=t)
+            t &= m16
+            s += t
+        np.right_shift(z, np.uint64(48), out=t)
+        s += t
+        w = (s.view(np.int64) - GEN_MEAN4).astype(np.float32)
+        w *= scale
+        if mean != 0.0:
+            w += np.float32(mean)
+        out[c0:c0 + n] = round_bf16(w)
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -146,11 +189,12 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 
 def model_weights(shape: ModelShape, seed: int, std: float = 0.02,
                   lm_head_scale: float = 1.0, norm_gain_std: float = 0.0,
-                  layers=None) -> dict:
+                  layers=None, global_tensors: bool = True) -> dict:
     """Weights of ``shape`` from the counter-based generator, as bf16-exact float32.
 
     Matrices are [out][in] (the nn.Linear layout).  Norm gains are 1 + N(0, norm_gain_std).
-    ``layers`` restricts the per-layer tensors generated (all by default).
+    ``layers`` restricts the per-layer tensors generated (all by default);
+    ``global_tensors=False`` leaves out the embedding, final norm and LM head (None).
     """
     d, hd, H, G, F, V = (shape.d_model, shape.head_dim, shape.n_heads,
                          shape.n_kv_heads, shape.ffn_dim, shape.vocab)
@@ -175,13 +219,30 @@ def model_weights(shape: ModelShape, seed: int, std: float = 0.02,
     names = {TensorKind.ATTN_NORM: "attn_norm", TensorKind.WQ: "wq", TensorKind.WK: "wk",
              TensorKind.WV: "wv", TensorKind.WO: "wo", TensorKind.MLP_NORM: "mlp_norm",
              TensorKind.W_GATE: "w_gate", TensorKind.W_UP: "w_up", TensorKind.W_DOWN: "w_down"}
-    out = {"embed": gen(TensorKind.EMBED, 0), "final_norm": gen(TensorKind.FINAL_NORM, 0),
-           "lm_head": gen(TensorKind.LM_HEAD, 0), "layers": []}
+    if global_tensors:
+        out = {"embed": gen(TensorKind.EMBED, 0), "final_norm": gen(TensorKind.FINAL_NORM, 0),
+               "lm_head": gen(TensorKind.LM_HEAD, 0), "layers": []}
+    else:
+        out = {"embed": None, "final_norm": None, "lm_head": None, "layers": []}
     for li in range(shape.n_layers):
         if layers is not None and li not in layers:
             out["layers"].append(None)
             continue
         out["layers"].append({names[k]: gen(k, li) for k in names})
+    return out
+
+
+def embed_rows(shape: ModelShape, seed: int, ids, std: float = 0.02) -> np.ndarray:
+    """Rows ``ids`` of the embedding table of ``model_weights(shape, seed, std)`` (float32
+    [len(ids)][d]) without generating the whole table."""
+    d = shape.d_model
+    tid = tensor_id(TensorKind.EMBED, 0)
+    ids = np.asarray(ids, dtype=np.int64).reshape(-1)
+    out = np.empty((len(ids), d), np.float32)
+    for r, i in enumerate(ids):
+        if not 0 <= i < shape.vocab:
+            raise ValueError("token id out of range")
+        out[r] = weight_values(seed, tid, int(i) * d, d, std)
     return out
 
 

@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 import torch
 
+import paper_2607_20467_gb300 as dcl
 import synthetic as syn
 from oracle import model
 
@@ -18,7 +19,6 @@ pytestmark = pytest.mark.gpu
 def ops():
     import __graft_entry__
     __graft_entry__.build()
-    import paper_2607_20467_gb300 as dcl
     ctx = dcl.Context(None, 1, 1)
     yield ctx
     ctx.close()
@@ -62,24 +62,42 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
-# auto, one-CTA 128 / 256 columns, CTA pair 256 x 256, CTA pair with 2 / 3 K splits
-TILES = [0, 128, 256, 2, 2 | (2 << 8), 2 | (3 << 8)]
+PAIR, SK = 2, 1 << 16
+# auto, one-CTA 128 / 256 columns, CTA pair (library's K schedule), CTA pair unsplit,
+# CTA pair with 2 / 3 K splits, CTA pair with the stream-K schedule
+TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK]
 
 
 def _splits(tile):
-    return (tile >> 8) if (tile & 0xff) == 2 else 1
+    return max(1, (tile >> 8) & 0xff) if (tile & 0xff) == PAIR else 1
+
+
+def _streamk_possible(M, N, K):
+    """Stream-K needs a partly filled last round of pair tiles with at least one 64-wide
+    K block per CTA pair."""
+    pairs = torch.cuda.get_device_properties(0).multi_processor_count // 2
+    left = ((M + 255) // 256) * ((N + 255) // 256) % pairs
+    return left > 0 and left * (K // 64) >= pairs
+
+
+def _unsupported(M, N, K, tile):
+    """True when the tile choice cannot run this shape (then the call must be refused)."""
+    return K // 64 < _splits(tile) or (tile & SK and not _streamk_possible(M, N, K))
 
 
 @pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("M,N,K", [(96, 768, 256), (128, 256, 64), (300, 512, 1024), (1, 128, 64),
-                                   (257, 384, 192), (512, 4096, 4096), (200, 1024, 12288)])
+                                   (257, 384, 192), (512, 4096, 4096), (200, 1024, 12288),
+                                   (300, 1280, 4096)])
 def test_linear_bf16(ops, M, N, K, tile):
-    if K // 64 < _splits(tile):
-        pytest.skip("fewer K blocks than splits")
     rng = np.random.default_rng(M + N + K)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
     out = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    if _unsupported(M, N, K, tile):
+        with pytest.raises(dcl.DcleapError):
+            ops.op_linear(_bf16(a), _bf16(w), out, mode=0, tile=tile)
+        return
     ops.op_linear(_bf16(a), _bf16(w), out, mode=0, tile=tile)
     torch.cuda.synchronize()
     ref = a.astype(np.float64) @ w.astype(np.float64).T
@@ -90,24 +108,28 @@ def test_linear_bf16(ops, M, N, K, tile):
 
 
 @pytest.mark.parametrize("tile", TILES)
-@pytest.mark.parametrize("M,N,K", [(96, 256, 256), (512, 4096, 4096), (70, 3584, 3584)])
+@pytest.mark.parametrize("M,N,K", [(96, 256, 256), (512, 4096, 4096), (70, 3584, 3584), (300, 1280, 4096)])
 def test_linear_residual(ops, M, N, K, tile):
-    if K // 64 < _splits(tile):
-        pytest.skip("fewer K blocks than splits")
     rng = np.random.default_rng(7 * M + N)
     a = syn.round_bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
     w = syn.round_bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
     h0 = rng.normal(0, 2, (M, N)).astype(np.float32)
     h = torch.from_numpy(h0).cuda()
+    if _unsupported(M, N, K, tile):
+        with pytest.raises(dcl.DcleapError):
+            ops.op_linear(_bf16(a), _bf16(w), h, mode=1, tile=tile)
+        return
     ops.op_linear(_bf16(a), _bf16(w), h, mode=1, tile=tile)
     torch.cuda.synchronize()
     ref = h0.astype(np.float64) + a.astype(np.float64) @ w.astype(np.float64).T
     assert np.abs(h.cpu().numpy() - ref).max() <= 1e-4 * np.sqrt((ref ** 2).mean()) * 10
 
 
-@pytest.mark.parametrize("tile,mode", [(2 | (3 << 8), 1), (2 | (2 << 8), 0), (0, 1)])
+@pytest.mark.parametrize("tile,mode", [(PAIR | (3 << 8), 1), (PAIR | (2 << 8), 0), (0, 1), (0, 0),
+                                       (PAIR | SK, 0), (PAIR | SK, 1)])
 def test_linear_split_k_is_deterministic(ops, tile, mode):
-    """Split-K partial sums are combined in split order: two runs give the same bits."""
+    """Split-K and stream-K partial sums are combined in K order: two runs give the same
+    bits."""
     rng = np.random.default_rng(5)
     M, N, K = 512, 4096, 12288
     a = _bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
@@ -148,9 +170,10 @@ def test_attention_non_causal(ops, B, T, H, G, hd):
 
 
 # ------------------------------------------------------------------ LM head + confidence
-@pytest.mark.parametrize("tile", [0, 256, 2])
+@pytest.mark.parametrize("tile", [0, 256, PAIR, PAIR | SK])
 @pytest.mark.parametrize("R,V,d,sz", [(37, 4096, 256, 12.0), (5, 1000, 128, 6.0), (130, 4096, 64, 20.0),
-                                      (300, 4096, 256, 12.0), (64, 126464, 4096, 15.0)])
+                                      (300, 4096, 256, 12.0), (64, 126464, 4096, 15.0),
+                                      (300, 126464, 4096, 15.0)])
 def test_lmhead_top2(ops, R, V, d, sz, tile):
     rng = np.random.default_rng(R * V + d)
     x = syn.round_bf16(rng.normal(0, 1, (R, d)).astype(np.float32))
@@ -164,6 +187,10 @@ def test_lmhead_top2(ops, R, V, d, sz, tile):
     top1 = torch.zeros(R, dtype=torch.int32, device="cuda")
     p1 = torch.zeros(R, dtype=torch.float32, device="cuda")
     p2 = torch.zeros(R, dtype=torch.float32, device="cuda")
+    if _unsupported(R, V, d, tile):
+        with pytest.raises(dcl.DcleapError):
+            ops.op_lmhead_top2(_bf16(x), _bf16(w), top1, p1, p2, tile=tile)
+        return
     ops.op_lmhead_top2(_bf16(x), _bf16(w), top1, p1, p2, tile=tile)
     torch.cuda.synchronize()
     rows = np.arange(R) if R <= 64 else rng.choice(R, 32, replace=False)

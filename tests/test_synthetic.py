@@ -47,3 +47,19 @@ def test_accept_inputs_recipe():
     z = syn.bf16_to_f32(d["logits_bf16"]).astype(np.float64)
     top = np.argmax(z, axis=2)
     assert (top == d["top_index"]).all()
+
+
+def test_weight_values_chunked_threaded_equals_definition():
+    """The generator runs in threaded, cache-sized chunks; it must equal the definition in
+    its docstring evaluated in one pass (a sub-range straddling thread boundaries)."""
+    seed, tid, start, count, std, mean = 3, syn.tensor_id(syn.TensorKind.W_UP, 7), 12_345, 5_000_003, 0.3, -0.5
+    idx = np.arange(start, start + count, dtype=np.uint64)
+    key = (np.uint64(seed) << np.uint64(48)) | (np.uint64(tid) << np.uint64(32)) | idx
+    h = syn.splitmix64(key)
+    m16 = np.uint64(0xFFFF)
+    s = ((h & m16) + ((h >> np.uint64(16)) & m16) + ((h >> np.uint64(32)) & m16)
+         + (h >> np.uint64(48))).astype(np.int64)
+    w = (s - 131070).astype(np.float32) * np.float32(float(np.float32(std)) / syn.GEN_SIGMA4)
+    w = syn.round_bf16(w + np.float32(mean))
+    got = syn.weight_values(seed, tid, start, count, std, mean)
+    assert np.array_equal(got.view(np.uint32), w.view(np.uint32))
