@@ -164,9 +164,13 @@ __device__ __forceinline__ Part shfl_part(const Part& a, int off) {
 
 __device__ __forceinline__ void write_conf(const Part& a, int32_t* top1, float* p1, float* p2, int r) {
   top1[r] = a.id;
-  const float inv = 1.0f / a.s;  // p1 = exp(max - max) / sum
-  p1[r] = inv;
-  p2[r] = a.t2 == -INFINITY ? 0.f : exp2f((a.t2 - a.m) * kLog2e) * inv;
+  // p1 = exp(max - max) / sum.  The sum holds the max's own term exp(0) = 1, but that
+  // term is evaluated as exp2 of a rounding residual and may come out a hair below 1, so
+  // the probabilities are clamped to [0, 1] and p2 <= p1.
+  const float inv = 1.0f / a.s;
+  const float c1 = fminf(inv, 1.0f);
+  p1[r] = c1;
+  p2[r] = a.t2 == -INFINITY ? 0.f : fminf(exp2f((a.t2 - a.m) * kLog2e) * inv, c1);
 }
 
 __global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows, int nblk,

@@ -6,8 +6,13 @@ prompt 256 + generation 256, window 128, thresholds 0.7 / 0.98, LM head x12, wei
 
 A 32-layer forward of an 8B model in fp64 is out of reach of a test, so:
   * the residual stream after the embedding (exactly) and after blocks 0 and 1 is compared
-    with the bf16-operand oracle on every one of the 512 rows (relative rms error per row
-    <= 3e-3, the per-layer tolerance of the small-model tests);
+    with the bf16-operand oracle on every one of the 512 rows.  Tolerance: at this size the
+    fp32 accumulation alone moves values across bf16 rounding boundaries often enough
+    that an IEEE-fp32 evaluation of block 0 with the same rounding points (PyTorch on the
+    CPU) lies 2.1e-3 (mean) / 4.4e-3 (max) from the fp64 oracle in relative rms per row,
+    the GPU 2.7e-3 / 4.2e-3; dropping any one of the bf16 rounding points moves the
+    oracle by 2.5e-3 .. 6.8e-3 (mean).  Block 0 must stay within 3.5e-3 (mean) and 6e-3
+    (max), block 1 (whose input already differs) within 5e-3 and 1e-2;
   * every step of a whole generation must apply the acceptance rule (Eq. compute_k,
     Eq. draft_update, Algorithm 1; strict thresholds in float32, K raised to 1, window
     clipped to the sequence end) to the step's own predictions, which
@@ -76,10 +81,11 @@ def test_first_blocks_match_oracle(dcl):
     w = syn.model_weights(SH, SEED, STD, LM_SCALE, 0.0, layers=(0, 1), global_tensors=False)
     w["embed"] = syn.embed_rows(SH, SEED, uniq, STD)
     assert (got[0] == w["embed"][inv]).all()  # the embedding is an exact copy
-    for layer in (0, 1):
+    for layer, (tol_mean, tol_max) in ((0, (3.5e-3, 6e-3)), (1, (5e-3, 1e-2))):
         ref = model.forward_hidden(SH, w, inv, bf16_operands=True, upto_layer=layer)
         err = np.sqrt(((got[layer + 1] - ref) ** 2).mean(axis=1)) / np.sqrt((ref ** 2).mean(axis=1))
-        assert err.max() <= 3e-3, (layer, float(err.max()))
+        print(f"block {layer}: relative rms error per row mean {err.mean():.2e} max {err.max():.2e}")
+        assert err.mean() <= tol_mean and err.max() <= tol_max, (layer, float(err.mean()), float(err.max()))
 
 
 def _expected_step(x0, p0, top1, c1, N, L):
