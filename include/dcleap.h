@@ -236,8 +236,9 @@ dcl_status dcl_op_linear(dcl_ctx* ctx, const void* a_dev, const void* w_dev, voi
                          int32_t M, int32_t N, int32_t K, int32_t mode, int32_t tile);
 
 /* Non-causal attention softmax(q k^T / sqrt(hd)) v over all T positions of each of
- * `batch` sequences.  qkv_dev bf16 [batch*T][(H+2G)*hd] (q | k | v column blocks, RoPE
- * already applied), out_dev bf16 [batch*T][H*hd].  hd in {64, 128}.  Async. */
+ * `batch` sequences (the attention of the bidirectional pass, Eq. 2).  qkv_dev bf16
+ * [batch*T][(H+2G)*hd] (q | k | v column blocks, RoPE already applied), out_dev bf16
+ * [batch*T][H*hd]; both 16-byte aligned.  hd in {64, 128}.  Synchronises. */
 dcl_status dcl_op_attention(dcl_ctx* ctx, const void* qkv_dev, void* out_dev, int32_t batch,
                             int32_t T, int32_t H, int32_t G, int32_t hd);
 

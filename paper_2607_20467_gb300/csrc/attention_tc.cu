@@ -1,0 +1,463 @@
+// Non-causal attention of the bidirectional forward (Eq. 2 runs one full pass in which
+// every position attends to every position of its sequence), on the tcgen05 tensor
+// cores of sm_103a.
+//
+// One CTA = 128 query rows of one (sequence, head); the key axis is walked in blocks of
+// 128 in two passes:
+//   pass 1: S_j = Q K_j^T into TMEM, row maxima m (softmax warps, one query row per
+//           thread);
+//   pass 2: S_j again; P_j = exp2(S_j * log2(e)/sqrt(hd) - m) with the row sum l kept in
+//           fp32; P_j is written to shared memory as a bf16 pair hi + lo (hi = P with its
+//           low 16 bits cleared, lo = bf16(P - hi): about 16 significant bits together)
+//           and O += P_hi V_j + P_lo V_j accumulates in TMEM.
+// O / l leaves through TMA.  Two passes cost one more Q K^T than an online softmax but
+// need no rescaling of the TMEM accumulator and give the exact row maximum.
+//
+// Roles (192 threads): warp 0 lane 0 TMA producer (Q once, then K / V^T blocks through a
+// 2-stage ring in the order the MMAs consume them); warp 1 allocates TMEM and its lane 0
+// issues the MMAs; warps 2..5 run the softmax and the epilogue.  P is double-buffered so
+// that the softmax of block j + 1 overlaps the P V MMAs of block j.  V enters as V^T (a
+// K-major operand, kv contiguous), written by v_transpose_kernel from the q|k|v buffer.
+// Every wait is bounded (DERR_WAIT_TIMEOUT).
+#include "common.cuh"
+#include "tc_ptx.cuh"
+
+namespace dcl {
+namespace {
+
+constexpr int AT_THREADS = 192;
+constexpr int AT_STAGES = 2;
+constexpr int AT_BOX = 128 * 128;  // one 128-row x 128-byte swizzle box
+
+template <int HD>
+struct AttnCfg {
+  static constexpr int KB = HD / 64;                   // 64-wide boxes along hd
+  static constexpr int Q_BYTES = 128 * HD * 2;         // Q tile [128][HD]
+  static constexpr int STAGE_BYTES = 128 * HD * 2;     // K block [128][HD] or V^T block [HD][128]
+  static constexpr int VBOX = HD * 128;                // one V^T box: [HD rows][64 kv]
+  static constexpr int P_BYTES = 2 * 2 * 2 * AT_BOX;   // 2 buffers of P_hi and P_lo, [128][128] each
+  static constexpr int BARS = 256;
+  static constexpr size_t SMEM = 1024 + (size_t)Q_BYTES + AT_STAGES * STAGE_BYTES + P_BYTES + BARS;
+  static constexpr uint32_t TMEM_COLS = 512;           // S double buffer (2 x 128) + O (HD)
+};
+
+// vt[(b*G + g)*hd + d][t] = v of token t, kv head g, component d (row pitch Tp, zero pad).
+// A block moves a 64-token x 64-channel tile with 16-byte loads and stores.
+__global__ void __launch_bounds__(256) v_transpose_kernel(const __nv_bfloat16* __restrict__ qkv,
+                                                          __nv_bfloat16* __restrict__ vt, int T, int Tp, int cols,
+                                                          int v0, int ghd) {
+  __shared__ __nv_bfloat16 tile[64][72];  // [channel][token], rows padded by 16 bytes
+  const int t0 = blockIdx.x * 64, c0 = blockIdx.y * 64, b = blockIdx.z;
+  for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+    const int r = i >> 3, cv = (i & 7) * 8;  // token row, first channel of the vector
+    const int t = t0 + r;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (t < T && c0 + cv < ghd)
+      v = *reinterpret_cast<const uint4*>(qkv + ((size_t)b * T + t) * cols + v0 + c0 + cv);
+    const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&v);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) tile[cv + k][r] = e[k];
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 64 * 8; i += 256) {
+    const int c = i >> 3, tv = (i & 7) * 8;  // channel row, first token of the vector
+    if (c0 + c < ghd && t0 + tv < Tp)
+      *reinterpret_cast<uint4*>(vt + ((size_t)b * ghd + c0 + c) * Tp + t0 + tv) =
+          *reinterpret_cast<const uint4*>(&tile[c][tv]);
+  }
+}
+
+template <int HD>
+__global__ void __launch_bounds__(AT_THREADS, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tv,
+                   const __grid_constant__ CUtensorMap to, int T, int H, int G, int* err) {
+  using C = AttnCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+  const uint32_t sQ = base;
+  const uint32_t sKV = sQ + C::Q_BYTES;
+  const uint32_t sP = sKV + AT_STAGES * C::STAGE_BYTES;  // per buffer: P_hi boxes, then P_lo boxes
+  const uint32_t bars = sP + C::P_BYTES;
+  const uint32_t q_full = bars;
+  const uint32_t kv_full0 = bars + 8;                   // + 8 s
+  const uint32_t kv_empty0 = kv_full0 + 8 * AT_STAGES;  // + 8 s
+  const uint32_t s_full0 = kv_empty0 + 8 * AT_STAGES;   // + 8 b
+  const uint32_t s_empty0 = s_full0 + 16;               // + 8 b
+  const uint32_t p_full0 = s_empty0 + 16;  // + 8 buffer
+  const uint32_t p_empty0 = p_full0 + 16;  // + 8 buffer
+  const uint32_t o_full = p_empty0 + 16;
+  const uint32_t drain = o_full + 8;
+  const uint32_t holder = drain + 8;
+  volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int g = h / (H / G);
+  const int nb = (T + 127) / 128;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < AT_STAGES; ++s) {
+      mbar_init(kv_full0 + 8 * s, 1);
+      mbar_init(kv_empty0 + 8 * s, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(s_full0 + 8 * i, 1);
+      mbar_init(s_empty0 + 8 * i, 4);  // the 4 softmax warps
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(p_full0 + 8 * i, 4);
+      mbar_init(p_empty0 + 8 * i, 1);
+    }
+    mbar_init(o_full, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tq);
+    prefetch_tmap(&tv);
+    prefetch_tmap(&to);
+  }
+  if (warp == 1) tmem_alloc(holder, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *holder_ptr;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      bool ok = true;
+      int stage = 0;
+      uint32_t phase = 0;
+      long issued = 0;
+      mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+      for (int bx = 0; bx < C::KB; ++bx) tma_load_3d(sQ + bx * AT_BOX, &tq, h * HD + bx * 64, qt * 128, b, q_full);
+      // consumption order: K_0 .. K_{nb-1} (pass 1); K_0, K_1, then per j: K_{j+2}, V_j
+      // (pass 2; K only while j + 2 < nb)
+      const int n_loads = 3 * nb;
+      const int head = nb < 2 ? nb : 2, npairs = nb > 2 ? nb - 2 : 0;
+      for (int u = 0; u < n_loads && ok; ++u) {
+        bool is_v;
+        int j;
+        if (u < nb) {
+          is_v = false, j = u;
+        } else if (u - nb < head) {
+          is_v = false, j = u - nb;
+        } else {
+          const int r = u - nb - head;
+          if (r < 2 * npairs) {
+            is_v = (r & 1) != 0;
+            j = (r >> 1) + (is_v ? 0 : 2);
+          } else {
+            is_v = true;
+            j = npairs + (r - 2 * npairs);
+          }
+        }
+        if (!mbar_wait(kv_empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = sKV + stage * C::STAGE_BYTES, bar = kv_full0 + 8 * stage;
+        mbar_arrive_expect_tx(bar, C::STAGE_BYTES);
+        if (!is_v) {
+          for (int bx = 0; bx < C::KB; ++bx)
+            tma_load_3d(dst + bx * AT_BOX, &tq, (H + g) * HD + bx * 64, j * 128, b, bar);
+        } else {
+          for (int bx = 0; bx < 2; ++bx) tma_load_3d(dst + bx * C::VBOX, &tv, j * 128 + bx * 64, 0, b * G + g, bar);
+        }
+        ++issued;
+        if (++stage == AT_STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+        // wait (bounded) for the copies this thread issued before leaving
+        volatile int no_abort = 0;
+        mbar_wait(q_full, 0, &no_abort);
+        for (int s = 0; s < AT_STAGES && s < issued; ++s) {
+          const long arms = (issued - 1 - s) / AT_STAGES + 1;
+          mbar_wait(kv_full0 + 8 * s, (uint32_t)((arms - 1) & 1), &no_abort);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc_s = make_idesc(128, 128);
+      constexpr uint32_t idesc_o = make_idesc(128, HD);
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      int stage = 0;
+      uint32_t phase = 0;
+      int si = 0;  // S-buffer uses so far
+      auto take = [&](uint32_t& st_addr) -> bool {
+        if (!mbar_wait(kv_full0 + 8 * stage, phase, abort_flag)) return false;
+        st_addr = sKV + stage * C::STAGE_BYTES;
+        return true;
+      };
+      auto release = [&]() {
+        umma_commit(kv_empty0 + 8 * stage);
+        if (++stage == AT_STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      };
+      auto issue_s = [&]() -> bool {  // S[si & 1] = Q K^T with the K block at the ring head
+        uint32_t kaddr;
+        if (!take(kaddr)) return false;
+        const int sb = si & 1;
+        if (!mbar_wait(s_empty0 + 8 * sb, (((uint32_t)si >> 1) & 1u) ^ 1u, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(sb * 128);
+#pragma unroll
+        for (int k = 0; k < HD / 16; ++k)
+          umma_bf16(d, sw128_desc(sQ + (k >> 2) * AT_BOX) + 2 * (k & 3), sw128_desc(kaddr + (k >> 2) * AT_BOX) + 2 * (k & 3),
+                    idesc_s, k > 0 ? 1u : 0u);
+        release();
+        umma_commit(s_full0 + 8 * sb);
+        ++si;
+        return true;
+      };
+      auto issue_pv = [&](int j) -> bool {  // O += P_hi V_j + P_lo V_j
+        uint32_t vaddr;
+        if (!take(vaddr)) return false;
+        const int pb = j & 1;
+        if (!mbar_wait(p_full0 + 8 * pb, ((uint32_t)j >> 1) & 1u, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t d = tmem + 256u;
+        const uint32_t pbase = sP + (uint32_t)pb * 4 * AT_BOX;
+#pragma unroll
+        for (int part = 0; part < 2; ++part)
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            umma_bf16(d, sw128_desc(pbase + part * 2 * AT_BOX + (k >> 2) * AT_BOX) + 2 * (k & 3),
+                      sw128_desc(vaddr + (k >> 2) * C::VBOX) + 2 * (k & 3), idesc_o, (j > 0 || part > 0 || k > 0) ? 1u : 0u);
+        release();
+        umma_commit(p_empty0 + 8 * pb);
+        return true;
+      };
+      for (int j = 0; ok && j < nb; ++j) ok = issue_s();  // pass 1
+      if (ok) ok = issue_s();                              // pass 2: S_0, S_1
+      if (ok && nb > 1) ok = issue_s();
+      for (int j = 0; ok && j < nb; ++j) {  // S_{j+2} (its buffer frees with P_j) before PV_j
+        if (j + 2 < nb) ok = issue_s();
+        if (ok) ok = issue_pv(j);
+      }
+      if (ok) umma_commit(o_full);
+      if (!ok) {
+        *abort_flag = 1;
+        report_error(err, DERR_WAIT_TIMEOUT);
+      }
+      umma_commit(drain);  // every MMA issued here completes before TMEM is released
+      volatile int no_abort = 0;
+      mbar_wait(drain, 0, &no_abort);
+    }
+  } else {
+    // ------------------------------------------------ softmax + epilogue (warps 2..5)
+    const int q = warp & 3;             // TMEM lane quarter = 32-row band
+    const int r = q * 32 + lane;        // query row within the tile
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const float scale2 = kLog2e * rsqrtf((float)HD);
+    bool ok = true;
+    int si = 0;
+    float m = -INFINITY;
+    for (int j = 0; ok && j < nb; ++j) {  // pass 1: row maxima
+      const int sb = si & 1;
+      ok = mbar_wait(s_full0 + 8 * sb, ((uint32_t)si >> 1) & 1u, abort_flag);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc_fence_after();
+      const int valid = T - j * 128;
+      uint32_t v[4][32];  // the whole 128-column row, one wait
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * c), v[c]);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_empty0 + 8 * sb);
+      float mm = -INFINITY;
+      if (valid >= 128) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e) mm = fmaxf(mm, f32(v[c][e]));
+      } else {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (32 * c + e < valid) mm = fmaxf(mm, f32(v[c][e]));
+      }
+      m = fmaxf(m, mm * scale2);
+      ++si;
+    }
+    float l = 0.f;
+    for (int j = 0; ok && j < nb; ++j) {  // pass 2: P = exp2(s - m), l, P_hi / P_lo
+      const int sb = si & 1, pb = j & 1;
+      ok = mbar_wait(s_full0 + 8 * sb, ((uint32_t)si >> 1) & 1u, abort_flag);
+      if (ok && j >= 2) ok = mbar_wait(p_empty0 + 8 * pb, ((uint32_t)(j - 2) >> 1) & 1u, abort_flag);  // PV_{j-2} read it
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc_fence_after();
+      const int valid = T - j * 128;
+      const uint32_t pbase = sP + (uint32_t)pb * 4 * AT_BOX;
+      uint32_t v[2][32];
+      tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128), v[0]);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        tmem_ld_wait();
+        if (c + 1 < 4) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * (c + 1)), v[(c + 1) & 1]);
+        // P = hi + lo: hi = P with its low 16 bits cleared (a bf16 value), lo = P - hi
+        // (exact) rounded to bf16, so P is carried to about 2^-16 relative
+        uint32_t hb[32];
+        float lo[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          float p = ex2_approx(fmaf(f32(v[c & 1][e]), scale2, -m));
+          if (valid < 128 && 32 * c + e >= valid) p = 0.f;
+          l += p;
+          hb[e] = __float_as_uint(p) & 0xFFFF0000u;
+          lo[e] = p - __uint_as_float(hb[e]);
+        }
+        const uint32_t box = pbase + (uint32_t)(c >> 1) * AT_BOX;
+        const int k0 = (c & 1) * 4;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          st_shared_v4(box + swz(r, k0 + k), __byte_perm(hb[8 * k], hb[8 * k + 1], 0x7632),
+                       __byte_perm(hb[8 * k + 2], hb[8 * k + 3], 0x7632), __byte_perm(hb[8 * k + 4], hb[8 * k + 5], 0x7632),
+                       __byte_perm(hb[8 * k + 6], hb[8 * k + 7], 0x7632));
+          st_shared_v4(box + 2 * AT_BOX + swz(r, k0 + k), pack_bf16x2(lo[8 * k], lo[8 * k + 1]),
+                       pack_bf16x2(lo[8 * k + 2], lo[8 * k + 3]), pack_bf16x2(lo[8 * k + 4], lo[8 * k + 5]),
+                       pack_bf16x2(lo[8 * k + 6], lo[8 * k + 7]));
+        }
+      }
+      tc_fence_before();
+      fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(s_empty0 + 8 * sb);
+        mbar_arrive(p_full0 + 8 * pb);
+      }
+      ++si;
+    }
+    if (ok) ok = mbar_wait(o_full, 0, abort_flag);
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+      // epilogue: O / l -> bf16 -> TMA store (staged in this warp's part of the P
+      // buffers, free once every PV MMA has completed)
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      const int row0 = qt * 128 + q * 32;
+      const uint32_t stg = sP + (uint32_t)q * (C::KB * 32 * 128);
+#pragma unroll 1
+      for (int c = 0; c < HD; c += 64) {
+        const uint32_t bx = stg + (uint32_t)(c >> 6) * (32 * 128);
+#pragma unroll 1
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t v[32];
+          tmem_ld32(tmem + lane_off + 256u + (uint32_t)(c + 32 * hh), v);
+          tmem_ld_wait();
+          float o[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = f32(v[e]) * inv;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            st_shared_v4(bx + swz(lane, 4 * hh + k), pack_bf16x2(o[8 * k], o[8 * k + 1]), pack_bf16x2(o[8 * k + 2], o[8 * k + 3]),
+                         pack_bf16x2(o[8 * k + 4], o[8 * k + 5]), pack_bf16x2(o[8 * k + 6], o[8 * k + 7]));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0 && row0 < T) tma_store_3d(&to, bx, h * HD + c, row0, b);
+      }
+      if (lane == 0) {
+        bulk_commit();
+        bulk_wait_all();
+      }
+      __syncwarp();
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      report_error(err, DERR_WAIT_TIMEOUT);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int HD>
+cudaError_t launch_attn(const AttnPlan& p, int* err, cudaStream_t stream) {
+  static bool attr_set = false;
+  auto kern = attn_tc_kernel<HD>;
+  if (!attr_set) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnCfg<HD>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid((p.T + 127) / 128, p.H, p.batch);
+  kern<<<grid, AT_THREADS, AttnCfg<HD>::SMEM, stream>>>(p.tq, p.tv, p.to, p.T, p.H, p.G, err);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int attn_vt_pitch(int T) { return (T + 7) & ~7; }
+
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16* vt, __nv_bfloat16* out, int batch,
+                           int T, int H, int G, int hd) {
+  if (batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128)) return cudaErrorInvalidValue;
+  if ((reinterpret_cast<uintptr_t>(qkv) & 15) || (reinterpret_cast<uintptr_t>(vt) & 15) ||
+      (reinterpret_cast<uintptr_t>(out) & 15))
+    return cudaErrorInvalidValue;
+  const uint64_t cols = (uint64_t)(H + 2 * G) * hd, ocols = (uint64_t)H * hd, Tp = attn_vt_pitch(T);
+  {  // q | k | v rows as [batch][T][cols]: rows past T of a sequence read as zero
+    const uint64_t dims[3] = {cols, (uint64_t)T, (uint64_t)batch};
+    const uint64_t strides[2] = {cols * 2, (uint64_t)T * cols * 2};
+    const uint32_t box[3] = {64, 128, 1};
+    if (!encode_tmap(&p->tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(qkv), dims, strides, box,
+                     CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  }
+  {  // v^T as [batch*G][hd][T] (row pitch Tp)
+    const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
+    const uint64_t strides[2] = {Tp * 2, (uint64_t)hd * Tp * 2};
+    const uint32_t box[3] = {64, (uint32_t)hd, 1};
+    if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  }
+  {  // output as [batch][T][H*hd]: stores of rows past T are clipped
+    const uint64_t dims[3] = {ocols, (uint64_t)T, (uint64_t)batch};
+    const uint64_t strides[2] = {ocols * 2, (uint64_t)T * ocols * 2};
+    const uint32_t box[3] = {64, 32, 1};
+    if (!encode_tmap(&p->to, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, out, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  }
+  p->qkv = qkv;
+  p->vt = vt;
+  p->batch = batch;
+  p->T = T;
+  p->H = H;
+  p->G = G;
+  p->hd = hd;
+  return cudaSuccess;
+}
+
+cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream) {
+  const int cols = (p.H + 2 * p.G) * p.hd, ghd = p.G * p.hd;
+  dim3 tgrid((attn_vt_pitch(p.T) + 63) / 64, (ghd + 63) / 64, p.batch);
+  v_transpose_kernel<<<tgrid, 256, 0, stream>>>(p.qkv, p.vt, p.T, attn_vt_pitch(p.T), cols, (p.H + p.G) * p.hd, ghd);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return p.hd == 128 ? launch_attn<128>(p, err, stream) : launch_attn<64>(p, err, stream);
+}
+
+}  // namespace dcl

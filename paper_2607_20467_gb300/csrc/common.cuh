@@ -15,7 +15,7 @@ namespace dcl {
 enum DevErr : int {
   DERR_NONE = 0,
   DERR_TOKEN_RANGE = 1,     // a token id outside [0, vocab) reached the embedding
-  DERR_WAIT_TIMEOUT = 2,    // a bounded mbarrier wait gave up (GEMM pipeline)
+  DERR_WAIT_TIMEOUT = 2,    // a bounded wait gave up (GEMM / attention pipeline)
   DERR_BAD_SHAPE = 3,       // a kernel was launched with a shape it does not support
 };
 
@@ -93,10 +93,26 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
 cudaError_t gemm_bind_scratch(GemmPlan* plan, int* flags, float* ws);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
+// cuTensorMapEncodeTiled through the runtime's driver entry point: dims / box in elements
+// (innermost first), strides in bytes for dimensions 1 .. rank-1; out-of-range elements
+// read as zero.
+bool encode_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, void* ptr, const uint64_t* dims,
+                 const uint64_t* strides, const uint32_t* box, CUtensorMapSwizzle swizzle);
 
-// ---------------------------------------------------------------- attention (attention.cu)
-cudaError_t attention_launch(const __nv_bfloat16* qkv, __nv_bfloat16* out, int batch, int T,
-                             int H, int G, int hd, cudaStream_t stream);
+// ---------------------------------------------------------------- attention (attention_tc.cu)
+// softmax(q k^T / sqrt(hd)) v per (sequence, head) over all T positions (non-causal), on
+// the tcgen05 tensor cores.  qkv bf16 [batch*T][(H+2G)*hd] (q | k | v column blocks),
+// out bf16 [batch*T][H*hd]; vt is scratch for v transposed, bf16 [batch*G*hd][attn_vt_pitch(T)].
+struct AttnPlan {
+  CUtensorMap tq, tv, to;
+  const __nv_bfloat16* qkv = nullptr;
+  __nv_bfloat16* vt = nullptr;
+  int batch = 0, T = 0, H = 0, G = 0, hd = 0;
+};
+int attn_vt_pitch(int T);
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16* vt, __nv_bfloat16* out, int batch,
+                           int T, int H, int G, int hd);
+cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream);
 
 // ---------------------------------------------------------------- other kernels (kernels.cu)
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,

@@ -51,6 +51,7 @@ struct dcl_ctx {
   // activations, sized for max_batch * max_seq rows
   float* h = nullptr;
   __nv_bfloat16 *xn = nullptr, *qkv = nullptr, *attn = nullptr, *act = nullptr, *xg = nullptr;
+  __nv_bfloat16* vt = nullptr;  // v transposed for the attention kernel
   float4* part = nullptr;
   int32_t* top1 = nullptr;
   float *p1 = nullptr, *p2 = nullptr;
@@ -75,6 +76,7 @@ struct dcl_ctx {
   int B = 0, N = 0, M = 0, T = 0, window = 0;
   dcl_decode_config dcfg{};
   std::vector<GemmPlan> plans;  // 4 per layer + LM head
+  AttnPlan attn_plan;
   cudaGraphExec_t gexec = nullptr;
   bool profiling = false;
   std::vector<Launch> launches;
@@ -160,7 +162,7 @@ dcl_status check_device(dcl_ctx* c) {
     // an aborted split-K launch may leave its counters set: clear them for the next one
     if (c->gemm_flags) cudaMemset(c->gemm_flags, 0, sizeof(int) * c->gemm_flags_n);
     if (e == DERR_WAIT_TIMEOUT)
-      return fail(c, DCL_ERR_TIMEOUT, "a GEMM pipeline wait timed out on the device (kernel returned)");
+      return fail(c, DCL_ERR_TIMEOUT, "a pipeline wait timed out on the device (kernel returned)");
     if (e == DERR_TOKEN_RANGE) return fail(c, DCL_ERR_INVALID_ARG, "a token id outside [0, vocab) reached the embedding");
     return fail(c, DCL_ERR_CUDA, "device error code %d", e);
   }
@@ -217,8 +219,7 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
     q.begin(DCL_K_GEMM_QKV);
     q.end(gemm_launch(P[0], c->derr, c->stream), "gemm_qkv");
     q.begin(DCL_K_ATTENTION);
-    q.end(attention_launch(c->qkv, c->attn, c->B, c->T, m.n_heads, m.n_kv_heads, m.head_dim, c->stream),
-          "attention");
+    q.end(attention_launch(c->attn_plan, c->derr, c->stream), "attention");
     q.begin(DCL_K_GEMM_O);
     q.end(gemm_launch(P[1], c->derr, c->stream), "gemm_o");
     q.begin(DCL_K_RMSNORM);
@@ -332,6 +333,8 @@ dcl_status build_plans(dcl_ctx* c) {
                   t_down, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "down plan: %s", why ? why : "?");
   }
+  if (attention_plan(&c->attn_plan, c->qkv, c->vt, c->attn, c->B, c->T, m.n_heads, m.n_kv_heads, hd) != cudaSuccess)
+    return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
   EpiParams el;
   el.out = c->part;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,
@@ -552,6 +555,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->xn = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->qkv = (__nv_bfloat16*)dev_alloc(c, 2 * R * (H + 2 * G) * hd);
     c->attn = (__nv_bfloat16*)dev_alloc(c, 2 * R * H * hd);
+    c->vt = (__nv_bfloat16*)dev_alloc(c, 2 * (size_t)max_batch * G * hd * attn_vt_pitch(max_seq));
     c->act = (__nv_bfloat16*)dev_alloc(c, 2 * R * F);
     c->xg = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->part = (float4*)dev_alloc(c, sizeof(float4) * R * nblk);
@@ -567,7 +571,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->p_init = (int32_t*)dev_alloc(c, 4 * max_batch);
     c->rope_cos = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
     c->rope_sin = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
-    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->act || !c->xg || !c->part || !c->top1 ||
+    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->act || !c->xg || !c->part || !c->top1 ||
         !c->p1 || !c->p2 || !c->x || !c->p || !c->k || !c->steps || !c->done_count || !c->x_init || !c->p_init || !c->rope_cos ||
         !c->rope_sin) {
       dev_free_all(c);
@@ -907,9 +911,23 @@ dcl_status dcl_op_attention(dcl_ctx* c, const void* qkv_dev, void* out_dev, int3
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!qkv_dev || !out_dev || batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128))
     return fail(c, DCL_ERR_INVALID_ARG, "bad attention args");
-  CUDA_TRY(c, attention_launch(static_cast<const __nv_bfloat16*>(qkv_dev), static_cast<__nv_bfloat16*>(out_dev), batch,
-                               T, H, G, hd, c->stream));
-  return DCL_OK;
+  __nv_bfloat16* vt = static_cast<__nv_bfloat16*>(dev_alloc(c, 2 * (size_t)batch * G * hd * attn_vt_pitch(T)));
+  if (!vt) return fail(c, DCL_ERR_OOM, "attention scratch allocation failed");
+  AttnPlan pl;
+  if (attention_plan(&pl, static_cast<const __nv_bfloat16*>(qkv_dev), vt, static_cast<__nv_bfloat16*>(out_dev), batch, T,
+                     H, G, hd) != cudaSuccess) {
+    dev_free_one(c, vt);
+    return fail(c, DCL_ERR_INVALID_ARG, "attention: operands must be 16-byte aligned");
+  }
+  const cudaError_t e = attention_launch(pl, c->derr, c->stream);
+  if (e != cudaSuccess) {
+    cudaStreamSynchronize(c->stream);
+    dev_free_one(c, vt);
+    return fail(c, DCL_ERR_CUDA, "attention launch: %s", cudaGetErrorString(e));
+  }
+  const dcl_status s = check_device(c);
+  dev_free_one(c, vt);
+  return s;
 }
 
 dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, int32_t R, int32_t V, int32_t d,
