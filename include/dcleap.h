@@ -220,11 +220,11 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * 128 / 256 force a one-CTA 128 x 128 / 128 x 256 tile, DCL_TILE_PAIR a CTA-pair
  * (tcgen05 cta_group::2) 256 x 256 tile with the library's choice of K splitting,
  * DCL_TILE_PAIR | (S << 8) that tile with the K dimension split S ways (S = 1: unsplit),
- * DCL_TILE_PAIR | DCL_TILE_STREAMK that tile with the stream-K schedule (the tiles of a
- * partly filled last round of the persistent grid are shared out by K ranges over all
- * CTA pairs; rejected with DCL_ERR_INVALID_ARG when the last round is full or holds
- * fewer K blocks than there are CTA pairs).  Partial sums are always combined in K order,
- * so every choice is deterministic. */
+ * DCL_TILE_PAIR | DCL_TILE_STREAMK | (S << 8) that tile with the stream-K schedule: the
+ * tiles of a partly filled last round of the persistent grid are cut into about S K
+ * segments each (S = 0: shared out over all CTA pairs) run by different pairs; rejected
+ * with DCL_ERR_INVALID_ARG when the last round is full or a sharing pair would get no K
+ * block.  Partial sums are always combined in K order, so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
 #define DCL_TILE_STREAMK (1 << 16)
 
@@ -269,7 +269,8 @@ typedef enum {
   DCL_K_GEMM_DOWN = 6,   /* down projection + residual */
   DCL_K_GEMM_LMHEAD = 7, /* LM head + softmax/top-2 partials */
   DCL_K_COMBINE = 8,     /* merge of the LM-head partials */
-  DCL_K_DCV = 9          /* commit / draft / advance */
+  DCL_K_DCV = 9,         /* commit / draft / advance */
+  DCL_K_VTRANSPOSE = 10  /* v written transposed for the attention kernel */
 } dcl_kernel_kind;
 
 /* enable = 1 re-captures the step graph with a pair of timing events (CUDA event record

@@ -451,13 +451,20 @@ cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16*
   return cudaSuccess;
 }
 
-cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream) {
+cudaError_t attention_transpose_launch(const AttnPlan& p, cudaStream_t stream) {
   const int cols = (p.H + 2 * p.G) * p.hd, ghd = p.G * p.hd;
   dim3 tgrid((attn_vt_pitch(p.T) + 63) / 64, (ghd + 63) / 64, p.batch);
   v_transpose_kernel<<<tgrid, 256, 0, stream>>>(p.qkv, p.vt, p.T, attn_vt_pitch(p.T), cols, (p.H + p.G) * p.hd, ghd);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+cudaError_t attention_core_launch(const AttnPlan& p, int* err, cudaStream_t stream) {
   return p.hd == 128 ? launch_attn<128>(p, err, stream) : launch_attn<64>(p, err, stream);
+}
+
+cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream) {
+  const cudaError_t e = attention_transpose_launch(p, stream);
+  return e != cudaSuccess ? e : attention_core_launch(p, err, stream);
 }
 
 }  // namespace dcl

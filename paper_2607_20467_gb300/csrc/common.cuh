@@ -70,7 +70,7 @@ struct GemmPlan {
   int n_tiles = 0;
   size_t smem = 0;
   int splits = 1;          // split-K factor (pair tiles only)
-  int streamk = 0;         // 1: left-over pair tiles shared out by K (stream-K)
+  int streamk = 0;         // > 0: left-over pair tiles shared out by K over this many pairs
   int ws_slots = 0;        // stream-K partial slots per left-over tile
   size_t flags_needed = 0; // ints of zero-initialised split counters the launch needs
   size_t ws_needed = 0;    // floats of workspace for split-K partials
@@ -82,7 +82,8 @@ struct GemmPlan {
 // W is [N][K] bf16.  tile: 0 lets the planner choose; 128 or 256 force a one-CTA tile of
 // that width; kTilePair forces the CTA-pair 256 x 256 tile, kTilePair | (S << 8) that
 // tile with S K splits (S = 0: the planner chooses, S = 1: unsplit),
-// kTilePair | kTileStreamK the pair tile with the stream-K schedule.
+// kTilePair | kTileStreamK | (S << 8) the pair tile with the stream-K schedule, each
+// left-over tile cut into about S K segments (S = 0: shared out over all pairs).
 constexpr int kTilePair = 2;
 constexpr int kTileStreamK = 1 << 16;
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
@@ -112,7 +113,9 @@ struct AttnPlan {
 int attn_vt_pitch(int T);
 cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16* vt, __nv_bfloat16* out, int batch,
                            int T, int H, int G, int hd);
-cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream);
+cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream);  // both kernels
+cudaError_t attention_transpose_launch(const AttnPlan& p, cudaStream_t stream);  // v -> vt
+cudaError_t attention_core_launch(const AttnPlan& p, int* err, cudaStream_t stream);  // the attention
 
 // ---------------------------------------------------------------- other kernels (kernels.cu)
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,

@@ -218,8 +218,10 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
     q.end(rmsnorm_launch(c->h, L.attn_norm, c->xn, R, d, m.rms_eps, R, 0, 0, c->stream), "rmsnorm");
     q.begin(DCL_K_GEMM_QKV);
     q.end(gemm_launch(P[0], c->derr, c->stream), "gemm_qkv");
+    q.begin(DCL_K_VTRANSPOSE);
+    q.end(attention_transpose_launch(c->attn_plan, c->stream), "v_transpose");
     q.begin(DCL_K_ATTENTION);
-    q.end(attention_launch(c->attn_plan, c->derr, c->stream), "attention");
+    q.end(attention_core_launch(c->attn_plan, c->derr, c->stream), "attention");
     q.begin(DCL_K_GEMM_O);
     q.end(gemm_launch(P[1], c->derr, c->stream), "gemm_o");
     q.begin(DCL_K_RMSNORM);
@@ -277,8 +279,8 @@ dcl_status build_graph(dcl_ctx* c) {
 
 // Tile of one of the step's GEMMs ("qkv", "o", "gateup", "down", "lmhead") forced by the
 // environment variable DCL_GEMM_TILES, e.g. "o=128,down=pair:2" (128 / 256 = one-CTA tile
-// width, pair[:S] = CTA-pair tile with S K-splits, pair:sk = CTA-pair tile with the
-// stream-K schedule); 0 = let the planner choose.
+// width, pair[:S] = CTA-pair tile with S K-splits, pair:sk[:S] = CTA-pair tile with the
+// stream-K schedule, S segments per left-over tile); 0 = let the planner choose.
 int tile_override(const char* name) {
   const char* env = getenv("DCL_GEMM_TILES");
   if (!env) return 0;
@@ -288,7 +290,7 @@ int tile_override(const char* name) {
     const size_t len = e ? (size_t)(e - s) : strlen(s);
     if (len > n && strncmp(s, name, n) == 0 && s[n] == '=') {
       const char* v = s + n + 1;
-      if (strncmp(v, "pair:sk", 7) == 0) return kTilePair | kTileStreamK;
+      if (strncmp(v, "pair:sk", 7) == 0) return kTilePair | kTileStreamK | ((v[7] == ':' ? atoi(v + 8) : 0) << 8);
       if (strncmp(v, "pair", 4) == 0) return kTilePair | ((v[4] == ':' ? atoi(v + 5) : 0) << 8);
       return atoi(v);
     }

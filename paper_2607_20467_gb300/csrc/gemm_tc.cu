@@ -21,6 +21,8 @@
 #include <cudaTypedefs.h>
 #include <string.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "tc_ptx.cuh"
 
@@ -782,7 +784,8 @@ __device__ __noinline__ bool fixup_to_tmem(const CUtensorMap* tmw, int y0, int s
 //   plain    : pair c takes tiles c, c + C, ...  (C pairs)
 //   split-K  : items w = split * tiles + tile (split-major), pair c takes w = c, c + C, ...
 //   stream-K : the first (tiles / C) * C tiles as plain rounds; the R left-over tiles'
-//              R * U K units are then cut into C equal contiguous ranges, one per pair.
+//              R * U K units are then cut into Csk <= C equal contiguous ranges, one for
+//              each of the first Csk pairs (Csk = 2R: every left-over tile in two halves).
 //              A range covers the tail of one tile and/or the head of the next; the pair
 //              processes the head first (it only writes a partial) and the tail second
 //              (the tile's last segment: it waits for the other segments' partials, sums
@@ -790,7 +793,8 @@ __device__ __noinline__ bool fixup_to_tmem(const CUtensorMap* tmw, int y0, int s
 //              itself waiting.
 enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3 };
 struct Sched {
-  int tiles, ku, C, splits, streamk;
+  int tiles, ku, C, splits;
+  int streamk;  // 0: off; else the number of pairs (<= C) that share the left-over tiles
 };
 struct Item {
   int t, ku0, ku1, kind;
@@ -819,10 +823,10 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
     it.kind = IT_PLAIN;
     return true;
   }
-  if (!s.streamk) return false;
+  if (!s.streamk || c >= s.streamk) return false;
   const int first = rounds * s.C;
   const long RU = (long)(s.tiles - first) * s.ku;
-  const long lo = (long)c * RU / s.C, hi = (long)(c + 1) * RU / s.C;
+  const long lo = (long)c * RU / s.streamk, hi = (long)(c + 1) * RU / s.streamk;
   if (hi <= lo) return false;
   const int ta = (int)(lo / s.ku), tb = (int)((hi - 1) / s.ku);
   const int k = idx - rounds;
@@ -843,7 +847,7 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
   } else {
     return false;
   }
-  const int c_first = (int)((((long)rel * s.ku + 1) * s.C - 1) / RU);  // owner of the tile's first unit
+  const int c_first = (int)((((long)rel * s.ku + 1) * s.streamk - 1) / RU);  // owner of the tile's first unit
   it.t = first + rel;
   it.rel = rel;
   it.ku0 = k0;
@@ -1236,9 +1240,11 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   // Tile choice (measured on the LLaDA-8B step's shapes): the CTA-pair tile keeps the
   // tensor pipe busiest and is used whenever M spans more than one 128-row tile; a
   // residual GEMM whose pair tiles fill less than 3/4 of the GPU and whose K is long
-  // splits K in two; small M uses one-CTA tiles, 256 or 128 wide by wave fill.  Stream-K
-  // is available on request (kTileStreamK): with a fix-up that reads (segments - 1) fp32
-  // partials of 256 KB per tile it lost to the plain schedule on those shapes.
+  // splits K in two (ordered adds into the residual stream); small M uses one-CTA tiles,
+  // 256 or 128 wide by wave fill.  Stream-K (left-over tiles cut into K segments, fp32
+  // partials summed in K order in TMEM) is available on request: every partial costs a
+  // 256 KB store and reload per tile, and at ~55 GB/s of stores per SM when all SMs store
+  // at once that outweighs the balance it buys on these shapes.
   const bool pair_forced = (tile & 0xff) == kTilePair;
   const bool sk_forced = pair_forced && (tile & kTileStreamK);
   int bn = pair_forced ? kTilePair : (tile & 0xff), cg = 1, splits = 1, streamk = 0;
@@ -1250,6 +1256,7 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   const long units = (K + BK * KA2 - 1) / (BK * KA2);
   const long pair_tiles = (long)((M + 255) / 256) * ((N + 255) / 256);
   const long left = pairs > 0 ? pair_tiles % pairs : 0;
+  const int split_auto = (epi == EPI_RESID_F32 && 4 * pair_tiles < 3L * pairs && nkb >= 128) ? 2 : 1;
   if (pair_forced && pairs < 1) {
     *why = "gemm: the CTA-pair tile needs two SMs";
     return cudaErrorInvalidValue;
@@ -1257,21 +1264,22 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   if (bn == kTilePair) {
     bn = 256;
     cg = 2;
-    splits = forced_splits > 0 ? forced_splits : 1;
     if (sk_forced) {
-      if (forced_splits > 1 || left == 0 || left * units < pairs) {
-        *why = "gemm: stream-K needs one split and a partial last round of at least one K unit per pair";
+      // forced_splits here counts segments per left-over tile (0: all pairs share them)
+      const long csk = forced_splits == 0 ? pairs : std::min<long>(pairs, (long)forced_splits * left);
+      if (forced_splits == 1 || left == 0 || left * units < csk) {
+        *why = "gemm: stream-K needs a partial last round and at least one K block per sharing pair";
         return cudaErrorInvalidValue;
       }
-      streamk = 1;
-    } else if (forced_splits == 0) {
-      splits = (epi == EPI_RESID_F32 && 4 * pair_tiles < 3L * pairs && nkb >= 128) ? 2 : 1;
+      streamk = (int)csk;
+    } else {
+      splits = forced_splits > 0 ? forced_splits : split_auto;
     }
   } else if (bn == 0) {
     if (M > BM && pairs >= 1) {
       bn = 256;
       cg = 2;
-      splits = (epi == EPI_RESID_F32 && 4 * pair_tiles < 3L * pairs && nkb >= 128) ? 2 : 1;
+      splits = split_auto;
     } else if (wide_only) {
       bn = 256;
     } else {
@@ -1339,7 +1347,9 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   }
   if (cg == 2) {
     plan->n_tiles = (int)pair_tiles;
-    const long items = streamk ? pairs : pair_tiles * splits;
+    // stream-K: all pairs when there are plain rounds, else only the sharing ones (the
+    // kernel derives the round stride from the grid)
+    const long items = streamk ? (pair_tiles >= pairs ? pairs : streamk) : pair_tiles * splits;
     plan->grid = 2 * (int)(items < pairs ? items : pairs);
     plan->smem = SMEM2;
     if (splits > 1) {
@@ -1348,13 +1358,13 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     }
     if (streamk) {
       // left-over tile r's K units [r*U, (r+1)*U) are owned by pairs
-      // owner(r*U) .. owner((r+1)*U - 1), owner(u) = ((u + 1) * C - 1) / (R * U); all
+      // owner(r*U) .. owner((r+1)*U - 1), owner(u) = ((u + 1) * Csk - 1) / (R * U); all
       // but the last write a partial slot
-      const long RU = left * units;
+      const long RU = left * units, csk = streamk;
       long slots = 1;
       for (long r = 0; r < left; ++r) {
-        const long c0 = ((r * units + 1) * pairs - 1) / RU;
-        const long c1 = (((r + 1) * units) * pairs - 1) / RU;
+        const long c0 = ((r * units + 1) * csk - 1) / RU;
+        const long c1 = (((r + 1) * units) * csk - 1) / RU;
         slots = (c1 - c0) > slots ? (c1 - c0) : slots;
       }
       plan->ws_slots = (int)slots;

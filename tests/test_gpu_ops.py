@@ -64,25 +64,30 @@ def test_rmsnorm(ops, rows, d):
 # ------------------------------------------------------------------ tcgen05 GEMM
 PAIR, SK = 2, 1 << 16
 # auto, one-CTA 128 / 256 columns, CTA pair (library's K schedule), CTA pair unsplit,
-# CTA pair with 2 / 3 K splits, CTA pair with the stream-K schedule
-TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK]
+# CTA pair with 2 / 3 K splits, CTA pair with stream-K over all pairs / in K halves
+TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK, PAIR | SK | (2 << 8)]
 
 
 def _splits(tile):
-    return max(1, (tile >> 8) & 0xff) if (tile & 0xff) == PAIR else 1
+    if (tile & 0xff) != PAIR or tile & SK:
+        return 1
+    return max(1, (tile >> 8) & 0xff)
 
 
-def _streamk_possible(M, N, K):
-    """Stream-K needs a partly filled last round of pair tiles with at least one 64-wide
-    K block per CTA pair."""
+def _streamk_possible(M, N, K, segments):
+    """Stream-K needs a partly filled last round of pair tiles and at least one 64-wide
+    K block for every sharing CTA pair."""
     pairs = torch.cuda.get_device_properties(0).multi_processor_count // 2
     left = ((M + 255) // 256) * ((N + 255) // 256) % pairs
-    return left > 0 and left * (K // 64) >= pairs
+    sharing = pairs if segments == 0 else min(pairs, segments * left)
+    return segments != 1 and left > 0 and left * (K // 64) >= sharing
 
 
 def _unsupported(M, N, K, tile):
     """True when the tile choice cannot run this shape (then the call must be refused)."""
-    return K // 64 < _splits(tile) or (tile & SK and not _streamk_possible(M, N, K))
+    if tile & SK:
+        return not _streamk_possible(M, N, K, (tile >> 8) & 0xff)
+    return K // 64 < _splits(tile)
 
 
 @pytest.mark.parametrize("tile", TILES)
@@ -126,7 +131,7 @@ def test_linear_residual(ops, M, N, K, tile):
 
 
 @pytest.mark.parametrize("tile,mode", [(PAIR | (3 << 8), 1), (PAIR | (2 << 8), 0), (0, 1), (0, 0),
-                                       (PAIR | SK, 0), (PAIR | SK, 1)])
+                                       (PAIR | SK, 0), (PAIR | SK, 1), (PAIR | SK | (2 << 8), 1)])
 def test_linear_split_k_is_deterministic(ops, tile, mode):
     """Split-K and stream-K partial sums are combined in K order: two runs give the same
     bits."""
@@ -170,7 +175,7 @@ def test_attention_non_causal(ops, B, T, H, G, hd):
 
 
 # ------------------------------------------------------------------ LM head + confidence
-@pytest.mark.parametrize("tile", [0, 256, PAIR, PAIR | SK])
+@pytest.mark.parametrize("tile", [0, 256, PAIR, PAIR | SK, PAIR | SK | (2 << 8)])
 @pytest.mark.parametrize("R,V,d,sz", [(37, 4096, 256, 12.0), (5, 1000, 128, 6.0), (130, 4096, 64, 20.0),
                                       (300, 4096, 256, 12.0), (64, 126464, 4096, 15.0),
                                       (300, 126464, 4096, 15.0)])
