@@ -55,12 +55,14 @@ struct EpiParams {
   int head_dim = 0;
   int seq_T = 1;                    // rows per sequence (position = row % seq_T)
   int vocab = 0;
+  int vt_heads = 0;                 // QKV: > 0 writes v transposed (G kv heads) through tv
 };
 
 struct GemmPlan {
   CUtensorMap ta, tb;
   CUtensorMap tc;        // pair tiles: the output (bf16 / fp32 boxes of 32 rows x 128 bytes)
   CUtensorMap tw;        // pair tiles with partials: the fp32 workspace [rows][256]
+  CUtensorMap tv;        // QKV with ep.vt_heads > 0: v^T boxes [64 channels][32 tokens]
   int M = 0, N = 0, K = 0;
   int bn = 256;          // output columns per tile
   int cg = 1;            // 1: one CTA per 128 x bn tile; 2: a CTA pair per 256 x 256 tile
@@ -92,6 +94,9 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
 // (>= ws_needed floats, 16-byte aligned) a plan needs; they may be shared by plans that
 // run one after another on one stream.
 cudaError_t gemm_bind_scratch(GemmPlan* plan, int* flags, float* ws);
+// Make a CTA-pair QKV plan write v transposed into vt (bf16 [batch*G][hd][Tp]) instead of
+// the v columns of its output; false (plan unchanged) when the shape does not allow it.
+bool gemm_fuse_vt(GemmPlan* plan, void* vt, int batch, int T, int G, int hd, int Tp);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
 // cuTensorMapEncodeTiled through the runtime's driver entry point: dims / box in elements

@@ -77,6 +77,7 @@ struct dcl_ctx {
   dcl_decode_config dcfg{};
   std::vector<GemmPlan> plans;  // 4 per layer + LM head
   AttnPlan attn_plan;
+  bool vt_fused = false;  // the QKV GEMMs write v transposed (no transpose launch)
   cudaGraphExec_t gexec = nullptr;
   bool profiling = false;
   std::vector<Launch> launches;
@@ -218,8 +219,10 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
     q.end(rmsnorm_launch(c->h, L.attn_norm, c->xn, R, d, m.rms_eps, R, 0, 0, c->stream), "rmsnorm");
     q.begin(DCL_K_GEMM_QKV);
     q.end(gemm_launch(P[0], c->derr, c->stream), "gemm_qkv");
-    q.begin(DCL_K_VTRANSPOSE);
-    q.end(attention_transpose_launch(c->attn_plan, c->stream), "v_transpose");
+    if (!c->vt_fused) {
+      q.begin(DCL_K_VTRANSPOSE);
+      q.end(attention_transpose_launch(c->attn_plan, c->stream), "v_transpose");
+    }
     q.begin(DCL_K_ATTENTION);
     q.end(attention_core_launch(c->attn_plan, c->derr, c->stream), "attention");
     q.begin(DCL_K_GEMM_O);
@@ -337,6 +340,11 @@ dcl_status build_plans(dcl_ctx* c) {
   }
   if (attention_plan(&c->attn_plan, c->qkv, c->vt, c->attn, c->B, c->T, m.n_heads, m.n_kv_heads, hd) != cudaSuccess)
     return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
+  c->vt_fused = true;
+  for (int l = 0; l < m.n_layers && c->vt_fused; ++l)
+    c->vt_fused = gemm_fuse_vt(&c->plans[4 * l], c->vt, c->B, c->T, m.n_kv_heads, hd, attn_vt_pitch(c->T));
+  if (!c->vt_fused)
+    for (int l = 0; l < m.n_layers; ++l) c->plans[4 * l].ep.vt_heads = 0;
   EpiParams el;
   el.out = c->part;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,

@@ -493,6 +493,16 @@ struct Stage {
     }
     ++n;
   }
+  // the same for a box of a 3-D tensor (x, y, z)
+  __device__ __forceinline__ void issue3(const CUtensorMap* tm, uint32_t box, int x, int y, int z) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (live) tma_store_3d(tm, box, x, y, z);
+      bulk_commit();
+    }
+    ++n;
+  }
   // every store issued so far has completed and is ordered before later generic
   // accesses of this warp (before a release that publishes it)
   __device__ __forceinline__ void drain() {
@@ -564,8 +574,8 @@ __device__ __forceinline__ void store_bf16_box(const Src& s, Stage& o, const CUt
 // The fused epilogues of a 256 x 256 pair tile, for one warp's 32-row band of one CTA
 // half.  All tcgen05.ld run warp-uniformly.
 template <int EPI>
-__device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUtensorMap* tmc, int row, int n_blk,
-                                              int M, int N, const EpiParams& ep) {
+__device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUtensorMap* tmc, const CUtensorMap* tmv,
+                                              int row, int n_blk, int M, int N, const EpiParams& ep) {
   const int n0 = n_blk * 256;
   if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
@@ -621,6 +631,24 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
         }
         o.issue(tmc, b0, n0 + hb, o.row0, false);
         if (hd == 128) o.issue(tmc, b1, n0 + hb + 64, o.row0, false);
+      }
+    } else if (ep.vt_heads > 0) {
+      // v columns leave transposed, as the attention's K-major operand: boxes of 64
+      // channels x 32 tokens of vt [batch * G][hd][T] (the band's 32 rows are 32
+      // consecutive tokens of one sequence: T is a multiple of 32)
+      const int bz = o.row0 / ep.seq_T, t0 = o.row0 - bz * ep.seq_T;
+#pragma unroll 1
+      for (int c = 0; c < 256 && n0 + c < N; c += 64) {
+        const int cv = n0 + c - ep.rope_cols, g = cv / ep.head_dim, d0 = cv - g * ep.head_dim;
+        const uint32_t b = o.acquire();
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          float v[32];
+          src_cols(s, c + 32 * h, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) st_shared_u16(b + (uint32_t)((32 * h + e) * 64 + 2 * o.lane), bf16_bits(v[e]));
+        }
+        o.issue3(tmv, b, t0, d0, bz * ep.vt_heads + g);
       }
     } else {
 #pragma unroll 1
@@ -871,7 +899,8 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
 template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
-                    const __grid_constant__ CUtensorMap tmc, const __grid_constant__ CUtensorMap tmw, int M,
+                    const __grid_constant__ CUtensorMap tmc, const __grid_constant__ CUtensorMap tmw,
+                    const __grid_constant__ CUtensorMap tmv, int M,
                     int N, int K, EpiParams ep, int splits, int streamk, int ws_slots, int* flags, float* ws,
                     int* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -1043,7 +1072,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       s.taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
       s.row = row_local;
       if (it.kind == IT_PLAIN) {
-        epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+        epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
         int* flag = flags + t * 2 + rank;
@@ -1053,7 +1082,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             report_error(err, DERR_WAIT_TIMEOUT);
           }
           epilogue_bar();
-          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
           o.drain();
           epilogue_bar();
           if (et == 0) {
@@ -1080,7 +1109,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             s.part = ws + ((size_t)t * S1 * 2 + rank) * 128 * 256;
             s.part_stride = (size_t)2 * 128 * 256;
             s.nparts = S1;
-            if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+            if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
             epilogue_bar();
             if (et == 0) atomicExch(flag, 0);
           }
@@ -1111,7 +1140,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
               s.tsum = tsum;
             }
           }
-          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, row, n_blk, M, N, ep);
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
           epilogue_bar();
           if (et == 0) atomicExch(flag, 0);
         }
@@ -1196,7 +1225,7 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.tc, p.tw, p.M, p.N, p.K, p.ep, p.splits, p.streamk,
+  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.tc, p.tw, p.tv, p.M, p.N, p.K, p.ep, p.splits, p.streamk,
                                                 p.ws_slots, p.flags, p.ws, err);
   return cudaGetLastError();
 }
@@ -1331,6 +1360,8 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   plan->ws = nullptr;
   memset(&plan->tc, 0, sizeof(plan->tc));
   memset(&plan->tw, 0, sizeof(plan->tw));
+  memset(&plan->tv, 0, sizeof(plan->tv));
+  plan->ep.vt_heads = 0;
   if (cg == 2 && epi != EPI_LMHEAD) {
     const bool f32 = (epi == EPI_RESID_F32);
     const int es = f32 ? 4 : 2;
@@ -1377,6 +1408,19 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     plan->smem = (bn == 256) ? Cfg<256>::SMEM : Cfg<128>::SMEM;
   }
   return cudaSuccess;
+}
+
+bool gemm_fuse_vt(GemmPlan* p, void* vt, int batch, int T, int G, int hd, int Tp) {
+  if (p->cg != 2 || p->epi != EPI_QKV_ROPE || T % 32 != 0 || p->ep.rope_cols % 256 != 0 ||
+      (reinterpret_cast<uintptr_t>(vt) & 15) || Tp % 8 != 0)
+    return false;
+  const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
+  const uint64_t strides[2] = {(uint64_t)Tp * 2, (uint64_t)hd * Tp * 2};
+  const uint32_t box[3] = {32, 64, 1};
+  if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return false;
+  p->ep.vt_heads = G;
+  return true;
 }
 
 cudaError_t gemm_bind_scratch(GemmPlan* p, int* flags, float* ws) {

@@ -201,6 +201,12 @@ __device__ __forceinline__ float4 ld_shared_v4(uint32_t addr) {
                : "memory");
   return v;
 }
+__device__ __forceinline__ void st_shared_u16(uint32_t addr, uint16_t v) {
+  asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
+}
+__device__ __forceinline__ uint16_t bf16_bits(float x) {  // round to nearest even
+  return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
 // Byte offset of 16-byte chunk k of row r in a 1024-byte-aligned box of 128-byte rows
 // written / read by TMA with 128-byte swizzle.
 __device__ __forceinline__ uint32_t swz(int r, int k) { return (uint32_t)(r * 128 + ((k ^ (r & 7)) << 4)); }
