@@ -47,6 +47,8 @@ __global__ void __launch_bounds__(256) v_transpose_kernel(const __nv_bfloat16* _
                                                           __nv_bfloat16* __restrict__ vt, int T, int Tp, int cols,
                                                           int v0, int ghd) {
   __shared__ __nv_bfloat16 tile[64][72];  // [channel][token], rows padded by 16 bytes
+  pdl_wait();
+  pdl_launch_dependents();
   const int t0 = blockIdx.x * 64, c0 = blockIdx.y * 64, b = blockIdx.z;
   for (int i = threadIdx.x; i < 64 * 8; i += 256) {
     const int r = i >> 3, cv = (i & 7) * 8;  // token row, first channel of the vector
@@ -125,6 +127,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *holder_ptr;
+  pdl_wait();  // the previous kernel of the step has completed
+  pdl_launch_dependents();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -404,8 +408,7 @@ cudaError_t launch_attn(const AttnPlan& p, int* err, cudaStream_t stream) {
     attr_set = true;
   }
   dim3 grid((p.T + 127) / 128, p.H, p.batch);
-  kern<<<grid, AT_THREADS, AttnCfg<HD>::SMEM, stream>>>(p.tq, p.tv, p.to, p.T, p.H, p.G, err);
-  return cudaGetLastError();
+  return launch_pdl(kern, grid, AT_THREADS, AttnCfg<HD>::SMEM, stream, p.tq, p.tv, p.to, p.T, p.H, p.G, err);
 }
 
 }  // namespace
@@ -454,8 +457,8 @@ cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16*
 cudaError_t attention_transpose_launch(const AttnPlan& p, cudaStream_t stream) {
   const int cols = (p.H + 2 * p.G) * p.hd, ghd = p.G * p.hd;
   dim3 tgrid((attn_vt_pitch(p.T) + 63) / 64, (ghd + 63) / 64, p.batch);
-  v_transpose_kernel<<<tgrid, 256, 0, stream>>>(p.qkv, p.vt, p.T, attn_vt_pitch(p.T), cols, (p.H + p.G) * p.hd, ghd);
-  return cudaGetLastError();
+  return launch_pdl(v_transpose_kernel, tgrid, 256, 0, stream, p.qkv, p.vt, p.T, attn_vt_pitch(p.T), cols,
+                    (p.H + p.G) * p.hd, ghd);
 }
 
 cudaError_t attention_core_launch(const AttnPlan& p, int* err, cudaStream_t stream) {

@@ -253,6 +253,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *holder_ptr;
+  pdl_wait();  // the previous kernel of the step has completed
+  pdl_launch_dependents();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -955,6 +957,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   cluster_sync_all();  // the peer's barriers exist before any remote arrive / multicast
   tc_fence_after();
   const uint32_t tmem_base = *holder_ptr;
+  pdl_wait();  // the previous kernel of the step has completed
+  pdl_launch_dependents();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1212,8 +1216,7 @@ cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream>>>(p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
-  return cudaGetLastError();
+  return launch_pdl(kern, p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream, p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
 }
 
 template <int EPI>
@@ -1225,9 +1228,8 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<p.grid, NUM_THREADS, SMEM2, stream>>>(p.ta, p.tb, p.tc, p.tw, p.tv, p.M, p.N, p.K, p.ep, p.splits, p.streamk,
-                                                p.ws_slots, p.flags, p.ws, err);
-  return cudaGetLastError();
+  return launch_pdl(kern, p.grid, NUM_THREADS, SMEM2, stream, p.ta, p.tb, p.tc, p.tw, p.tv, p.M, p.N, p.K, p.ep, p.splits,
+                    p.streamk, p.ws_slots, p.flags, p.ws, err);
 }
 
 double wave_efficiency(long tiles, int sms) {

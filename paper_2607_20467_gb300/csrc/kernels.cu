@@ -22,6 +22,8 @@ __global__ void embed_remask_kernel(int32_t* __restrict__ x, const int32_t* __re
                                     int window, int mask_id, int vocab,
                                     const __nv_bfloat16* __restrict__ embed, int d,
                                     float* __restrict__ h, int* err) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int row = blockIdx.x;
   const int b = row / T, t = row % T;
   __shared__ int tok_s;
@@ -55,6 +57,8 @@ __global__ void __launch_bounds__(THREADS) rmsnorm_kernel(const float* __restric
                                                           __nv_bfloat16* __restrict__ y, int d,
                                                           float eps, int rows_per_seq,
                                                           int seq_stride, int row_offset) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int r = blockIdx.x;
   const int in_row = (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
@@ -93,6 +97,8 @@ template <int VPT, int ROWS>
 __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
     const float* __restrict__ x, const __nv_bfloat16* __restrict__ gain, __nv_bfloat16* __restrict__ y,
     int rows, int d, float eps, int rows_per_seq, int seq_stride, int row_offset) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int sub = threadIdx.x >> 7, t = threadIdx.x & 127;
   const int r = blockIdx.x * ROWS + sub;
   const bool live = r < rows;
@@ -176,6 +182,8 @@ __device__ __forceinline__ void write_conf(const Part& a, int32_t* top1, float* 
 __global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows, int nblk,
                                       int32_t* __restrict__ top1, float* __restrict__ p1,
                                       float* __restrict__ p2) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -234,6 +242,8 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
                                   int32_t* __restrict__ k_out, int32_t* __restrict__ steps,
                                   const int32_t* __restrict__ ids, const float* __restrict__ c,
                                   int N, int M, DcvParams prm, int32_t* done_count) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int b = blockIdx.x;
   const int T = N + M;
   const int pb = p[b];
@@ -358,8 +368,7 @@ cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, 
                                 int mask_id, int vocab, const __nv_bfloat16* embed, int d, float* h,
                                 int* err, cudaStream_t stream) {
   if (d % 8) return cudaErrorInvalidValue;
-  embed_remask_kernel<<<batch * T, 128, 0, stream>>>(x, p, T, window, mask_id, vocab, embed, d, h, err);
-  return cudaGetLastError();
+  return launch_pdl(embed_remask_kernel, batch * T, 128, 0, stream, x, p, T, window, mask_id, vocab, embed, d, h, err);
 }
 
 cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows, int d,
@@ -369,30 +378,27 @@ cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloa
   const int vpt = (d / 4 + 127) / 128;  // float4 per thread with 128 threads per row
   const int grid2 = (rows + 1) / 2;
   switch (vpt) {
-    case 1: rmsnorm_reg_kernel<1, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
-    case 2: rmsnorm_reg_kernel<2, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
-    case 4: case 3: rmsnorm_reg_kernel<4, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+    case 1: return launch_pdl(rmsnorm_reg_kernel<1, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
+    case 2: return launch_pdl(rmsnorm_reg_kernel<2, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
+    case 4: case 3: return launch_pdl(rmsnorm_reg_kernel<4, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
     case 5: case 6: case 7: case 8:
-      rmsnorm_reg_kernel<8, 2><<<grid2, 256, 0, stream>>>(x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset); break;
+      return launch_pdl(rmsnorm_reg_kernel<8, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
     default:
-      rmsnorm_kernel<256><<<rows, 256, 0, stream>>>(x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
+      return launch_pdl(rmsnorm_kernel<256>, rows, 256, 0, stream, x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
   }
-  return cudaGetLastError();
 }
 
 cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
                                   float* p2, cudaStream_t stream) {
   const int threads = 256;
   const int blocks = (rows * 32 + threads - 1) / threads;
-  lmhead_combine_kernel<<<blocks, threads, 0, stream>>>(part, rows, nblk, top1, p1, p2);
-  return cudaGetLastError();
+  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, rows, nblk, top1, p1, p2);
 }
 
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
                               const int32_t* ids, const float* c, int batch, int N, int M,
                               const DcvParams& prm, int32_t* done_count, cudaStream_t stream) {
-  dcv_commit_kernel<<<batch, 32, 0, stream>>>(x, p, k_out, steps, ids, c, N, M, prm, done_count);
-  return cudaGetLastError();
+  return launch_pdl(dcv_commit_kernel, batch, 32, 0, stream, x, p, k_out, steps, ids, c, N, M, prm, done_count);
 }
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
