@@ -22,7 +22,13 @@ Readings where the paper is silent or inconsistent (each one is also a test):
     advance (the order of Algorithm 1);
   * drafts are refreshed at every future position, masked or already drafted;
   * decisions compare the confidence and the threshold as float32 values, the
-    precision in which the CUDA kernel takes them.
+    precision in which the CUDA kernel takes them;
+  * the approximate cache (``kv_cache = 1``; the paper pairs DC-Leap with a dLLM cache in
+    Sec. 4 / Tab. 6 without describing its policy): per row, a step computes all
+    positions at the first step and whenever the block-aligned prefix end
+    N + Bk * floor((p - N) / Bk) changes, else only the positions from that prefix end on,
+    attending to the keys and values the prefix had at its last refresh
+    (``model.forward_rows``).
 """
 from __future__ import annotations
 
@@ -80,13 +86,22 @@ def commit_and_draft(x: np.ndarray, p: int, ids: np.ndarray, c: np.ndarray,
     return K
 
 
+def prefix_end(p: int, n_prompt: int, block_len: int) -> int:
+    """Block-aligned start of the current block: N + Bk * floor((p - N) / Bk)."""
+    return n_prompt + block_len * ((p - n_prompt) // block_len)
+
+
 def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
              max_steps: int = 1 << 30, record: bool = True) -> dict:
     """Algorithm 1 for a batch of independent rows.
 
-    predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) for the generation positions.
-    Returns the final x [B][T], per-row steps, the K of every step, and (if ``record``)
-    the forward input of every step and the predictions it produced.
+    predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) for the generation positions.  With
+    ``cfg.kv_cache`` it is called as predict_fn(tokens[T], start, state): only positions
+    >= start need be computed and ``state`` is the row's cache; start is 0 at the first
+    step and whenever prefix_end(p) changes (a refresh), else prefix_end(p).
+    Returns the final x [B][T], per-row steps, the K of every step, the start of every
+    step (-1 for finished rows), and (if ``record``) the forward input of every step and
+    the predictions it produced.
     """
     prompt = np.atleast_2d(np.asarray(prompt, dtype=np.int32))
     B, N = prompt.shape
@@ -97,10 +112,12 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
     x[:, :N] = prompt
     p = np.full(B, N, dtype=np.int64)
     steps = np.zeros(B, dtype=np.int64)
-    ks, inputs, preds = [], [], []
+    ks, starts, inputs, preds = [], [], [], []
+    caches = [{"pe": None} for _ in range(B)]
     n_iter = 0
     while (p < T).any() and n_iter < max_steps:
         k_step = np.zeros(B, dtype=np.int64)
+        s_step = np.full(B, -1, dtype=np.int64)
         in_step = np.empty((B, T), dtype=np.int32)
         pr = np.zeros((3, B, M))
         for b in range(B):
@@ -109,7 +126,14 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
                 continue
             remask(x[b], int(p[b]), L, mask_id)                  # (i)
             in_step[b] = x[b]
-            ids, p1, p2 = predict_fn(x[b].copy())                # (ii)
+            if cfg.kv_cache:                                     # (ii), approximate cache
+                pe = prefix_end(int(p[b]), N, cfg.block_len)
+                s_step[b] = 0 if caches[b]["pe"] != pe else pe
+                ids, p1, p2 = predict_fn(x[b].copy(), int(s_step[b]), caches[b])
+                caches[b]["pe"] = pe
+            else:                                                # (ii)
+                s_step[b] = 0
+                ids, p1, p2 = predict_fn(x[b].copy())
             full_ids = np.zeros(T, dtype=np.int32)
             full_c = np.zeros(T, dtype=np.float64)
             full_ids[N:] = ids
@@ -119,10 +143,11 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             steps[b] += 1
             pr[0, b], pr[1, b], pr[2, b] = ids, p1, p2
         ks.append(k_step)
+        starts.append(s_step)
         if record:
             inputs.append(in_step)
             preds.append(pr)
         n_iter += 1
-    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "inputs": inputs,
+    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "start": np.array(starts), "inputs": inputs,
             "preds": preds, "n_iter": n_iter, "done": bool((p >= T).all())}
 

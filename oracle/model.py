@@ -122,6 +122,82 @@ def forward_hidden(shape, weights: dict, tokens: np.ndarray, bf16_operands: bool
     return _maybe_bf16(rms_norm(h, weights["final_norm"], shape.rms_eps), bf16_operands)
 
 
+# ---------------------------------------------------------------- approximate prefix cache
+# The paper's accelerated setting pairs DC-Leap with a dLLM cache (Sec. 4, Tab. 6) whose
+# policy it does not describe.  The reading built here keeps, per layer, the keys and
+# values of all T positions of a sequence between steps.  At the first step and whenever
+# the block-aligned prefix end N + Bk * floor((p - N) / Bk) changes, a step computes all
+# T positions (refreshing every stored key and value); otherwise it computes only the
+# positions from that prefix end on: their fresh keys and values overwrite the stored
+# ones, and their queries attend to all T stored positions, so the prefix contributes the
+# keys and values of its last refresh.
+
+
+def block_rows(shape, lw: dict, h: np.ndarray, pos: np.ndarray, kv, angles: np.ndarray,
+               bf16_operands: bool = False) -> np.ndarray:
+    """One block for the rows h [len(pos), d] at positions ``pos`` of one sequence.
+
+    kv = [k, v], each [T, G, hd]: the layer's stored keys and values; the rows' own keys
+    and values (after RoPE, rounded like the model stores them) are written at ``pos``
+    before their queries attend to all T stored positions.  ``angles`` are the RoPE angles
+    of ``pos``."""
+    n = h.shape[0]
+    H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    r = bf16_operands
+    xn = _maybe_bf16(rms_norm(h, lw["attn_norm"], shape.rms_eps), r)
+    q = (xn @ _f64(lw["wq"]).T).reshape(n, H, hd)
+    k = (xn @ _f64(lw["wk"]).T).reshape(n, G, hd)
+    v = _maybe_bf16((xn @ _f64(lw["wv"]).T).reshape(n, G, hd), r)
+    q = _maybe_bf16(apply_rope(q, angles), r)
+    kv[0][pos] = _maybe_bf16(apply_rope(k, angles), r)
+    kv[1][pos] = v
+    h = h + _maybe_bf16(attention(q, kv[0], kv[1]), r) @ _f64(lw["wo"]).T
+    xn = _maybe_bf16(rms_norm(h, lw["mlp_norm"], shape.rms_eps), r)
+    a = _maybe_bf16(silu(xn @ _f64(lw["w_gate"]).T) * (xn @ _f64(lw["w_up"]).T), r)
+    return h + a @ _f64(lw["w_down"]).T
+
+
+def forward_rows(shape, weights: dict, tokens: np.ndarray, pos: np.ndarray, kv_store: list,
+                 bf16_operands: bool = False) -> np.ndarray:
+    """Final-normed hidden states [len(pos), d] of positions ``pos`` of one sequence,
+    reading and updating ``kv_store`` (one [k, v] pair of [T, G, hd] arrays per layer).
+    With every position and any store this is ``forward_hidden``."""
+    tokens = np.asarray(tokens)
+    pos = np.asarray(pos, dtype=np.int64)
+    if tokens.min() < 0 or tokens.max() >= shape.vocab:
+        raise ValueError("token id out of range")
+    h = _f64(weights["embed"])[tokens[pos]]
+    angles = rope_angles(len(tokens), shape.head_dim, shape.rope_theta)[pos]
+    for lw, kv in zip(weights["layers"], kv_store):
+        h = block_rows(shape, lw, h, pos, kv, angles, bf16_operands)
+    return _maybe_bf16(rms_norm(h, weights["final_norm"], shape.rms_eps), bf16_operands)
+
+
+def new_kv_store(shape, T: int) -> list:
+    G, hd = shape.n_kv_heads, shape.head_dim
+    return [[np.zeros((T, G, hd)), np.zeros((T, G, hd))] for _ in range(shape.n_layers)]
+
+
+def predict_from(shape, weights: dict, tokens: np.ndarray, start: int, state: dict, n_prompt: int,
+                 bf16_operands: bool = False):
+    """(ids, p1, p2) over the generation positions [n_prompt, T) computing only positions
+    >= start (the others are returned as -1 / NaN); ``state["kv"]`` is the sequence's
+    key / value store, created on first use."""
+    T = len(tokens)
+    if state.get("kv") is None:
+        state["kv"] = new_kv_store(shape, T)
+    pos = np.arange(start, T)
+    hid = forward_rows(shape, weights, tokens, pos, state["kv"], bf16_operands)
+    M = T - n_prompt
+    ids = np.full(M, -1, np.int32)
+    p1 = np.full(M, np.nan)
+    p2 = np.full(M, np.nan)
+    gen = pos >= n_prompt
+    i, c1, c2 = confidence(logits(weights, hid[gen]))
+    ids[pos[gen] - n_prompt], p1[pos[gen] - n_prompt], p2[pos[gen] - n_prompt] = i, c1, c2
+    return ids, p1, p2
+
+
 def logits(weights: dict, hidden: np.ndarray) -> np.ndarray:
     """LM-head logits z = hidden @ W_lm^T, [R, V]."""
     return np.asarray(hidden, np.float64) @ _f64(weights["lm_head"]).T
