@@ -270,7 +270,8 @@ typedef enum {
   DCL_K_GEMM_LMHEAD = 7, /* LM head + softmax/top-2 partials */
   DCL_K_COMBINE = 8,     /* merge of the LM-head partials */
   DCL_K_DCV = 9,         /* commit / draft / advance */
-  DCL_K_VTRANSPOSE = 10  /* v written transposed for the attention kernel */
+  DCL_K_VTRANSPOSE = 10, /* v written transposed for the attention kernel */
+  DCL_K_ROWPLAN = 11     /* the rows the step computes (full recompute or cache suffix) */
 } dcl_kernel_kind;
 
 /* enable = 1 re-captures the step graph with a pair of timing events (CUDA event record

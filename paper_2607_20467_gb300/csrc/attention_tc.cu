@@ -71,8 +71,9 @@ __global__ void __launch_bounds__(256) v_transpose_kernel(const __nv_bfloat16* _
 
 template <int HD>
 __global__ void __launch_bounds__(AT_THREADS, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tv,
-                   const __grid_constant__ CUtensorMap to, int T, int H, int G, int* err) {
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
+                   const __grid_constant__ CUtensorMap tv, const __grid_constant__ CUtensorMap to, int T, int H,
+                   int G, int kcol0, const int* __restrict__ seq_off, const int* __restrict__ seq_len, int* err) {
   using C = AttnCfg<HD>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -119,6 +120,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tq);
+    prefetch_tmap(&tk);
     prefetch_tmap(&tv);
     prefetch_tmap(&to);
   }
@@ -129,8 +131,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   const uint32_t tmem = *holder_ptr;
   pdl_wait();  // the previous kernel of the step has completed
   pdl_launch_dependents();
+  // the query rows of sequence b are rows [off, off + len) of q and of the output; a tile
+  // past them has nothing to do
+  const int q_off = seq_off ? seq_off[b] : b * T;
+  const int q_len = seq_len ? seq_len[b] : T;
+  const bool active = qt * 128 < q_len;
 
-  if (warp == 0) {
+  if (!active) {
+    // an empty query tile
+  } else if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------ TMA producer
       bool ok = true;
@@ -138,7 +147,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       uint32_t phase = 0;
       long issued = 0;
       mbar_arrive_expect_tx(q_full, C::Q_BYTES);
-      for (int bx = 0; bx < C::KB; ++bx) tma_load_3d(sQ + bx * AT_BOX, &tq, h * HD + bx * 64, qt * 128, b, q_full);
+      for (int bx = 0; bx < C::KB; ++bx) tma_load_2d(sQ + bx * AT_BOX, &tq, h * HD + bx * 64, q_off + qt * 128, q_full);
       // consumption order: K_0 .. K_{nb-1} (pass 1); K_0, K_1, then per j: K_{j+2}, V_j
       // (pass 2; K only while j + 2 < nb)
       const int n_loads = 3 * nb;
@@ -168,7 +177,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         mbar_arrive_expect_tx(bar, C::STAGE_BYTES);
         if (!is_v) {
           for (int bx = 0; bx < C::KB; ++bx)
-            tma_load_3d(dst + bx * AT_BOX, &tq, (H + g) * HD + bx * 64, j * 128, b, bar);
+            tma_load_3d(dst + bx * AT_BOX, &tk, kcol0 + g * HD + bx * 64, j * 128, b, bar);
         } else {
           for (int bx = 0; bx < 2; ++bx) tma_load_3d(dst + bx * C::VBOX, &tv, j * 128 + bx * 64, 0, b * G + g, bar);
         }
@@ -376,7 +385,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         }
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0 && row0 < T) tma_store_3d(&to, bx, h * HD + c, row0, b);
+        if (lane == 0 && row0 < q_len) {
+          if (seq_off)
+            tma_store_2d(&to, bx, h * HD + c, q_off + row0);
+          else
+            tma_store_3d(&to, bx, h * HD + c, row0, b);
+        }
       }
       if (lane == 0) {
         bulk_commit();
@@ -408,27 +422,40 @@ cudaError_t launch_attn(const AttnPlan& p, int* err, cudaStream_t stream) {
     attr_set = true;
   }
   dim3 grid((p.T + 127) / 128, p.H, p.batch);
-  return launch_pdl(kern, grid, AT_THREADS, AttnCfg<HD>::SMEM, stream, p.tq, p.tv, p.to, p.T, p.H, p.G, err);
+  return launch_pdl(kern, grid, AT_THREADS, AttnCfg<HD>::SMEM, stream, p.tq, p.tk, p.tv, p.to, p.T, p.H, p.G, p.kcol0,
+                    p.seq_off, p.seq_len, err);
 }
 
 }  // namespace
 
 int attn_vt_pitch(int T) { return (T + 7) & ~7; }
 
-cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16* vt, __nv_bfloat16* out, int batch,
-                           int T, int H, int G, int hd) {
-  if (batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128)) return cudaErrorInvalidValue;
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __nv_bfloat16* vt,
+                           __nv_bfloat16* out, int batch, int T, int H, int G, int hd, int rows_max,
+                           const int* seq_off, const int* seq_len) {
+  if (batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128) || rows_max <= 0)
+    return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(qkv) & 15) || (reinterpret_cast<uintptr_t>(vt) & 15) ||
-      (reinterpret_cast<uintptr_t>(out) & 15))
+      (reinterpret_cast<uintptr_t>(out) & 15) || (kbuf && (reinterpret_cast<uintptr_t>(kbuf) & 15)))
     return cudaErrorInvalidValue;
   const uint64_t cols = (uint64_t)(H + 2 * G) * hd, ocols = (uint64_t)H * hd, Tp = attn_vt_pitch(T);
-  {  // q | k | v rows as [batch][T][cols]: rows past T of a sequence read as zero
-    const uint64_t dims[3] = {cols, (uint64_t)T, (uint64_t)batch};
-    const uint64_t strides[2] = {cols * 2, (uint64_t)T * cols * 2};
-    const uint32_t box[3] = {64, 128, 1};
-    if (!encode_tmap(&p->tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(qkv), dims, strides, box,
+  {  // q rows of the step: [rows_max][cols]
+    const uint64_t dims[2] = {cols, (uint64_t)rows_max};
+    const uint64_t strides[1] = {cols * 2};
+    const uint32_t box[2] = {64, 128};
+    if (!encode_tmap(&p->tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(qkv), dims, strides, box,
                      CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
+  }
+  {  // keys of every position as [batch][T][kcols]: the key store, or the k columns of q|k|v
+    const uint64_t kcols = kbuf ? (uint64_t)G * hd : cols;
+    const uint64_t dims[3] = {kcols, (uint64_t)T, (uint64_t)batch};
+    const uint64_t strides[2] = {kcols * 2, (uint64_t)T * kcols * 2};
+    const uint32_t box[3] = {64, 128, 1};
+    if (!encode_tmap(&p->tk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(kbuf ? kbuf : qkv), dims,
+                     strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+    p->kcol0 = kbuf ? 0 : H * hd;
   }
   {  // v^T as [batch*G][hd][T] (row pitch Tp)
     const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
@@ -437,7 +464,13 @@ cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16*
     if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
   }
-  {  // output as [batch][T][H*hd]: stores of rows past T are clipped
+  if (seq_off) {  // output rows of the step: [rows_max][H*hd] (32-row bands of one sequence)
+    const uint64_t dims[2] = {ocols, (uint64_t)rows_max};
+    const uint64_t strides[1] = {ocols * 2};
+    const uint32_t box[2] = {64, 32};
+    if (!encode_tmap(&p->to, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, out, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return cudaErrorInvalidValue;
+  } else {  // [batch][T][H*hd]: stores of rows past T are clipped
     const uint64_t dims[3] = {ocols, (uint64_t)T, (uint64_t)batch};
     const uint64_t strides[2] = {ocols * 2, (uint64_t)T * ocols * 2};
     const uint32_t box[3] = {64, 32, 1};
@@ -446,6 +479,8 @@ cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16*
   }
   p->qkv = qkv;
   p->vt = vt;
+  p->seq_off = seq_off;
+  p->seq_len = seq_len;
   p->batch = batch;
   p->T = T;
   p->H = H;

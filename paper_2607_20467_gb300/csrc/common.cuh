@@ -82,6 +82,11 @@ struct EpiParams {
   int seq_T = 1;                    // rows per sequence (position = row % seq_T)
   int vocab = 0;
   int vt_heads = 0;                 // QKV: > 0 writes v transposed (G kv heads) through tv
+  int k_store = 0;                  // QKV: 1 writes k (after RoPE) through tk, not to out
+  int k_col0 = 0;                   // QKV: first k column (H * head_dim)
+  const int* m_dev = nullptr;       // device row count (<= M) of the launch, or NULL
+  const int* row_pos = nullptr;     // device position of each row (NULL: row % seq_T)
+  const int* row_seq = nullptr;     // device sequence of each row (NULL: row / seq_T)
 };
 
 struct GemmPlan {
@@ -89,6 +94,7 @@ struct GemmPlan {
   CUtensorMap tc;        // pair tiles: the output (bf16 / fp32 boxes of 32 rows x 128 bytes)
   CUtensorMap tw;        // pair tiles with partials: the fp32 workspace [rows][256]
   CUtensorMap tv;        // QKV with ep.vt_heads > 0: v^T boxes [64 channels][32 tokens]
+  CUtensorMap tk;        // QKV with ep.k_store: k boxes [32 tokens][64 channels] of [B][T][G*hd]
   int M = 0, N = 0, K = 0;
   int bn = 256;          // output columns per tile
   int cg = 1;            // 1: one CTA per 128 x bn tile; 2: a CTA pair per 256 x 256 tile
@@ -120,9 +126,11 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
 // (>= ws_needed floats, 16-byte aligned) a plan needs; they may be shared by plans that
 // run one after another on one stream.
 cudaError_t gemm_bind_scratch(GemmPlan* plan, int* flags, float* ws);
-// Make a CTA-pair QKV plan write v transposed into vt (bf16 [batch*G][hd][Tp]) instead of
-// the v columns of its output; false (plan unchanged) when the shape does not allow it.
-bool gemm_fuse_vt(GemmPlan* plan, void* vt, int batch, int T, int G, int hd, int Tp);
+// Make a CTA-pair QKV plan write k (after RoPE) into kbuf (bf16 [batch][T][G*hd]) and v
+// transposed into vt (bf16 [batch*G][hd][Tp]) instead of the k and v columns of its
+// output, the positions / sequences of its rows given by ep.row_pos / ep.row_seq; false
+// (plan unchanged) when the shape does not allow it (T a multiple of 32 is needed).
+bool gemm_fuse_kv(GemmPlan* plan, void* kbuf, void* vt, int batch, int T, int H, int G, int hd, int Tp);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
 // cuTensorMapEncodeTiled through the runtime's driver entry point: dims / box in elements
@@ -132,33 +140,56 @@ bool encode_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, void* ptr, c
                  const uint64_t* strides, const uint32_t* box, CUtensorMapSwizzle swizzle);
 
 // ---------------------------------------------------------------- attention (attention_tc.cu)
-// softmax(q k^T / sqrt(hd)) v per (sequence, head) over all T positions (non-causal), on
-// the tcgen05 tensor cores.  qkv bf16 [batch*T][(H+2G)*hd] (q | k | v column blocks),
-// out bf16 [batch*T][H*hd]; vt is scratch for v transposed, bf16 [batch*G*hd][attn_vt_pitch(T)].
+// softmax(q k^T / sqrt(hd)) v per (sequence, head): the query rows of sequence b are rows
+// [seq_off[b], seq_off[b] + seq_len[b]) of qkv (q columns) and of out (NULL tables: b*T and
+// T; with tables every seq_len and seq_off is a multiple of 32), its keys and values are
+// all T positions: keys from kbuf [batch][T][G*hd] (NULL: the
+// k columns of qkv, rows b*T + t), values from vt [batch*G][hd][attn_vt_pitch(T)]
+// (v transposed: the attention_transpose_launch output, or what the QKV epilogue wrote).
 struct AttnPlan {
-  CUtensorMap tq, tv, to;
+  CUtensorMap tq, tk, tv, to;
   const __nv_bfloat16* qkv = nullptr;
   __nv_bfloat16* vt = nullptr;
-  int batch = 0, T = 0, H = 0, G = 0, hd = 0;
+  const int* seq_off = nullptr;
+  const int* seq_len = nullptr;
+  int batch = 0, T = 0, H = 0, G = 0, hd = 0, kcol0 = 0;
 };
 int attn_vt_pitch(int T);
-cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, __nv_bfloat16* vt, __nv_bfloat16* out, int batch,
-                           int T, int H, int G, int hd);
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __nv_bfloat16* vt,
+                           __nv_bfloat16* out, int batch, int T, int H, int G, int hd, int rows_max,
+                           const int* seq_off, const int* seq_len);
 cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream);  // both kernels
 cudaError_t attention_transpose_launch(const AttnPlan& p, cudaStream_t stream);  // v -> vt
 cudaError_t attention_core_launch(const AttnPlan& p, int* err, cudaStream_t stream);  // the attention
 
 // ---------------------------------------------------------------- other kernels (kernels.cu)
+// The rows a step computes, in order: sequence b contributes positions [start_b, T) at
+// rows [seq_off[b], seq_off[b] + seq_len[b]); start_b is 0 under full recompute and on a
+// cache refresh, the block-aligned prefix end otherwise, T for a finished sequence.  The
+// LM rows are the computed rows at generation positions.  Written on the device at the
+// start of every step, read by the step's kernels (the step graph is shape-static).
+struct RowPlan {
+  int* counts = nullptr;    // [2]: computed rows R, LM rows R_lm
+  int* row_seq = nullptr;   // [B*T] sequence of row r
+  int* row_pos = nullptr;   // [B*T] position of row r
+  int* seq_off = nullptr;   // [B]
+  int* seq_len = nullptr;   // [B]
+  int* lm_src = nullptr;    // [B*M] computed row of LM row j
+  int* lm_slot = nullptr;   // [B*M] b*M + position - N of LM row j
+  int* pe_cache = nullptr;  // [B] prefix end the stored keys / values belong to (-1: none)
+};
+// update = 0 plans the rows without recording the prefix end (a forward that commits
+// nothing, e.g. a debug pass, leaves the next step's refresh decision unchanged).
+cudaError_t row_plan_launch(const RowPlan& rp, const int32_t* p, int batch, int N, int T, int block_len,
+                            int cached, int update, cudaStream_t stream);
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
                                 int mask_id, int vocab, const __nv_bfloat16* embed, int d,
-                                float* h, int* err, cudaStream_t stream);
-// rows_per_seq / seq_stride / row_offset map output row r to input row
-// (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq.
+                                float* h, int* err, const RowPlan& rp, cudaStream_t stream);
+// y row r = normalised x row src[r] (src NULL: r), for r < min(rows, *rows_dev).
 cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows,
-                           int d, float eps, int rows_per_seq, int seq_stride, int row_offset,
-                           cudaStream_t stream);
+                           int d, float eps, const int* rows_dev, const int* src, cudaStream_t stream);
 cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
-                                  float* p2, cudaStream_t stream);
+                                  float* p2, const int* rows_dev, const int* slot, cudaStream_t stream);
 struct DcvParams {
   float tau_commit, tau_draft;
   int window, min_commit, contiguous_drafts;

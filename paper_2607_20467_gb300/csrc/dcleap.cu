@@ -51,7 +51,12 @@ struct dcl_ctx {
   // activations, sized for max_batch * max_seq rows
   float* h = nullptr;
   __nv_bfloat16 *xn = nullptr, *qkv = nullptr, *attn = nullptr, *act = nullptr, *xg = nullptr;
-  __nv_bfloat16* vt = nullptr;  // v transposed for the attention kernel
+  __nv_bfloat16* vt = nullptr;    // v transposed for the attention kernel (full recompute)
+  __nv_bfloat16* kbuf = nullptr;  // keys after RoPE [B][T][G*hd] (full recompute)
+  __nv_bfloat16* kvstore = nullptr;  // approximate cache: per layer keys [B][T][G*hd], v^T
+  size_t kvstore_bytes = 0;
+  int* rp_buf = nullptr;          // the row plan's tables
+  RowPlan rp;
   float4* part = nullptr;
   int32_t* top1 = nullptr;
   float *p1 = nullptr, *p2 = nullptr;
@@ -76,8 +81,8 @@ struct dcl_ctx {
   int B = 0, N = 0, M = 0, T = 0, window = 0;
   dcl_decode_config dcfg{};
   std::vector<GemmPlan> plans;  // 4 per layer + LM head
-  AttnPlan attn_plan;
-  bool vt_fused = false;  // the QKV GEMMs write v transposed (no transpose launch)
+  std::vector<AttnPlan> attn_plans;  // one per layer
+  bool kv_fused = false;  // the QKV GEMMs write k and v^T (no transpose launch)
   cudaGraphExec_t gexec = nullptr;
   bool profiling = false;
   std::vector<Launch> launches;
@@ -206,9 +211,13 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
   const int d = m.d_model;
   Enq q{c, prof};
   if (prof) c->launch_i = 0;
+  q.begin(DCL_K_ROWPLAN);
+  q.end(row_plan_launch(c->rp, c->p, c->B, c->N, c->T, c->dcfg.block_len, c->dcfg.kv_cache, with_dcv ? 1 : 0,
+                        c->stream),
+        "row_plan");
   q.begin(DCL_K_EMBED);
   q.end(embed_remask_launch(c->x, c->p, c->B, c->T, c->window, m.mask_id, m.vocab, c->embed, d, c->h,
-                            c->derr, c->stream),
+                            c->derr, c->rp, c->stream),
         "embed");
   if (snapshots && q.err == cudaSuccess)
     q.err = cudaMemcpyAsync(c->snap, c->h, sizeof(float) * R * d, cudaMemcpyDeviceToDevice, c->stream);
@@ -216,19 +225,19 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
     const Layer& L = c->layers[l];
     const GemmPlan* P = &c->plans[4 * l];
     q.begin(DCL_K_RMSNORM);
-    q.end(rmsnorm_launch(c->h, L.attn_norm, c->xn, R, d, m.rms_eps, R, 0, 0, c->stream), "rmsnorm");
+    q.end(rmsnorm_launch(c->h, L.attn_norm, c->xn, R, d, m.rms_eps, c->rp.counts, nullptr, c->stream), "rmsnorm");
     q.begin(DCL_K_GEMM_QKV);
     q.end(gemm_launch(P[0], c->derr, c->stream), "gemm_qkv");
-    if (!c->vt_fused) {
+    if (!c->kv_fused) {
       q.begin(DCL_K_VTRANSPOSE);
-      q.end(attention_transpose_launch(c->attn_plan, c->stream), "v_transpose");
+      q.end(attention_transpose_launch(c->attn_plans[l], c->stream), "v_transpose");
     }
     q.begin(DCL_K_ATTENTION);
-    q.end(attention_core_launch(c->attn_plan, c->derr, c->stream), "attention");
+    q.end(attention_core_launch(c->attn_plans[l], c->derr, c->stream), "attention");
     q.begin(DCL_K_GEMM_O);
     q.end(gemm_launch(P[1], c->derr, c->stream), "gemm_o");
     q.begin(DCL_K_RMSNORM);
-    q.end(rmsnorm_launch(c->h, L.mlp_norm, c->xn, R, d, m.rms_eps, R, 0, 0, c->stream), "rmsnorm");
+    q.end(rmsnorm_launch(c->h, L.mlp_norm, c->xn, R, d, m.rms_eps, c->rp.counts, nullptr, c->stream), "rmsnorm");
     q.begin(DCL_K_GEMM_GATEUP);
     q.end(gemm_launch(P[2], c->derr, c->stream), "gemm_gateup");
     q.begin(DCL_K_GEMM_DOWN);
@@ -237,15 +246,16 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
       q.err = cudaMemcpyAsync(c->snap + (size_t)(l + 1) * R * d, c->h, sizeof(float) * R * d,
                               cudaMemcpyDeviceToDevice, c->stream);
   }
-  // final norm on the generation rows only: row b*M + i <- row b*T + N + i
+  // final norm on the computed generation rows only (LM row j <- computed row lm_src[j])
   q.begin(DCL_K_RMSNORM);
-  q.end(rmsnorm_launch(c->h, c->final_norm, c->xg, c->B * c->M, d, m.rms_eps, c->M, c->T, c->N, c->stream),
+  q.end(rmsnorm_launch(c->h, c->final_norm, c->xg, c->B * c->M, d, m.rms_eps, c->rp.counts + 1, c->rp.lm_src,
+                       c->stream),
         "final_rmsnorm");
   q.begin(DCL_K_GEMM_LMHEAD);
   q.end(gemm_launch(c->plans[4 * m.n_layers], c->derr, c->stream), "gemm_lmhead");
   q.begin(DCL_K_COMBINE);
   q.end(lmhead_combine_launch(c->part, c->B * c->M, gemm_lmhead_blocks(m.vocab), c->top1, c->p1, c->p2,
-                              c->stream),
+                              c->rp.counts + 1, c->rp.lm_slot, c->stream),
         "combine");
   if (with_dcv) {
     DcvParams prm{c->dcfg.tau_commit, c->dcfg.tau_draft, c->window, c->dcfg.min_commit,
@@ -304,12 +314,32 @@ int tile_override(const char* name) {
 
 dcl_status build_plans(dcl_ctx* c) {
   const dcl_model_config& m = c->cfg;
-  const int R = c->B * c->T, d = m.d_model, hd = m.head_dim;
-  const int nqkv = (m.n_heads + 2 * m.n_kv_heads) * hd;
+  const int R = c->B * c->T, d = m.d_model, hd = m.head_dim, H = m.n_heads, G = m.n_kv_heads;
+  const int nqkv = (H + 2 * G) * hd;
+  const bool cached = c->dcfg.kv_cache != 0;
   c->plans.assign(4 * m.n_layers + 1, GemmPlan{});
   const char* why = nullptr;
-  const int t_qkv = tile_override("qkv"), t_o = tile_override("o"), t_gu = tile_override("gateup"),
-            t_down = tile_override("down"), t_lm = tile_override("lmhead");
+  // the step's GEMMs run CTA-pair tiles (their epilogues know the step's row plan); an
+  // override may still ask for another tile
+  auto pick = [](int t) { return t ? t : kTilePair; };
+  const int t_qkv = pick(tile_override("qkv")), t_o = pick(tile_override("o")), t_gu = pick(tile_override("gateup")),
+            t_down = pick(tile_override("down")), t_lm = pick(tile_override("lmhead"));
+  // keys / values: one set shared by the layers (full recompute), or a set per layer kept
+  // between steps (approximate cache)
+  const int Tp = attn_vt_pitch(c->T);
+  const size_t k_elems = (size_t)c->B * c->T * G * hd, v_elems = (size_t)c->B * G * hd * Tp;
+  if (cached) {
+    const size_t need = 2 * (k_elems + v_elems) * m.n_layers;
+    if (need > c->kvstore_bytes) {
+      CUDA_TRY(c, cudaStreamSynchronize(c->stream));
+      dev_free_one(c, c->kvstore);
+      c->kvstore = static_cast<__nv_bfloat16*>(dev_alloc(c, need));
+      c->kvstore_bytes = c->kvstore ? need : 0;
+      if (!c->kvstore) return fail(c, DCL_ERR_OOM, "key / value store allocation (%.2f GB) failed", need / 1e9);
+    }
+  }
+  auto kbuf_of = [&](int l) { return cached ? c->kvstore + (size_t)l * (k_elems + v_elems) : c->kbuf; };
+  auto vbuf_of = [&](int l) { return cached ? c->kvstore + (size_t)l * (k_elems + v_elems) + k_elems : c->vt; };
   for (int l = 0; l < m.n_layers; ++l) {
     const Layer& L = c->layers[l];
     EpiParams e0;
@@ -317,39 +347,58 @@ dcl_status build_plans(dcl_ctx* c) {
     e0.ldo = nqkv;
     e0.rope_cos = c->rope_cos;
     e0.rope_sin = c->rope_sin;
-    e0.rope_cols = (m.n_heads + m.n_kv_heads) * hd;
+    e0.rope_cols = (H + G) * hd;
     e0.head_dim = hd;
     e0.seq_T = c->T;
+    e0.m_dev = c->rp.counts;
+    e0.row_pos = c->rp.row_pos;
+    e0.row_seq = c->rp.row_seq;
     if (gemm_plan(&c->plans[4 * l], c->xn, R, d, L.wqkv, nqkv, EPI_QKV_ROPE, e0, c->num_sms, t_qkv, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "QKV plan: %s", why ? why : "?");
     EpiParams e1;
     e1.out = c->h;
     e1.ldo = d;
-    if (gemm_plan(&c->plans[4 * l + 1], c->attn, R, m.n_heads * hd, L.wo, d, EPI_RESID_F32, e1,
-                  c->num_sms, t_o, &why))
+    e1.m_dev = c->rp.counts;
+    if (gemm_plan(&c->plans[4 * l + 1], c->attn, R, H * hd, L.wo, d, EPI_RESID_F32, e1, c->num_sms, t_o, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "O plan: %s", why ? why : "?");
     EpiParams e2;
     e2.out = c->act;
     e2.ldo = m.ffn_dim;
-    if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms,
-                  t_gu, &why))
+    e2.m_dev = c->rp.counts;
+    if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms, t_gu, &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "gate/up plan: %s", why ? why : "?");
-    if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms,
-                  t_down, &why))
+    if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms, t_down,
+                  &why))
       return fail(c, DCL_ERR_UNSUPPORTED, "down plan: %s", why ? why : "?");
+    for (int i = 0; i < 4; ++i)
+      if (c->plans[4 * l + i].streamk)
+        return fail(c, DCL_ERR_UNSUPPORTED, "stream-K needs a fixed row count; the step's GEMMs cannot use it");
   }
-  if (attention_plan(&c->attn_plan, c->qkv, c->vt, c->attn, c->B, c->T, m.n_heads, m.n_kv_heads, hd) != cudaSuccess)
-    return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
-  c->vt_fused = true;
-  for (int l = 0; l < m.n_layers && c->vt_fused; ++l)
-    c->vt_fused = gemm_fuse_vt(&c->plans[4 * l], c->vt, c->B, c->T, m.n_kv_heads, hd, attn_vt_pitch(c->T));
-  if (!c->vt_fused)
-    for (int l = 0; l < m.n_layers; ++l) c->plans[4 * l].ep.vt_heads = 0;
+  c->kv_fused = true;
+  for (int l = 0; l < m.n_layers && c->kv_fused; ++l)
+    c->kv_fused = gemm_fuse_kv(&c->plans[4 * l], kbuf_of(l), vbuf_of(l), c->B, c->T, H, G, hd, Tp);
+  if (!c->kv_fused) {
+    if (cached) return fail(c, DCL_ERR_UNSUPPORTED, "the key / value cache needs N + M a multiple of 32");
+    for (int l = 0; l < m.n_layers; ++l) {
+      c->plans[4 * l].ep.vt_heads = 0;
+      c->plans[4 * l].ep.k_store = 0;
+    }
+  }
+  c->attn_plans.assign(m.n_layers, AttnPlan{});
+  for (int l = 0; l < m.n_layers; ++l)
+    // (without the fused key store the rows are the identity layout b*T + t: no tables)
+    if (attention_plan(&c->attn_plans[l], c->qkv, c->kv_fused ? kbuf_of(l) : nullptr, vbuf_of(l), c->attn, c->B, c->T,
+                       H, G, hd, R, c->kv_fused ? c->rp.seq_off : nullptr, c->kv_fused ? c->rp.seq_len : nullptr) !=
+        cudaSuccess)
+      return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
   EpiParams el;
   el.out = c->part;
+  el.m_dev = c->rp.counts + 1;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,
                 c->num_sms, t_lm, &why))
     return fail(c, DCL_ERR_UNSUPPORTED, "LM-head plan: %s", why ? why : "?");
+  if (c->plans[4 * m.n_layers].streamk)
+    return fail(c, DCL_ERR_UNSUPPORTED, "stream-K needs a fixed row count; the step's GEMMs cannot use it");
   // split-K counters and partials, shared by the step's GEMMs (they run one after another)
   size_t need_f = 0, need_w = 0;
   for (const GemmPlan& p : c->plans) {
@@ -566,6 +615,8 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->qkv = (__nv_bfloat16*)dev_alloc(c, 2 * R * (H + 2 * G) * hd);
     c->attn = (__nv_bfloat16*)dev_alloc(c, 2 * R * H * hd);
     c->vt = (__nv_bfloat16*)dev_alloc(c, 2 * (size_t)max_batch * G * hd * attn_vt_pitch(max_seq));
+    c->kbuf = (__nv_bfloat16*)dev_alloc(c, 2 * R * G * hd);
+    c->rp_buf = (int*)dev_alloc(c, sizeof(int) * (2 + 4 * R + 3 * (size_t)max_batch));
     c->act = (__nv_bfloat16*)dev_alloc(c, 2 * R * F);
     c->xg = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->part = (float4*)dev_alloc(c, sizeof(float4) * R * nblk);
@@ -581,7 +632,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->p_init = (int32_t*)dev_alloc(c, 4 * max_batch);
     c->rope_cos = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
     c->rope_sin = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
-    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->act || !c->xg || !c->part || !c->top1 ||
+    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->kbuf || !c->rp_buf || !c->act || !c->xg || !c->part || !c->top1 ||
         !c->p1 || !c->p2 || !c->x || !c->p || !c->k || !c->steps || !c->done_count || !c->x_init || !c->p_init || !c->rope_cos ||
         !c->rope_sin) {
       dev_free_all(c);
@@ -598,6 +649,15 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     for (int l = 0; l < m.n_layers; ++l)
       c->layers[l] = {W + lo[6 * l], W + lo[6 * l + 1], W + lo[6 * l + 2], W + lo[6 * l + 3], W + lo[6 * l + 4],
                       W + lo[6 * l + 5]};
+    int* q = c->rp_buf;
+    c->rp.counts = q;
+    c->rp.row_seq = q + 2;
+    c->rp.row_pos = c->rp.row_seq + R;
+    c->rp.lm_src = c->rp.row_pos + R;
+    c->rp.lm_slot = c->rp.lm_src + R;
+    c->rp.seq_off = c->rp.lm_slot + R;
+    c->rp.seq_len = c->rp.seq_off + max_batch;
+    c->rp.pe_cache = c->rp.seq_len + max_batch;
     if (rope_table_build(c->rope_cos, c->rope_sin, max_seq, (int)hd, m.rope_theta, c->stream) != cudaSuccess) {
       dev_free_all(c);
       release_stream(c);
@@ -683,13 +743,16 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   if (batch <= 0 || batch > c->max_batch) return fail(c, DCL_ERR_INVALID_ARG, "batch %d outside [1, %d]", batch, c->max_batch);
   if (n_prompt < 0 || cfg->gen_len <= 0 || n_prompt + cfg->gen_len > c->max_seq)
     return fail(c, DCL_ERR_INVALID_ARG, "N + M = %d + %d exceeds max_seq %d", n_prompt, cfg->gen_len, c->max_seq);
-  if (cfg->kv_cache != 0) return fail(c, DCL_ERR_UNSUPPORTED, "only full recompute (kv_cache = 0) is built");
+  if (cfg->kv_cache != 0 && cfg->kv_cache != 1) return fail(c, DCL_ERR_INVALID_ARG, "kv_cache must be 0 or 1");
+  if (cfg->kv_cache && (cfg->block_len <= 0 || cfg->block_len % 32 || n_prompt % 32 || cfg->gen_len % 32))
+    return fail(c, DCL_ERR_UNSUPPORTED, "the key / value cache needs N, M and the block length multiples of 32");
   if (cfg->max_window < 0 || cfg->min_commit < 0 || !(cfg->tau_commit == cfg->tau_commit) ||
       !(cfg->tau_draft == cfg->tau_draft))
     return fail(c, DCL_ERR_INVALID_ARG, "bad decode config");
   dcl_status s = validate_ids(c, prompt, (size_t)batch * n_prompt);
   if (s != DCL_OK) return s;
-  const bool reshape = !c->prompt_set || batch != c->B || n_prompt != c->N || cfg->gen_len != c->M;
+  const bool reshape = !c->prompt_set || batch != c->B || n_prompt != c->N || cfg->gen_len != c->M ||
+                       cfg->kv_cache != c->dcfg.kv_cache;
   const int window = cfg->max_window > 0 ? cfg->max_window : (cfg->gen_len / 2 > 0 ? cfg->gen_len / 2 : 1);
   const bool redcv = !c->prompt_set || window != c->window || memcmp(cfg, &c->dcfg, sizeof *cfg) != 0;
   c->B = batch;
@@ -707,6 +770,7 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   CUDA_TRY(c, cudaMemcpyAsync(c->k, zero.data(), 4 * batch, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->x_init, c->x, 4 * xh.size(), cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p_init, c->p, 4 * batch, cudaMemcpyDeviceToDevice, c->stream));
+  CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)batch, c->stream));  // no stored keys / values
   s = reset_done_count(c, ph.data());
   if (s != DCL_OK) return s;
   if (reshape) {
@@ -794,6 +858,7 @@ dcl_status dcl_restart(dcl_ctx* c) {
   CUDA_TRY(c, cudaMemsetAsync(c->steps, 0, 4 * B, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->k, 0, 4 * B, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->done_count, 0, 4, c->stream));
+  CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * B, c->stream));
   return DCL_OK;
 }
 
@@ -816,6 +881,7 @@ dcl_status dcl_set_state(dcl_ctx* c, const int32_t* x, const int32_t* p) {
     if (p[b] < c->N || p[b] > c->T) return fail(c, DCL_ERR_INVALID_ARG, "p[%d] = %d outside [N, N+M]", b, p[b]);
   CUDA_TRY(c, cudaMemcpyAsync(c->x, x, 4 * (size_t)c->B * c->T, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p, p, 4 * (size_t)c->B, cudaMemcpyHostToDevice, c->stream));
+  CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)c->B, c->stream));  // the next step refreshes
   return reset_done_count(c, p);
 }
 
@@ -891,7 +957,7 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* c, const float* x_dev, const void* gain_dev, 
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!x_dev || !gain_dev || !y_dev || rows <= 0 || d <= 0 || d % 4) return fail(c, DCL_ERR_INVALID_ARG, "bad rmsnorm args");
   CUDA_TRY(c, rmsnorm_launch(x_dev, static_cast<const __nv_bfloat16*>(gain_dev), static_cast<__nv_bfloat16*>(y_dev),
-                             rows, d, eps, rows, 0, 0, c->stream));
+                             rows, d, eps, nullptr, nullptr, c->stream));
   return DCL_OK;
 }
 
@@ -924,8 +990,8 @@ dcl_status dcl_op_attention(dcl_ctx* c, const void* qkv_dev, void* out_dev, int3
   __nv_bfloat16* vt = static_cast<__nv_bfloat16*>(dev_alloc(c, 2 * (size_t)batch * G * hd * attn_vt_pitch(T)));
   if (!vt) return fail(c, DCL_ERR_OOM, "attention scratch allocation failed");
   AttnPlan pl;
-  if (attention_plan(&pl, static_cast<const __nv_bfloat16*>(qkv_dev), vt, static_cast<__nv_bfloat16*>(out_dev), batch, T,
-                     H, G, hd) != cudaSuccess) {
+  if (attention_plan(&pl, static_cast<const __nv_bfloat16*>(qkv_dev), nullptr, vt, static_cast<__nv_bfloat16*>(out_dev),
+                     batch, T, H, G, hd, batch * T, nullptr, nullptr) != cudaSuccess) {
     dev_free_one(c, vt);
     return fail(c, DCL_ERR_INVALID_ARG, "attention: operands must be 16-byte aligned");
   }
@@ -968,7 +1034,7 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
     dev_free_one(c, part);
     return fail(c, DCL_ERR_CUDA, "LM-head GEMM: %s", cudaGetErrorString(e));
   }
-  CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, c->stream));
+  CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, nullptr, nullptr, c->stream));
   s = check_device(c);
   dev_free_one(c, part);
   return s;

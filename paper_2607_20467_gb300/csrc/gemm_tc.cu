@@ -577,7 +577,8 @@ __device__ __forceinline__ void store_bf16_box(const Src& s, Stage& o, const CUt
 // half.  All tcgen05.ld run warp-uniformly.
 template <int EPI>
 __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUtensorMap* tmc, const CUtensorMap* tmv,
-                                              int row, int n_blk, int M, int N, const EpiParams& ep) {
+                                              const CUtensorMap* tmk, int row, int n_blk, int M, int N,
+                                              const EpiParams& ep) {
   const int n0 = n_blk * 256;
   if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
@@ -593,9 +594,16 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       o.issue(tmc, b, n0 + c, o.row0, true);
     }
   } else if constexpr (EPI == EPI_QKV_ROPE) {
+    // the band's sequence and first position (32 consecutive positions of one sequence)
+    int bz = 0, t0 = 0;
+    if (o.live) {
+      bz = ep.row_seq ? ep.row_seq[o.row0] : o.row0 / ep.seq_T;
+      t0 = ep.row_pos ? ep.row_pos[o.row0] : o.row0 - bz * ep.seq_T;
+    }
     if (n0 < ep.rope_cols) {
       const int hd = ep.head_dim, half = hd >> 1;
-      const int pos = row < M ? row % ep.seq_T : 0;
+      const int pos = row < M ? (ep.row_pos ? ep.row_pos[row] : row % ep.seq_T) : 0;
+      const bool to_k = ep.k_store && n0 >= ep.k_col0;  // k columns go to the key store
       const float* cs = ep.rope_cos + (size_t)pos * half;
       const float* sn = ep.rope_sin + (size_t)pos * half;
 #pragma unroll 1
@@ -631,14 +639,17 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
             stage_bf16(b0, o.lane, 1, hi);
           }
         }
-        o.issue(tmc, b0, n0 + hb, o.row0, false);
-        if (hd == 128) o.issue(tmc, b1, n0 + hb + 64, o.row0, false);
+        if (to_k) {
+          o.issue3(tmk, b0, n0 + hb - ep.k_col0, t0, bz);
+          if (hd == 128) o.issue3(tmk, b1, n0 + hb + 64 - ep.k_col0, t0, bz);
+        } else {
+          o.issue(tmc, b0, n0 + hb, o.row0, false);
+          if (hd == 128) o.issue(tmc, b1, n0 + hb + 64, o.row0, false);
+        }
       }
     } else if (ep.vt_heads > 0) {
       // v columns leave transposed, as the attention's K-major operand: boxes of 64
-      // channels x 32 tokens of vt [batch * G][hd][T] (the band's 32 rows are 32
-      // consecutive tokens of one sequence: T is a multiple of 32)
-      const int bz = o.row0 / ep.seq_T, t0 = o.row0 - bz * ep.seq_T;
+      // channels x 32 tokens of vt [batch * G][hd][T]
 #pragma unroll 1
       for (int c = 0; c < 256 && n0 + c < N; c += 64) {
         const int cv = n0 + c - ep.rope_cols, g = cv / ep.head_dim, d0 = cv - g * ep.head_dim;
@@ -902,7 +913,7 @@ template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
                     const __grid_constant__ CUtensorMap tmc, const __grid_constant__ CUtensorMap tmw,
-                    const __grid_constant__ CUtensorMap tmv, int M,
+                    const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmk, int M,
                     int N, int K, EpiParams ep, int splits, int streamk, int ws_slots, int* flags, float* ws,
                     int* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -926,14 +937,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();  // 0: leader (issues the MMAs), 1: peer
   const int cluster = blockIdx.x >> 1;
-  const int num_m = (M + 255) / 256;
-  const int num_n = (N + 255) / 256;
-  Sched sc;
-  sc.tiles = num_m * num_n;
-  sc.ku = (K + BK * KA2 - 1) / (BK * KA2);
-  sc.C = gridDim.x >> 1;
-  sc.splits = splits;
-  sc.streamk = streamk;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
@@ -959,6 +962,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem_base = *holder_ptr;
   pdl_wait();  // the previous kernel of the step has completed
   pdl_launch_dependents();
+  if (ep.m_dev) M = min(M, *ep.m_dev);  // the step's row count (written by an earlier kernel)
+  const int num_m = (M + 255) / 256;
+  const int num_n = (N + 255) / 256;
+  Sched sc;
+  sc.tiles = num_m * num_n;
+  sc.ku = (K + BK * KA2 - 1) / (BK * KA2);
+  sc.C = gridDim.x >> 1;
+  sc.splits = splits;
+  sc.streamk = streamk;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1076,7 +1088,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       s.taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
       s.row = row_local;
       if (it.kind == IT_PLAIN) {
-        epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
+        epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
         int* flag = flags + t * 2 + rank;
@@ -1086,7 +1098,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             report_error(err, DERR_WAIT_TIMEOUT);
           }
           epilogue_bar();
-          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
           o.drain();
           epilogue_bar();
           if (et == 0) {
@@ -1113,7 +1125,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             s.part = ws + ((size_t)t * S1 * 2 + rank) * 128 * 256;
             s.part_stride = (size_t)2 * 128 * 256;
             s.nparts = S1;
-            if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
+            if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
             epilogue_bar();
             if (et == 0) atomicExch(flag, 0);
           }
@@ -1144,7 +1156,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
               s.tsum = tsum;
             }
           }
-          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, row, n_blk, M, N, ep);
+          if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
           epilogue_bar();
           if (et == 0) atomicExch(flag, 0);
         }
@@ -1228,7 +1240,8 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  return launch_pdl(kern, p.grid, NUM_THREADS, SMEM2, stream, p.ta, p.tb, p.tc, p.tw, p.tv, p.M, p.N, p.K, p.ep, p.splits,
+  return launch_pdl(kern, p.grid, NUM_THREADS, SMEM2, stream, p.ta, p.tb, p.tc, p.tw, p.tv, p.tk, p.M, p.N, p.K, p.ep,
+                    p.splits,
                     p.streamk, p.ws_slots, p.flags, p.ws, err);
 }
 
@@ -1363,7 +1376,9 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   memset(&plan->tc, 0, sizeof(plan->tc));
   memset(&plan->tw, 0, sizeof(plan->tw));
   memset(&plan->tv, 0, sizeof(plan->tv));
+  memset(&plan->tk, 0, sizeof(plan->tk));
   plan->ep.vt_heads = 0;
+  plan->ep.k_store = 0;
   if (cg == 2 && epi != EPI_LMHEAD) {
     const bool f32 = (epi == EPI_RESID_F32);
     const int es = f32 ? 4 : 2;
@@ -1412,16 +1427,31 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   return cudaSuccess;
 }
 
-bool gemm_fuse_vt(GemmPlan* p, void* vt, int batch, int T, int G, int hd, int Tp) {
-  if (p->cg != 2 || p->epi != EPI_QKV_ROPE || T % 32 != 0 || p->ep.rope_cols % 256 != 0 ||
-      (reinterpret_cast<uintptr_t>(vt) & 15) || Tp % 8 != 0)
+bool gemm_fuse_kv(GemmPlan* p, void* kbuf, void* vt, int batch, int T, int H, int G, int hd, int Tp) {
+  if (p->cg != 2 || p->epi != EPI_QKV_ROPE || T % 32 != 0 || p->ep.rope_cols % 256 != 0 || (H * hd) % 256 != 0 ||
+      (reinterpret_cast<uintptr_t>(vt) & 15) || (reinterpret_cast<uintptr_t>(kbuf) & 15) || Tp % 8 != 0)
     return false;
-  const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
-  const uint64_t strides[2] = {(uint64_t)Tp * 2, (uint64_t)hd * Tp * 2};
-  const uint32_t box[3] = {32, 64, 1};
-  if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE))
-    return false;
+  CUtensorMap tv, tk;
+  {
+    const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
+    const uint64_t strides[2] = {(uint64_t)Tp * 2, (uint64_t)hd * Tp * 2};
+    const uint32_t box[3] = {32, 64, 1};
+    if (!encode_tmap(&tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE))
+      return false;
+  }
+  {
+    const uint64_t cols = (uint64_t)G * hd;
+    const uint64_t dims[3] = {cols, (uint64_t)T, (uint64_t)batch};
+    const uint64_t strides[2] = {cols * 2, (uint64_t)T * cols * 2};
+    const uint32_t box[3] = {64, 32, 1};
+    if (!encode_tmap(&tk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, kbuf, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+      return false;
+  }
+  p->tv = tv;
+  p->tk = tk;
   p->ep.vt_heads = G;
+  p->ep.k_store = 1;
+  p->ep.k_col0 = H * hd;
   return true;
 }
 

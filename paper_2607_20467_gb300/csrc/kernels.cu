@@ -17,22 +17,74 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 
+// ------------------------------------------------------------------ step row plan
+// One CTA: per sequence the first computed position (0 under full recompute and on a cache
+// refresh, the block-aligned prefix end N + Bk*floor((p-N)/Bk) when the stored keys and
+// values are that block's, T for a finished row), the row offsets, and the row tables.
+__global__ void __launch_bounds__(1024) row_plan_kernel(RowPlan rp, const int32_t* __restrict__ p, int B, int N,
+                                                        int T, int Bk, int cached, int update) {
+  pdl_wait();
+  pdl_launch_dependents();
+  extern __shared__ int lm_off[];  // [B]
+  const int M = T - N;
+  if (threadIdx.x == 0) {
+    int off = 0, lmoff = 0;
+    for (int b = 0; b < B; ++b) {
+      const int pb = p[b];
+      int start;
+      if (pb >= T) {
+        start = T;
+      } else if (!cached) {
+        start = 0;
+      } else {
+        const int pe = N + Bk * ((pb - N) / Bk);
+        start = (rp.pe_cache[b] == pe) ? pe : 0;
+        if (update) rp.pe_cache[b] = pe;
+      }
+      rp.seq_off[b] = off;
+      rp.seq_len[b] = T - start;
+      off += T - start;
+      lm_off[b] = lmoff;
+      lmoff += T - max(start, N);
+    }
+    rp.counts[0] = off;
+    rp.counts[1] = lmoff;
+  }
+  __syncthreads();
+  for (int b = 0; b < B; ++b) {
+    const int len = rp.seq_len[b], off = rp.seq_off[b], start = T - len;
+    for (int i = threadIdx.x; i < len; i += blockDim.x) {
+      rp.row_seq[off + i] = b;
+      rp.row_pos[off + i] = start + i;
+    }
+    const int s0 = max(start, N);
+    for (int i = threadIdx.x; i < T - s0; i += blockDim.x) {
+      const int pos = s0 + i;
+      rp.lm_src[lm_off[b] + i] = off + (pos - start);
+      rp.lm_slot[lm_off[b] + i] = b * M + (pos - N);
+    }
+  }
+}
+
 // ------------------------------------------------------------------ embedding + remask
+// Row r of the step (grid: the most rows a step can have) is position row_pos[r] of
+// sequence row_seq[r]; rows past the step's count return.
 __global__ void embed_remask_kernel(int32_t* __restrict__ x, const int32_t* __restrict__ p, int T,
                                     int window, int mask_id, int vocab,
                                     const __nv_bfloat16* __restrict__ embed, int d,
-                                    float* __restrict__ h, int* err) {
+                                    float* __restrict__ h, int* err, RowPlan rp) {
   pdl_wait();
   pdl_launch_dependents();
   const int row = blockIdx.x;
-  const int b = row / T, t = row % T;
+  if (row >= rp.counts[0]) return;
+  const int b = rp.row_seq[row], t = rp.row_pos[row];
   __shared__ int tok_s;
   if (threadIdx.x == 0) {
     const int pb = p[b];
-    int tok = x[row];
+    int tok = x[(size_t)b * T + t];
     if (t >= pb && t - pb < window) {  // x_{p+i} <- MASK for i in [0, L)
       tok = mask_id;
-      x[row] = mask_id;
+      x[(size_t)b * T + t] = mask_id;
     }
     if (tok < 0 || tok >= vocab) {
       report_error(err, DERR_TOKEN_RANGE);
@@ -55,12 +107,13 @@ template <int THREADS>
 __global__ void __launch_bounds__(THREADS) rmsnorm_kernel(const float* __restrict__ x,
                                                           const __nv_bfloat16* __restrict__ gain,
                                                           __nv_bfloat16* __restrict__ y, int d,
-                                                          float eps, int rows_per_seq,
-                                                          int seq_stride, int row_offset) {
+                                                          float eps, const int* __restrict__ rows_dev,
+                                                          const int* __restrict__ src) {
   pdl_wait();
   pdl_launch_dependents();
   const int r = blockIdx.x;
-  const int in_row = (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq;
+  if (rows_dev && r >= *rows_dev) return;
+  const int in_row = src ? src[r] : r;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
   const int n4 = d / 4;
   float ss = 0.f;
@@ -96,13 +149,14 @@ __global__ void __launch_bounds__(THREADS) rmsnorm_kernel(const float* __restric
 template <int VPT, int ROWS>
 __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
     const float* __restrict__ x, const __nv_bfloat16* __restrict__ gain, __nv_bfloat16* __restrict__ y,
-    int rows, int d, float eps, int rows_per_seq, int seq_stride, int row_offset) {
+    int rows, int d, float eps, const int* __restrict__ rows_dev, const int* __restrict__ src) {
   pdl_wait();
   pdl_launch_dependents();
+  if (rows_dev) rows = min(rows, *rows_dev);
   const int sub = threadIdx.x >> 7, t = threadIdx.x & 127;
   const int r = blockIdx.x * ROWS + sub;
   const bool live = r < rows;
-  const int in_row = (r / rows_per_seq) * seq_stride + row_offset + r % rows_per_seq;
+  const int in_row = live ? (src ? src[r] : r) : 0;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
   const int n4 = d / 4;
   float4 v[VPT];
@@ -179,13 +233,16 @@ __device__ __forceinline__ void write_conf(const Part& a, int32_t* top1, float* 
   p2[r] = a.t2 == -INFINITY ? 0.f : fminf(exp2f((a.t2 - a.m) * kLog2e) * inv, c1);
 }
 
+// LM row `row` (of *rows_dev) is written to slot slot[row] of top1 / p1 / p2.
 __global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows, int nblk,
                                       int32_t* __restrict__ top1, float* __restrict__ p1,
-                                      float* __restrict__ p2) {
+                                      float* __restrict__ p2, const int* __restrict__ rows_dev,
+                                      const int* __restrict__ slot) {
   pdl_wait();
   pdl_launch_dependents();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
+  if (rows_dev) rows = min(rows, *rows_dev);
   if (row >= rows) return;
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
   for (int i = lane; i < nblk; i += 32) {
@@ -194,7 +251,7 @@ __global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows,
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) merge(a, shfl_part(a, o));
-  if (lane == 0) write_conf(a, top1, p1, p2, row);
+  if (lane == 0) write_conf(a, top1, p1, p2, slot ? slot[row] : row);
 }
 
 // ------------------------------------------------------------------ DCV on one sequence
@@ -364,35 +421,42 @@ __global__ void generate_kernel(__nv_bfloat16* __restrict__ dst, uint64_t seed, 
 }  // namespace
 
 // ------------------------------------------------------------------ launchers
+cudaError_t row_plan_launch(const RowPlan& rp, const int32_t* p, int batch, int N, int T, int block_len, int cached,
+                            int update, cudaStream_t stream) {
+  if (batch <= 0 || batch > 4096 || (cached && block_len <= 0)) return cudaErrorInvalidValue;
+  return launch_pdl(row_plan_kernel, 1, 1024, sizeof(int) * batch, stream, rp, p, batch, N, T, block_len, cached,
+                    update);
+}
+
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
                                 int mask_id, int vocab, const __nv_bfloat16* embed, int d, float* h,
-                                int* err, cudaStream_t stream) {
+                                int* err, const RowPlan& rp, cudaStream_t stream) {
   if (d % 8) return cudaErrorInvalidValue;
-  return launch_pdl(embed_remask_kernel, batch * T, 128, 0, stream, x, p, T, window, mask_id, vocab, embed, d, h, err);
+  return launch_pdl(embed_remask_kernel, batch * T, 128, 0, stream, x, p, T, window, mask_id, vocab, embed, d, h, err,
+                    rp);
 }
 
 cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows, int d,
-                           float eps, int rows_per_seq, int seq_stride, int row_offset,
-                           cudaStream_t stream) {
+                           float eps, const int* rows_dev, const int* src, cudaStream_t stream) {
   if (d % 4 || rows <= 0) return cudaErrorInvalidValue;
   const int vpt = (d / 4 + 127) / 128;  // float4 per thread with 128 threads per row
   const int grid2 = (rows + 1) / 2;
   switch (vpt) {
-    case 1: return launch_pdl(rmsnorm_reg_kernel<1, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
-    case 2: return launch_pdl(rmsnorm_reg_kernel<2, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
-    case 4: case 3: return launch_pdl(rmsnorm_reg_kernel<4, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
+    case 1: return launch_pdl(rmsnorm_reg_kernel<1, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_dev, src);
+    case 2: return launch_pdl(rmsnorm_reg_kernel<2, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_dev, src);
+    case 4: case 3: return launch_pdl(rmsnorm_reg_kernel<4, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_dev, src);
     case 5: case 6: case 7: case 8:
-      return launch_pdl(rmsnorm_reg_kernel<8, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_per_seq, seq_stride, row_offset);
+      return launch_pdl(rmsnorm_reg_kernel<8, 2>, grid2, 256, 0, stream, x, gain, y, rows, d, eps, rows_dev, src);
     default:
-      return launch_pdl(rmsnorm_kernel<256>, rows, 256, 0, stream, x, gain, y, d, eps, rows_per_seq, seq_stride, row_offset);
+      return launch_pdl(rmsnorm_kernel<256>, rows, 256, 0, stream, x, gain, y, d, eps, rows_dev, src);
   }
 }
 
 cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
-                                  float* p2, cudaStream_t stream) {
+                                  float* p2, const int* rows_dev, const int* slot, cudaStream_t stream) {
   const int threads = 256;
   const int blocks = (rows * 32 + threads - 1) / threads;
-  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, rows, nblk, top1, p1, p2);
+  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, rows, nblk, top1, p1, p2, rows_dev, slot);
 }
 
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,

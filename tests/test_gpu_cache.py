@@ -1,0 +1,111 @@
+"""The approximate prefix key / value cache (kv_cache = 1) on the GPU against the oracle's
+cached Algorithm 1 (``decode.generate`` with ``model.predict_from``, bf16 operands), on the
+2-layer / d 256 / 4x64 heads / vocab 4096 model (prompt 32, gen 64, block 32).
+
+Under the cache a step's result depends on the keys and values stored at earlier steps,
+so states cannot be loaded one by one (a loaded state forces a refresh): the GPU and the
+oracle each run the whole cached generation, and their states must agree step after
+step up to the first step whose oracle decision had a margin below E2E_TOL (the
+end-to-end tolerance of the uncached tests, derived there); a split without such a near
+tie is a failure.  The fraction of runs that split is printed."""
+import numpy as np
+import pytest
+
+import synthetic as syn
+from oracle import decode, model
+
+pytestmark = pytest.mark.gpu
+
+TINY = syn.SHAPES["tiny"]
+N, M = 32, 64
+T = N + M
+E2E_TOL = 5e-2
+
+
+@pytest.fixture(scope="module")
+def dcl():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2607_20467_gb300 as pkg
+    return pkg
+
+
+@pytest.fixture(scope="module")
+def weights():
+    return syn.model_weights(TINY, 0, lm_head_scale=40.0, norm_gain_std=0.1)
+
+
+def _cached(weights):
+    return lambda tok, start, state: model.predict_from(TINY, weights, tok, start, state, N, bf16_operands=True)
+
+
+def _split_is_near_tie(ref, s, b, p_prev, ocfg):
+    prev = ref["preds"][s - 1][:, b]
+    c = np.zeros(T)
+    c[N:] = np.nan_to_num(prev[1], nan=-1.0)
+    g = np.full(T, np.inf)
+    g[N:] = np.nan_to_num(prev[1] - prev[2], nan=np.inf)
+    return (np.abs(c[p_prev:] - ocfg.tau_commit) <= E2E_TOL).any() or \
+        (np.abs(c[p_prev:] - ocfg.tau_draft) <= E2E_TOL).any() or (g[p_prev:] <= E2E_TOL).any()
+
+
+@pytest.mark.parametrize("seed,B,tau_c,L", [(0, 1, 0.7, 32), (1, 1, 0.5, 16), (2, 3, 0.7, 32), (3, 2, 0.3, 64)])
+def test_cached_generation_matches_oracle(dcl, weights, seed, B, tau_c, L):
+    prompt = syn.prompt_ids(300 + seed, B, N, TINY.mask_id)
+    cfg = dcl.decode_config(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=1)
+    ocfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=1)
+    ref = decode.generate(_cached(weights), prompt, ocfg, TINY.mask_id)
+    assert ref["done"]
+    with dcl.Context(TINY, max_batch=B, max_seq=T) as ctx:
+        ctx.load_weights(weights)
+        ctx.set_prompt(prompt, cfg)
+        states = []
+        for _ in range(2 * M):
+            x, p = ctx.get_state()
+            states.append((x.copy(), p.copy()))
+            if (p >= T).all():
+                break
+            ctx.step()
+    assert (states[-1][1] == T).all()
+    outside = lambda p: (np.arange(T) < p) | (np.arange(T) >= p + ocfg.window())
+    split = [None] * B
+    p_o = np.full(B, N)
+    for s, xin in enumerate(ref["inputs"]):
+        xg, pg = states[min(s, len(states) - 1)]
+        for b in range(B):
+            if split[b] is not None:
+                continue
+            if pg[b] != p_o[b] or not (xg[b] == xin[b])[outside(p_o[b])].all():
+                p_prev = p_o[b] - int(ref["k"][s - 1, b])
+                assert _split_is_near_tie(ref, s, b, p_prev, ocfg), \
+                    f"row {b}: GPU and oracle diverged at step {s - 1} with a clear margin"
+                split[b] = s
+        p_o = p_o + ref["k"][s]
+    for b in range(B):
+        if split[b] is None:
+            assert (states[-1][0][b, N:] == ref["x"][b, N:]).all()
+    refreshes = int((ref["start"] == 0).sum())
+    print(f"seed {seed}: {ref['n_iter']} oracle steps ({refreshes} refresh row-steps); "
+          f"rows split at a near tie: {sum(x is not None for x in split)} of {B}")
+
+
+def test_cache_changes_the_result_only_through_stale_keys(dcl, weights):
+    """The first step of a cached generation is a refresh: it equals the uncached step.
+    A whole cached generation completes, commits contiguously and replays bit for bit."""
+    prompt = syn.prompt_ids(11, 2, N, TINY.mask_id)
+    with dcl.Context(TINY, max_batch=2, max_seq=T) as a, dcl.Context(TINY, max_batch=2, max_seq=T) as b:
+        a.load_weights(weights)
+        b.load_weights(weights)
+        a.set_prompt(prompt, dcl.decode_config(tau_commit=0.7, max_window=32, gen_len=M, kv_cache=1))
+        b.set_prompt(prompt, dcl.decode_config(tau_commit=0.7, max_window=32, gen_len=M, kv_cache=0))
+        ka, kb = a.step(return_k=True), b.step(return_k=True)
+        xa, pa = a.get_state()
+        xb, pb = b.get_state()
+        assert (ka == kb).all() and (xa == xb).all() and (pa == pb).all()
+        out, st, status = a.generate(max_steps=4 * M)
+        assert st.done == 1
+        x, p = a.get_state()
+        assert (p == T).all() and (x[:, N:] != TINY.mask_id).all() and (x[:, :N] == prompt).all()
+        a.restart()
+        out2, st2, _ = a.generate(max_steps=4 * M)
+        assert (out2 == out).all() and st2.steps == st.steps

@@ -272,9 +272,12 @@ def test_error_statuses(dcl, weights):
         assert e.value.status == dcl.DCL_ERR_INVALID_ARG
         with pytest.raises(dcl.DcleapError):
             c.set_prompt(syn.prompt_ids(0, 2, N, TINY.mask_id), cfg)   # batch > max_batch
-        with pytest.raises(dcl.DcleapError) as e:
-            c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=1))
+        with pytest.raises(dcl.DcleapError) as e:  # the cache needs 32-aligned blocks
+            c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=1, block_len=16))
         assert e.value.status == dcl.DCL_ERR_UNSUPPORTED
+        with pytest.raises(dcl.DcleapError) as e:
+            c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=2))
+        assert e.value.status == dcl.DCL_ERR_INVALID_ARG
         c.load_weights(weights)
         c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), cfg)
         x, p = c.get_state()

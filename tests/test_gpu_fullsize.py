@@ -21,7 +21,10 @@ A 32-layer forward of an 8B model in fp64 is out of reach of a test, so:
     which dcl_forward_debug reproduces bit for bit (same kernels, deterministic
     reductions), and every row must end with all positions committed;
   * a second generation of the same prompts through dcl_generate gives the same tokens.
-The rule is restated here in a few lines of numpy; the oracle is not fed GPU values.
+The same holds with the approximate prefix key / value cache on (a step's predictions
+then come from the computed suffix; dcl_forward_debug runs the same suffix without
+recording the refresh).  The rule is restated here in a few lines of numpy; the oracle
+is not fed GPU values.
 """
 import numpy as np
 import pytest
@@ -34,12 +37,17 @@ pytestmark = pytest.mark.gpu
 
 STD = 0.02
 TAU_C, TAU_D = 0.70, 0.98
-# name: (shape, batch, prompt, generation, window, weight seed, LM-head scale, steps checked)
+# name: (shape, batch, prompt, generation, window, weight seed, LM-head scale, steps checked,
+#        key / value cache)
 CONFIGS = {
-    "llada8b": ("llada8b", 1, 256, 256, 128, 1, 12.0, None),
-    "llada8b-long": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None),
-    "llada8b-long-b8": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 24),
-    "dream7b": ("dream7b", 16, 384, 512, 256, 2, 12.8, 12),
+    "llada8b": ("llada8b", 1, 256, 256, 128, 1, 12.0, None, 0),
+    "llada8b-long": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 0),
+    "llada8b-long-b8": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 24, 0),
+    "dream7b": ("dream7b", 16, 384, 512, 256, 2, 12.8, 12, 0),
+    # the approximate prefix key / value cache (refresh at every 32-position block)
+    "llada8b-long-cache": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 1),
+    "llada8b-long-b8-cache": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 40, 1),
+    "dream7b-cache": ("dream7b", 16, 384, 512, 256, 2, 12.8, 40, 1),
 }
 
 
@@ -52,20 +60,20 @@ def dcl():
 
 
 def _context(dcl, name):
-    shape, B, N, M, L, seed, lm_scale, _ = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, _, cache = CONFIGS[name]
     sh = syn.SHAPES[shape]
     stream = torch.cuda.Stream()
     ctx = dcl.Context(sh, max_batch=B, max_seq=N + M, stream=stream.cuda_stream)
     ctx.init_random_weights(seed, STD, lm_scale, 0.0)
     prompt = syn.prompt_ids(1000, B, N, sh.mask_id)
-    cfg = dcl.decode_config(tau_commit=TAU_C, tau_draft=TAU_D, max_window=L, block_len=32, gen_len=M)
+    cfg = dcl.decode_config(tau_commit=TAU_C, tau_draft=TAU_D, max_window=L, block_len=32, gen_len=M, kv_cache=cache)
     ctx.set_prompt(prompt, cfg)
     return ctx, stream, prompt
 
 
 @pytest.mark.parametrize("name,layers", [("llada8b", (0, 1)), ("dream7b", (0,))])
 def test_first_blocks_match_oracle(dcl, name, layers):
-    shape, B, N, M, L, seed, lm_scale, _ = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, _, _ = CONFIGS[name]
     sh = syn.SHAPES[shape]
     T = N + M
     ctx, stream, prompt = _context(dcl, name)
@@ -119,7 +127,7 @@ def _expected_step(x0, p0, top1, c1, N, L, mask_id):
 
 @pytest.mark.parametrize("name", list(CONFIGS))
 def test_generation_follows_acceptance_rule(dcl, name):
-    shape, B, N, M, L, seed, lm_scale, check_steps = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, check_steps, _ = CONFIGS[name]
     sh = syn.SHAPES[shape]
     T = N + M
     ctx, stream, prompt = _context(dcl, name)
