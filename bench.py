@@ -51,6 +51,13 @@ WORKLOADS = {
     # Dream-7B shape (GQA 28 / 4 heads), batch 16, prompt 384, gen 512, full recompute
     "dream7b": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
                     seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98),
+    # the same three with the approximate prefix key / value cache (BASELINE configs 4 / 5)
+    "llada8b-long-cache": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
+                               seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=1),
+    "llada8b-long-b8-cache": dict(shape="llada8b", batch=8, n_prompt=512, gen=1024, block=32, window=512,
+                                  seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=1),
+    "dream7b-cache": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
+                          seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98, cache=1),
     # the LLaDA-8B shape cut to 2 layers (~3 GB on the device): the same GEMM, attention and
     # LM-head launches as the full model, small enough for ncu captures with replay
     "llada8b-2l": dict(shape="llada8b-2l", batch=1, n_prompt=256, gen=256, block=32, window=128,
@@ -81,10 +88,15 @@ def _peaks():
                 "source": "fallback"}
 
 
-def step_work(shape, B, N, M):
-    """Algorithmic flops per step by kernel class, and the minimum HBM bytes of a step."""
+def step_work(shape, B, N, M, rows=None, lm_rows=None, cached=False):
+    """Algorithmic flops per step by kernel class, and the minimum HBM bytes of a step.
+
+    Full recompute computes all B*T rows; with the key / value cache a step computes
+    ``rows`` query rows (``lm_rows`` of them at generation positions), each attending to all
+    T positions, and reads the stored keys / values of every layer."""
     T = N + M
-    R = B * T
+    R = B * T if rows is None else rows
+    R_lm = B * M if lm_rows is None else lm_rows
     d, H, G, hd, F, V = (shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
                          shape.ffn_dim, shape.vocab)
     L = shape.n_layers
@@ -93,14 +105,39 @@ def step_work(shape, B, N, M):
         "gemm_o": 2.0 * R * H * hd * d,
         "gemm_gateup": 2.0 * R * d * 2 * F,
         "gemm_down": 2.0 * R * F * d,
-        "attention": 4.0 * B * T * T * H * hd,
+        "attention": 4.0 * R * T * H * hd,
     }
     per_layer = dict(flops)
     total = {k: v * L for k, v in flops.items()}
-    total["gemm_lmhead"] = 2.0 * B * M * d * V
+    total["gemm_lmhead"] = 2.0 * R_lm * d * V
     w_layer = 2.0 * (d * (H + 2 * G) * hd + H * hd * d + 2 * F * d + F * d + 2 * d)
     bytes_ = L * w_layer + 2.0 * V * d + 2.0 * R * d + 2.0 * d
+    if cached:
+        bytes_ += L * 2.0 * 2.0 * B * T * G * hd  # stored keys and values read by the attention
     return per_layer, total, bytes_
+
+
+def cached_rows(kper, N, M, block):
+    """Per step of a trajectory (per-row K values), the rows the cached step computes and
+    its LM rows (the refresh rule of the key / value cache)."""
+    B = len(kper[0])
+    T = N + M
+    p = [N] * B
+    pe_prev = [None] * B
+    out = []
+    for k in kper:
+        rows = lm = 0
+        for b in range(B):
+            if p[b] >= T:
+                continue
+            pe = N + block * ((p[b] - N) // block)
+            start = 0 if pe != pe_prev[b] else pe
+            pe_prev[b] = pe
+            rows += T - start
+            lm += T - max(start, N)
+            p[b] += int(k[b])
+        out.append((rows, lm))
+    return out
 
 
 # ---------------------------------------------------------------------- clocks
@@ -251,7 +288,8 @@ def run_reference(args):
 def _config(wl, args):
     return {"workload": f"{wl['shape']}-shape batch {wl['batch']}, prompt {wl['n_prompt']}, gen {wl['gen']}, "
                         f"block {wl['block']}, window {wl['window']}, tau_commit {wl['tau_c']}, "
-                        f"tau_draft {wl['tau_d']}, full recompute",
+                        f"tau_draft {wl['tau_d']}, "
+                        + ("approximate prefix key/value cache" if wl.get("cache") else "full recompute"),
             "global_batch": wl["batch"] * max(1, args.gpus), "seq_len": wl["n_prompt"] + wl["gen"],
             "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single",
             "l2": "no flush needed: every step streams all weights (>> 129 MB L2)"}
@@ -283,14 +321,17 @@ def run_ours(args):
     ctx = dcl.Context(shape, max_batch=B, max_seq=T, stream=stream.cuda_stream)
     ctx.init_random_weights(wl["seed"], 0.02, wl["lm_scale"], 0.0)
     prompt = syn.prompt_ids(1000 + rank, B, N, shape.mask_id)
+    cached = int(wl.get("cache", 0))
     cfg = dcl.decode_config(tau_commit=wl["tau_c"], tau_draft=wl["tau_d"], max_window=wl["window"],
-                            block_len=wl["block"], gen_len=M)
+                            block_len=wl["block"], gen_len=M, kv_cache=cached)
     ctx.set_prompt(prompt, cfg)
 
     # one generation step by step: the trajectory (tokens committed per step) + warm-up
-    ks = []
+    ks, kper = [], []
     while sum(ks) < B * M and len(ks) < 4 * M:
-        ks.append(int(ctx.step(return_k=True).sum()))
+        kr = ctx.step(return_k=True)
+        kper.append(kr.copy())
+        ks.append(int(kr.sum()))
     S = len(ks)
     ctx.restart()
     for _ in range(args.warmup):
@@ -372,10 +413,19 @@ def run_ours(args):
     # the trajectory's average rate, B*M tokens per S steps: the window need not cover
     # whole generations for the value to equal whole-generation throughput
     per_step = B * M / S
-    tokens_all = allsum(args.steps * per_step)
+    # (cached steps differ in cost: the window is credited the tokens it actually committed)
+    tokens_all = allsum(tokens if cached else args.steps * per_step)
     e2e_mean = allmax(statistics.mean(e2e_s))
     peaks = _peaks()
-    per_layer, total_flops, step_bytes = step_work(shape, B, N, M)
+    if cached:
+        # the cached step's work varies (refresh or suffix): the trajectory's mean
+        rl = cached_rows(kper, N, M, wl["block"])
+        works = [step_work(shape, B, N, M, r, l, True) for r, l in rl]
+        per_layer = works[0][0]
+        total_flops = {k: statistics.mean(w[1][k] for w in works) for k in works[0][1]}
+        step_bytes = statistics.mean(w[2] for w in works)
+    else:
+        per_layer, total_flops, step_bytes = step_work(shape, B, N, M)
 
     # per-kernel table and the dominant kernel's roofline
     names = dcl.KERNEL_KINDS
