@@ -224,9 +224,12 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * tiles of a partly filled last round of the persistent grid are cut into about S K
  * segments each (S = 0: shared out over all CTA pairs) run by different pairs; rejected
  * with DCL_ERR_INVALID_ARG when the last round is full or a sharing pair would get no K
- * block.  Partial sums are always combined in K order, so every choice is deterministic. */
+ * block; DCL_TILE_PAIR | DCL_TILE_MULTICAST clusters of two CTA pairs on consecutive
+ * 256-row blocks that load each weight tile from L2 once (TMA multicast; M > 256).
+ * Partial sums are always combined in K order, so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
 #define DCL_TILE_STREAMK (1 << 16)
+#define DCL_TILE_MULTICAST (1 << 17)
 
 /* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05
  * tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];
