@@ -7,9 +7,11 @@ fail loudly rather than fall back to it.
 
 Modules:
   model   - masked-diffusion transformer forward and per-position softmax
-            confidence (Eq. 1, Eq. 2, top-1 of Eq. threshold_pd, top-2 of Sec. 2.2)
+            confidence (Eq. 1, Eq. 2, top-1 of Eq. threshold_pd, top-2 of Sec. 2.2,
+            the marginal entropy of Eq. entropy_bound)
   decode  - Dynamic Contiguous Verification and draft-guided decoding
-            (Eq. compute_k, Eq. draft_update, Eq. remasking, Sec. 3.3, Algorithm 1)
+            (Eq. compute_k, Eq. draft_update, Eq. remasking, Sec. 3.3, Algorithm 1),
+            the entropy confidence and Eq. entropy_bound of each committed set
   accept  - the acceptance pass on given logits (Eq. 2 + Eq. compute_k +
             Eq. draft_update for a block of positions)
 

@@ -23,6 +23,14 @@ Readings where the paper is silent or inconsistent (each one is also a test):
   * drafts are refreshed at every future position, masked or already drafted;
   * decisions compare the confidence and the threshold as float32 values, the
     precision in which the CUDA kernel takes them;
+  * ``confidence = 1`` replaces the top-1 probability by the marginal-entropy confidence
+    c = exp(-H), H = -sum_v P(v) ln P(v) over the whole vocabulary (App. F.3 tries other
+    confidence definitions; this one needs only the same single forward, and H is the
+    per-token entropy of Eq. entropy_bound); exp(-H) <= sum_v P(v)^2 <= p1, so it never
+    accepts a position the top-1 probability would reject;
+  * every step records Eq. entropy_bound on the set it committed in parallel,
+    sum_{i in U} H_i - max_{j in U} H_j with U = [p, p + K) and the step's own marginal
+    entropies (0 when K = 1);
   * the approximate cache (``kv_cache = 1``; the paper pairs DC-Leap with a dLLM cache in
     Sec. 4 / Tab. 6 without describing its policy): per row, a step computes all
     positions at the first step and whenever the block-aligned prefix end
@@ -47,6 +55,7 @@ class DecodeConfig:
     min_commit: int = 1
     contiguous_drafts: bool = False  # App. E variant: drafts only as an unbroken chain
     kv_cache: int = 0
+    confidence: int = 0           # 0: top-1 probability (Eq. threshold_pd); 1: exp(-entropy)
 
     def window(self) -> int:
         return self.max_window if self.max_window > 0 else max(1, self.gen_len // 2)
@@ -86,6 +95,32 @@ def commit_and_draft(x: np.ndarray, p: int, ids: np.ndarray, c: np.ndarray,
     return K
 
 
+def entropy_confidence(H) -> np.ndarray:
+    """c = exp(-H) of the marginal entropy H (nats): 1 for a certain prediction, 1/V for a
+    uniform one."""
+    return np.exp(-np.asarray(H, dtype=np.float64))
+
+
+def jpde_bound(H_set) -> float:
+    """Eq. entropy_bound: sum_{i in U} H_i - max_{j in U} H_j for the marginal entropies of
+    a set U of positions decoded in parallel (0 for fewer than two positions)."""
+    H_set = np.asarray(H_set, dtype=np.float64)
+    if H_set.size < 2:
+        return 0.0
+    return float(H_set.sum() - H_set.max())
+
+
+def decision_confidence(p1, H, cfg: DecodeConfig) -> np.ndarray:
+    """The c compared with the thresholds: p1, or exp(-H) with ``cfg.confidence = 1``."""
+    if cfg.confidence == 0:
+        return np.asarray(p1, dtype=np.float64)
+    if cfg.confidence != 1:
+        raise ValueError("confidence must be 0 (top-1 probability) or 1 (exp(-entropy))")
+    if H is None:
+        raise ValueError("the entropy confidence needs the marginal entropies")
+    return entropy_confidence(H)
+
+
 def prefix_end(p: int, n_prompt: int, block_len: int) -> int:
     """Block-aligned start of the current block: N + Bk * floor((p - N) / Bk)."""
     return n_prompt + block_len * ((p - n_prompt) // block_len)
@@ -95,13 +130,15 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
              max_steps: int = 1 << 30, record: bool = True) -> dict:
     """Algorithm 1 for a batch of independent rows.
 
-    predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) for the generation positions.  With
+    predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) or (ids, p1, p2, H[M]) for the
+    generation positions (H, the marginal entropies, is needed by ``confidence = 1``).  With
     ``cfg.kv_cache`` it is called as predict_fn(tokens[T], start, state): only positions
     >= start need be computed and ``state`` is the row's cache; start is 0 at the first
     step and whenever prefix_end(p) changes (a refresh), else prefix_end(p).
     Returns the final x [B][T], per-row steps, the K of every step, the start of every
-    step (-1 for finished rows), and (if ``record``) the forward input of every step and
-    the predictions it produced.
+    step (-1 for finished rows), Eq. entropy_bound of every step's committed set (NaN
+    without entropies), and (if ``record``) the forward input of every step and the
+    predictions it produced (ids, p1, p2, H).
     """
     prompt = np.atleast_2d(np.asarray(prompt, dtype=np.int32))
     B, N = prompt.shape
@@ -112,14 +149,16 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
     x[:, :N] = prompt
     p = np.full(B, N, dtype=np.int64)
     steps = np.zeros(B, dtype=np.int64)
-    ks, starts, inputs, preds = [], [], [], []
+    ks, starts, inputs, preds, bounds = [], [], [], [], []
     caches = [{"pe": None} for _ in range(B)]
     n_iter = 0
     while (p < T).any() and n_iter < max_steps:
         k_step = np.zeros(B, dtype=np.int64)
         s_step = np.full(B, -1, dtype=np.int64)
         in_step = np.empty((B, T), dtype=np.int32)
-        pr = np.zeros((3, B, M))
+        pr = np.zeros((4, B, M))
+        pr[3] = np.nan
+        jp = np.zeros(B)
         for b in range(B):
             if p[b] >= T:
                 in_step[b] = x[b]
@@ -129,25 +168,33 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             if cfg.kv_cache:                                     # (ii), approximate cache
                 pe = prefix_end(int(p[b]), N, cfg.block_len)
                 s_step[b] = 0 if caches[b]["pe"] != pe else pe
-                ids, p1, p2 = predict_fn(x[b].copy(), int(s_step[b]), caches[b])
+                out = predict_fn(x[b].copy(), int(s_step[b]), caches[b])
                 caches[b]["pe"] = pe
             else:                                                # (ii)
                 s_step[b] = 0
-                ids, p1, p2 = predict_fn(x[b].copy())
+                out = predict_fn(x[b].copy())
+            ids, p1, p2 = out[:3]
+            H = out[3] if len(out) > 3 else None
             full_ids = np.zeros(T, dtype=np.int32)
             full_c = np.zeros(T, dtype=np.float64)
             full_ids[N:] = ids
-            full_c[N:] = p1
-            k_step[b] = commit_and_draft(x[b], int(p[b]), full_ids, full_c, cfg, L)  # (iii)-(iv)
+            full_c[N:] = decision_confidence(p1, H, cfg)
+            p0 = int(p[b])
+            k_step[b] = commit_and_draft(x[b], p0, full_ids, full_c, cfg, L)  # (iii)-(iv)
+            jp[b] = np.nan if H is None else jpde_bound(np.asarray(H)[p0 - N:p0 - N + k_step[b]])
             p[b] += k_step[b]                                    # dynamically advance
             steps[b] += 1
             pr[0, b], pr[1, b], pr[2, b] = ids, p1, p2
+            if H is not None:
+                pr[3, b] = H
         ks.append(k_step)
         starts.append(s_step)
+        bounds.append(jp)
         if record:
             inputs.append(in_step)
             preds.append(pr)
         n_iter += 1
-    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "start": np.array(starts), "inputs": inputs,
+    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "start": np.array(starts),
+            "jpde": np.array(bounds), "inputs": inputs,
             "preds": preds, "n_iter": n_iter, "done": bool((p >= T).all())}
 

@@ -179,10 +179,11 @@ def new_kv_store(shape, T: int) -> list:
 
 
 def predict_from(shape, weights: dict, tokens: np.ndarray, start: int, state: dict, n_prompt: int,
-                 bf16_operands: bool = False):
+                 bf16_operands: bool = False, with_entropy: bool = False):
     """(ids, p1, p2) over the generation positions [n_prompt, T) computing only positions
     >= start (the others are returned as -1 / NaN); ``state["kv"]`` is the sequence's
-    key / value store, created on first use."""
+    key / value store, created on first use.  With ``with_entropy`` the marginal entropy
+    H of every computed position follows (NaN elsewhere)."""
     T = len(tokens)
     if state.get("kv") is None:
         state["kv"] = new_kv_store(shape, T)
@@ -193,9 +194,14 @@ def predict_from(shape, weights: dict, tokens: np.ndarray, start: int, state: di
     p1 = np.full(M, np.nan)
     p2 = np.full(M, np.nan)
     gen = pos >= n_prompt
-    i, c1, c2 = confidence(logits(weights, hid[gen]))
+    z = logits(weights, hid[gen])
+    i, c1, c2 = confidence(z)
     ids[pos[gen] - n_prompt], p1[pos[gen] - n_prompt], p2[pos[gen] - n_prompt] = i, c1, c2
-    return ids, p1, p2
+    if not with_entropy:
+        return ids, p1, p2
+    H = np.full(M, np.nan)
+    H[pos[gen] - n_prompt] = entropy(z)
+    return ids, p1, p2, H
 
 
 def logits(weights: dict, hidden: np.ndarray) -> np.ndarray:
@@ -228,9 +234,24 @@ def confidence(z: np.ndarray):
     return ids.astype(np.int32), 1.0 / s, np.exp(z2 - m) / s
 
 
-def predict(shape, weights: dict, tokens: np.ndarray, rows=None, bf16_operands: bool = False):
-    """Forward + confidence: (ids, p1, p2) for positions ``rows`` (all positions by default)."""
+def entropy(z: np.ndarray) -> np.ndarray:
+    """Marginal entropy H = -sum_v P(v) ln P(v) of the Eq. 2 distribution, in nats, per row.
+
+    This is the per-token H(x_i | C) of Eq. entropy_bound; a term with P(v) = 0 (an
+    underflowed probability) contributes 0, its limit.
+    """
+    p = softmax(np.atleast_2d(z))
+    with np.errstate(divide="ignore", invalid="ignore"):
+        t = np.where(p > 0, p * np.log(p), 0.0)
+    return -t.sum(axis=-1)
+
+
+def predict(shape, weights: dict, tokens: np.ndarray, rows=None, bf16_operands: bool = False,
+            with_entropy: bool = False):
+    """Forward + confidence: (ids, p1, p2) for positions ``rows`` (all positions by
+    default), and the marginal entropy H of every position when ``with_entropy``."""
     hid = forward_hidden(shape, weights, tokens, bf16_operands)
     if rows is not None:
         hid = hid[rows]
-    return confidence(logits(weights, hid))
+    z = logits(weights, hid)
+    return confidence(z) + ((entropy(z),) if with_entropy else ())
