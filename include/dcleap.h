@@ -60,10 +60,15 @@ typedef struct {
   int32_t max_window;        /* L; 0 means gen_len / 2 */
   int32_t block_len;         /* 32: semi-autoregressive block length */
   int32_t gen_len;           /* M, the number of generated positions */
-  int32_t kv_cache;          /* 0: full recompute every step (the only mode built) */
+  int32_t kv_cache;          /* 0: full recompute every step; 1: approximate prefix key /
+                                value cache refreshed at block boundaries (see dcl_set_prompt) */
   int32_t min_commit;        /* 1: K = max(K, min_commit) so every step makes progress;
                                 0 keeps the literal rule (may stall; bounded by max_steps) */
   int32_t contiguous_drafts; /* 0; 1 = App. E variant (drafts only as an unbroken chain) */
+  int32_t confidence;        /* 0: c = top-1 probability (Eq. threshold_pd, the paper's choice);
+                                1: c = exp(-H), H = -sum_v P(v) ln P(v) the marginal entropy of
+                                Eq. entropy_bound (an alternative confidence, cf. App. F.3);
+                                exp(-H) <= p1, so it never accepts more than 0 */
 } dcl_decode_config;
 
 typedef struct {
@@ -71,6 +76,9 @@ typedef struct {
   int64_t tokens;     /* generated tokens committed (all rows) */
   double elapsed_ms;  /* wall time of dcl_generate, host clock */
   int32_t done;       /* 1 if every row reached p = N + M */
+  double jpde_bound;  /* Eq. entropy_bound (sum_U H - max_U H, nats) of every set U = [p, p+K)
+                         committed in parallel since dcl_set_prompt / dcl_restart /
+                         dcl_set_state, summed over steps and rows (fp32 per row) */
 } dcl_stats;
 
 /* Optional device allocator (e.g. a framework's caching allocator). */
@@ -130,7 +138,8 @@ dcl_status dcl_init_random_weights(dcl_ctx* ctx, uint64_t seed, float std, float
  * (Eq. 1).  prompt is host int32 [batch][n_prompt]; batch <= max_batch,
  * n_prompt + cfg->gen_len <= max_seq.  Validates ids, uploads the state and builds
  * (or reuses) the CUDA graph of one step for this shape.
- * Errors: INVALID_ARG, UNSUPPORTED (kv_cache != 0), CUDA. */
+ * Errors: INVALID_ARG (also kv_cache or confidence outside {0, 1}), UNSUPPORTED (kv_cache
+ * = 1 with N, M or block_len not a multiple of 32), CUDA. */
 dcl_status dcl_set_prompt(dcl_ctx* ctx, int32_t batch, const int32_t* prompt, int32_t n_prompt,
                           const dcl_decode_config* cfg);
 
@@ -161,11 +170,13 @@ dcl_status dcl_set_state(dcl_ctx* ctx, const int32_t* x, const int32_t* p);
 /* Parity hook: step (i) and (ii) only (re-mask, forward, confidence) on the current
  * state, without committing.  Any output may be NULL:
  *   logits_dev bf16 [batch][M][V] logits of the generation rows (an extra plain GEMM),
- *   top1_dev int32 [batch][M], p1_dev / p2_dev float [batch][M] from the fused
- *   LM-head epilogue (the values the step itself uses).
+ *   top1_dev int32 [batch][M], p1_dev / p2_dev float [batch][M] (top-1 / top-2
+ *   probabilities), conf_dev float [batch][M] (the confidence the thresholds see: p1, or
+ *   exp(-H) with confidence = 1), entropy_dev float [batch][M] (marginal entropy H in
+ *   nats), all from the fused LM-head epilogue (the values the step itself uses).
  * Errors: STATE, CUDA. */
 dcl_status dcl_forward_debug(dcl_ctx* ctx, void* logits_dev, int32_t* top1_dev, float* p1_dev,
-                             float* p2_dev);
+                             float* p2_dev, float* conf_dev, float* entropy_dev);
 
 /* Parity hook: the residual stream after the embedding (layer = -1) or after
  * transformer block `layer` of the last forward, copied to h_dev (float [batch*(N+M)][d]).
@@ -248,11 +259,12 @@ dcl_status dcl_op_attention(dcl_ctx* ctx, const void* qkv_dev, void* out_dev, in
 /* LM head + softmax confidence fused (Eq. 2; top-1 of Eq. threshold_pd; top-2 of
  * Sec. 2.2): for each row r of x_dev (bf16 [R][d]), z = x_r @ w^T (w_dev bf16 [V][d]);
  * top1_dev[r] = argmax (lowest index on ties), p1_dev[r] = max softmax(z), p2_dev[r] =
- * second largest probability.  Logits never reach memory.  d a multiple of 64;
- * tile 0, 256 or DCL_TILE_PAIR.  Synchronises. */
+ * second largest probability, entropy_dev[r] (may be NULL) = -sum_v P(v) ln P(v) (nats,
+ * the per-token entropy of Eq. entropy_bound).  Logits never reach memory.  d a multiple
+ * of 64; tile 0, 256 or DCL_TILE_PAIR.  Synchronises. */
 dcl_status dcl_op_lmhead_top2(dcl_ctx* ctx, const void* x_dev, const void* w_dev, int32_t R,
                               int32_t V, int32_t d, int32_t* top1_dev, float* p1_dev,
-                              float* p2_dev, int32_t tile);
+                              float* p2_dev, float* entropy_dev, int32_t tile);
 
 /* Fill dst_dev (bf16, count elements) from the weight generator of
  * dcl_init_random_weights for tensor id `tid` starting at element `start`.  Async. */

@@ -44,12 +44,14 @@ class DecodeConfig(ctypes.Structure):
     _fields_ = [("tau_commit", ctypes.c_float), ("tau_draft", ctypes.c_float),
                 ("max_window", ctypes.c_int32), ("block_len", ctypes.c_int32),
                 ("gen_len", ctypes.c_int32), ("kv_cache", ctypes.c_int32),
-                ("min_commit", ctypes.c_int32), ("contiguous_drafts", ctypes.c_int32)]
+                ("min_commit", ctypes.c_int32), ("contiguous_drafts", ctypes.c_int32),
+                ("confidence", ctypes.c_int32)]
 
 
 class Stats(ctypes.Structure):
     _fields_ = [("steps", ctypes.c_int64), ("tokens", ctypes.c_int64),
-                ("elapsed_ms", ctypes.c_double), ("done", ctypes.c_int32)]
+                ("elapsed_ms", ctypes.c_double), ("done", ctypes.c_int32),
+                ("jpde_bound", ctypes.c_double)]
 
 
 class Allocator(ctypes.Structure):
@@ -71,14 +73,14 @@ SIGNATURES = {
     "dcl_restart": (_I, [_P]),
     "dcl_get_state": (_I, [_P, _P, _P]),
     "dcl_set_state": (_I, [_P, _P, _P]),
-    "dcl_forward_debug": (_I, [_P, _P, _P, _P, _P]),
+    "dcl_forward_debug": (_I, [_P, _P, _P, _P, _P, _P, _P]),
     "dcl_debug_hidden": (_I, [_P, _I, _P]),
     "dcl_accept": (_I, [_P, _P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P]),
     "dcl_accept_noalloc": (_I, [_P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P, _P]),
     "dcl_op_rmsnorm": (_I, [_P, _P, _P, _P, _I, _I, _F]),
     "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I]),
     "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I]),
-    "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _I]),
+    "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _I]),
     "dcl_op_generate": (_I, [_P, _P, ctypes.c_uint64, _I, ctypes.c_int64, ctypes.c_int64, _F, _F]),
     "dcl_set_profiling": (_I, [_P, _I]),
     "dcl_profile_last_step": (_I, [_P, _P, _P, _I, _P]),
@@ -141,9 +143,10 @@ def model_config(shape) -> ModelConfig:
 
 
 def decode_config(tau_commit=0.70, tau_draft=0.98, max_window=0, block_len=32, gen_len=0,
-                  kv_cache=0, min_commit=1, contiguous_drafts=0) -> DecodeConfig:
+                  kv_cache=0, min_commit=1, contiguous_drafts=0, confidence=0) -> DecodeConfig:
+    """confidence: 0 = top-1 probability, 1 = exp(-entropy)."""
     return DecodeConfig(tau_commit, tau_draft, max_window, block_len, gen_len, kv_cache,
-                        min_commit, int(bool(contiguous_drafts)))
+                        min_commit, int(bool(contiguous_drafts)), confidence)
 
 
 class Context:
@@ -240,8 +243,9 @@ class Context:
         p = np.ascontiguousarray(p, dtype=np.int32)
         self._check(self._L.dcl_set_state(self.ptr, _ptr(x), _ptr(p)))
 
-    def forward_debug(self, logits=None, top1=None, p1=None, p2=None):
-        self._check(self._L.dcl_forward_debug(self.ptr, _ptr(logits), _ptr(top1), _ptr(p1), _ptr(p2)))
+    def forward_debug(self, logits=None, top1=None, p1=None, p2=None, conf=None, entropy=None):
+        self._check(self._L.dcl_forward_debug(self.ptr, _ptr(logits), _ptr(top1), _ptr(p1), _ptr(p2),
+                                              _ptr(conf), _ptr(entropy)))
 
     def debug_hidden(self, layer, h):
         self._check(self._L.dcl_debug_hidden(self.ptr, layer, _ptr(h)))
@@ -263,11 +267,11 @@ class Context:
     def op_attention(self, qkv, out, batch, T, H, G, hd):
         self._check(self._L.dcl_op_attention(self.ptr, _ptr(qkv), _ptr(out), batch, T, H, G, hd))
 
-    def op_lmhead_top2(self, x, w, top1, p1, p2, tile=0):
+    def op_lmhead_top2(self, x, w, top1, p1, p2, tile=0, entropy=None):
         R, d = x.shape
         V = w.shape[0]
         self._check(self._L.dcl_op_lmhead_top2(self.ptr, _ptr(x), _ptr(w), R, V, d, _ptr(top1),
-                                               _ptr(p1), _ptr(p2), tile))
+                                               _ptr(p1), _ptr(p2), _ptr(entropy), tile))
 
     def op_generate(self, dst, seed, tid, start, count, std, mean=0.0):
         self._check(self._L.dcl_op_generate(self.ptr, _ptr(dst), seed, tid, start, count, std, mean))

@@ -56,7 +56,7 @@ extern "C" dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int3
                              .c_str());
     return DCL_ERR_INVALID_ARG;
   }
-  if (cfg->max_window < 0 || cfg->min_commit < 0) {
+  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1)) {
     dcl::set_thread_error("dcl_accept_noalloc: bad decode config");
     return DCL_ERR_INVALID_ARG;
   }
@@ -78,7 +78,7 @@ extern "C" dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int3
   dcl::DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts};
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = dcl::accept_stats_launch(static_cast<const __nv_bfloat16*>(logits_dev), committed_dev, B, P, V, ids, c1,
-                               c2, s);
+                               c2, cfg->confidence, s);
   if (e == cudaSuccess) e = dcl::accept_commit_launch(committed_dev, ids, c1, x_dev, k_dev, B, P, prm, s);
   if (e != cudaSuccess) {
     dcl::set_thread_error((std::string("dcl_accept_noalloc: launch failed: ") + cudaGetErrorString(e)).c_str());

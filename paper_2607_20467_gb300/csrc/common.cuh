@@ -59,6 +59,7 @@ __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 
 // ---------------------------------------------------------------- GEMM (gemm_tc.cu)
 // out = A[M][K] @ W[N][K]^T on tcgen05 tensor cores, with a fused epilogue.
@@ -87,6 +88,7 @@ struct EpiParams {
   const int* m_dev = nullptr;       // device row count (<= M) of the launch, or NULL
   const int* row_pos = nullptr;     // device position of each row (NULL: row % seq_T)
   const int* row_seq = nullptr;     // device sequence of each row (NULL: row / seq_T)
+  float* ent_part = nullptr;        // LM head: [rows][tiles] sum of e * y (entropy partials) or NULL
 };
 
 struct GemmPlan {
@@ -191,19 +193,31 @@ cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, 
 // y row r = normalised x row src[r] (src NULL: r), for r < min(rows, *rows_dev).
 cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloat16* y, int rows,
                            int d, float eps, const int* rows_dev, const int* src, cudaStream_t stream);
-cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
-                                  float* p2, const int* rows_dev, const int* slot, cudaStream_t stream);
+// Per-position outputs of the softmax statistics (any pointer but top1 may be NULL).
+struct ConfOut {
+  int32_t* top1 = nullptr;
+  float* p1 = nullptr;    // top-1 probability
+  float* p2 = nullptr;    // top-2 probability
+  float* ent = nullptr;   // marginal entropy H (nats)
+  float* conf = nullptr;  // the confidence the thresholds see: p1 (mode 0) or exp(-H) (mode 1)
+  int mode = 0;
+};
+// part: [rows][nblk] {max, sum exp(z - max), id, second max}; upart: [rows][nblk] entropy
+// partials (sum of e * y, y = (z - max) log2 e) or NULL (then H is not available).
+cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int rows, int nblk, const ConfOut& o,
+                                  const int* rows_dev, const int* slot, cudaStream_t stream);
 struct DcvParams {
   float tau_commit, tau_draft;
   int window, min_commit, contiguous_drafts;
 };
-// One step's acceptance on the generation rows: ids/c are [batch][M] (position N + i).
+// One step's acceptance on the generation rows: ids/c (and ent) are [batch][M] (position
+// N + i).  With ent, jpde[b] accumulates Eq. entropy_bound of the set row b commits.
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
-                              const int32_t* ids, const float* c, int batch, int N, int M,
-                              const DcvParams& prm, int32_t* done_count, cudaStream_t stream);
-// Block acceptance from bf16 logits (dcl_accept).
+                              const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
+                              int N, int M, const DcvParams& prm, int32_t* done_count, cudaStream_t stream);
+// Block acceptance from bf16 logits (dcl_accept): c1 = p1 (mode 0) or exp(-H) (mode 1).
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B,
-                                int P, int V, int32_t* ids, float* c1, float* c2,
+                                int P, int V, int32_t* ids, float* c1, float* c2, int mode,
                                 cudaStream_t stream);
 cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, const float* c1,
                                  int32_t* x, int32_t* k, int B, int P, const DcvParams& prm,

@@ -58,8 +58,12 @@ struct dcl_ctx {
   int* rp_buf = nullptr;          // the row plan's tables
   RowPlan rp;
   float4* part = nullptr;
+  float* ent_part = nullptr;  // LM-head entropy partials [rows][tiles]
   int32_t* top1 = nullptr;
   float *p1 = nullptr, *p2 = nullptr;
+  float* ent = nullptr;   // marginal entropy H of every generation position
+  float* conf = nullptr;  // exp(-H) (the thresholds' input with confidence = 1)
+  float* jpde = nullptr;  // per row: Eq. entropy_bound summed over the committed sets
   int32_t *x = nullptr, *p = nullptr, *k = nullptr, *steps = nullptr, *done_count = nullptr;
   int32_t *x_init = nullptr, *p_init = nullptr;  // state at the last dcl_set_prompt
   int* derr = nullptr;
@@ -254,14 +258,21 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
   q.begin(DCL_K_GEMM_LMHEAD);
   q.end(gemm_launch(c->plans[4 * m.n_layers], c->derr, c->stream), "gemm_lmhead");
   q.begin(DCL_K_COMBINE);
-  q.end(lmhead_combine_launch(c->part, c->B * c->M, gemm_lmhead_blocks(m.vocab), c->top1, c->p1, c->p2,
-                              c->rp.counts + 1, c->rp.lm_slot, c->stream),
+  ConfOut co;
+  co.top1 = c->top1;
+  co.p1 = c->p1;
+  co.p2 = c->p2;
+  co.ent = c->ent;
+  co.mode = c->dcfg.confidence;
+  co.conf = co.mode ? c->conf : c->p1;
+  q.end(lmhead_combine_launch(c->part, c->ent_part, c->B * c->M, gemm_lmhead_blocks(m.vocab), co, c->rp.counts + 1,
+                              c->rp.lm_slot, c->stream),
         "combine");
   if (with_dcv) {
     DcvParams prm{c->dcfg.tau_commit, c->dcfg.tau_draft, c->window, c->dcfg.min_commit,
                   c->dcfg.contiguous_drafts};
     q.begin(DCL_K_DCV);
-    q.end(dcv_commit_launch(c->x, c->p, c->k, c->steps, c->top1, c->p1, c->B, c->N, c->M, prm,
+    q.end(dcv_commit_launch(c->x, c->p, c->k, c->steps, c->top1, co.conf, c->ent, c->jpde, c->B, c->N, c->M, prm,
                             c->done_count, c->stream),
           "dcv_commit");
   }
@@ -395,6 +406,7 @@ dcl_status build_plans(dcl_ctx* c) {
       return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
   EpiParams el;
   el.out = c->part;
+  el.ent_part = c->ent_part;
   el.m_dev = c->rp.counts + 1;
   if (gemm_plan(&c->plans[4 * m.n_layers], c->xg, c->B * c->M, d, c->lm_head, m.vocab, EPI_LMHEAD, el,
                 c->num_sms, t_lm, &why))
@@ -622,6 +634,10 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->act = (__nv_bfloat16*)dev_alloc(c, 2 * R * F);
     c->xg = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->part = (float4*)dev_alloc(c, sizeof(float4) * R * nblk);
+    c->ent_part = (float*)dev_alloc(c, sizeof(float) * R * nblk);
+    c->ent = (float*)dev_alloc(c, 4 * R);
+    c->conf = (float*)dev_alloc(c, 4 * R);
+    c->jpde = (float*)dev_alloc(c, 4 * (size_t)max_batch);
     c->top1 = (int32_t*)dev_alloc(c, 4 * R);
     c->p1 = (float*)dev_alloc(c, 4 * R);
     c->p2 = (float*)dev_alloc(c, 4 * R);
@@ -634,7 +650,8 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->p_init = (int32_t*)dev_alloc(c, 4 * max_batch);
     c->rope_cos = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
     c->rope_sin = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
-    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->kbuf || !c->rp_buf || !c->act || !c->xg || !c->part || !c->top1 ||
+    if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->kbuf || !c->rp_buf || !c->act || !c->xg || !c->part || !c->ent_part ||
+        !c->ent || !c->conf || !c->jpde || !c->top1 ||
         !c->p1 || !c->p2 || !c->x || !c->p || !c->k || !c->steps || !c->done_count || !c->x_init || !c->p_init || !c->rope_cos ||
         !c->rope_sin) {
       dev_free_all(c);
@@ -746,6 +763,7 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   if (n_prompt < 0 || cfg->gen_len <= 0 || n_prompt + cfg->gen_len > c->max_seq)
     return fail(c, DCL_ERR_INVALID_ARG, "N + M = %d + %d exceeds max_seq %d", n_prompt, cfg->gen_len, c->max_seq);
   if (cfg->kv_cache != 0 && cfg->kv_cache != 1) return fail(c, DCL_ERR_INVALID_ARG, "kv_cache must be 0 or 1");
+  if (cfg->confidence != 0 && cfg->confidence != 1) return fail(c, DCL_ERR_INVALID_ARG, "confidence must be 0 or 1");
   if (cfg->kv_cache && (cfg->block_len <= 0 || cfg->block_len % 32 || n_prompt % 32 || cfg->gen_len % 32))
     return fail(c, DCL_ERR_UNSUPPORTED, "the key / value cache needs N, M and the block length multiples of 32");
   if (cfg->max_window < 0 || cfg->min_commit < 0 || !(cfg->tau_commit == cfg->tau_commit) ||
@@ -773,6 +791,7 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   CUDA_TRY(c, cudaMemcpyAsync(c->x_init, c->x, 4 * xh.size(), cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p_init, c->p, 4 * batch, cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)batch, c->stream));  // no stored keys / values
+  CUDA_TRY(c, cudaMemsetAsync(c->jpde, 0, 4 * (size_t)batch, c->stream));
   s = reset_done_count(c, ph.data());
   if (s != DCL_OK) return s;
   if (reshape) {
@@ -828,8 +847,10 @@ dcl_status dcl_generate(dcl_ctx* c, int32_t max_steps, int32_t* out, dcl_stats* 
   dcl_status s = check_device(c);
   if (s != DCL_OK) return s;
   std::vector<int32_t> ph(c->B), sh(c->B);
+  std::vector<float> jh(c->B);
   CUDA_TRY(c, cudaMemcpy(ph.data(), c->p, 4 * c->B, cudaMemcpyDeviceToHost));
   CUDA_TRY(c, cudaMemcpy(sh.data(), c->steps, 4 * c->B, cudaMemcpyDeviceToHost));
+  CUDA_TRY(c, cudaMemcpy(jh.data(), c->jpde, 4 * c->B, cudaMemcpyDeviceToHost));
   if (out) {
     for (int b = 0; b < c->B; ++b)
       CUDA_TRY(c, cudaMemcpy(out + (size_t)b * c->M, c->x + (size_t)b * c->T + c->N, 4 * c->M,
@@ -838,10 +859,13 @@ dcl_status dcl_generate(dcl_ctx* c, int32_t max_steps, int32_t* out, dcl_stats* 
   const double ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
   if (st) {
     int64_t tok = 0, stp = 0;
+    double jp = 0.0;
     for (int b = 0; b < c->B; ++b) {
       tok += ph[b] - c->N;
       stp = sh[b] > stp ? sh[b] : stp;
+      jp += jh[b];
     }
+    st->jpde_bound = jp;
     st->steps = stp;
     st->tokens = tok;
     st->elapsed_ms = ms;
@@ -861,6 +885,7 @@ dcl_status dcl_restart(dcl_ctx* c) {
   CUDA_TRY(c, cudaMemsetAsync(c->k, 0, 4 * B, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->done_count, 0, 4, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * B, c->stream));
+  CUDA_TRY(c, cudaMemsetAsync(c->jpde, 0, 4 * B, c->stream));
   return DCL_OK;
 }
 
@@ -884,10 +909,12 @@ dcl_status dcl_set_state(dcl_ctx* c, const int32_t* x, const int32_t* p) {
   CUDA_TRY(c, cudaMemcpyAsync(c->x, x, 4 * (size_t)c->B * c->T, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p, p, 4 * (size_t)c->B, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)c->B, c->stream));  // the next step refreshes
+  CUDA_TRY(c, cudaMemsetAsync(c->jpde, 0, 4 * (size_t)c->B, c->stream));
   return reset_done_count(c, p);
 }
 
-dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev) {
+dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev,
+                             float* conf_dev, float* entropy_dev) {
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!c->prompt_set) return fail(c, DCL_ERR_STATE, "no prompt set");
   const size_t R = (size_t)c->B * c->T;
@@ -903,6 +930,10 @@ dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, fl
   if (top1_dev) CUDA_TRY(c, cudaMemcpyAsync(top1_dev, c->top1, 4 * G, cudaMemcpyDeviceToDevice, c->stream));
   if (p1_dev) CUDA_TRY(c, cudaMemcpyAsync(p1_dev, c->p1, 4 * G, cudaMemcpyDeviceToDevice, c->stream));
   if (p2_dev) CUDA_TRY(c, cudaMemcpyAsync(p2_dev, c->p2, 4 * G, cudaMemcpyDeviceToDevice, c->stream));
+  if (conf_dev)
+    CUDA_TRY(c, cudaMemcpyAsync(conf_dev, c->dcfg.confidence ? c->conf : c->p1, 4 * G, cudaMemcpyDeviceToDevice,
+                                c->stream));
+  if (entropy_dev) CUDA_TRY(c, cudaMemcpyAsync(entropy_dev, c->ent, 4 * G, cudaMemcpyDeviceToDevice, c->stream));
   if (logits_dev) {
     GemmPlan pl;
     EpiParams ep;
@@ -937,7 +968,8 @@ dcl_status dcl_accept(dcl_ctx* c, const void* logits_dev, int32_t B, int32_t P, 
   if (!logits_dev || !committed_dev || !x_dev || !cfg || !k_dev) return fail(c, DCL_ERR_INVALID_ARG, "NULL argument");
   if (B <= 0 || P <= 0 || V <= 1 || P > 4096 || (int64_t)B * P > (1 << 20))
     return fail(c, DCL_ERR_INVALID_ARG, "bad B/P/V (P <= 4096, B*P <= 2^20)");
-  if (cfg->max_window < 0 || cfg->min_commit < 0) return fail(c, DCL_ERR_INVALID_ARG, "bad decode config");
+  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1))
+    return fail(c, DCL_ERR_INVALID_ARG, "bad decode config");
   const size_t n = (size_t)B * P;
   if (c->acc_cap < n) {
     c->acc_ids = (int32_t*)dev_alloc(c, 4 * n);
@@ -949,7 +981,7 @@ dcl_status dcl_accept(dcl_ctx* c, const void* logits_dev, int32_t B, int32_t P, 
   const int window = cfg->max_window > 0 ? cfg->max_window : (P / 2 > 0 ? P / 2 : 1);
   DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts};
   CUDA_TRY(c, accept_stats_launch(static_cast<const __nv_bfloat16*>(logits_dev), committed_dev, B, P, V, c->acc_ids,
-                                  c->acc_c1, c->acc_c2, c->stream));
+                                  c->acc_c1, c->acc_c2, cfg->confidence, c->stream));
   CUDA_TRY(c, accept_commit_launch(committed_dev, c->acc_ids, c->acc_c1, x_dev, k_dev, B, P, prm, c->stream));
   return DCL_OK;
 }
@@ -1009,17 +1041,20 @@ dcl_status dcl_op_attention(dcl_ctx* c, const void* qkv_dev, void* out_dev, int3
 }
 
 dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, int32_t R, int32_t V, int32_t d,
-                              int32_t* top1_dev, float* p1_dev, float* p2_dev, int32_t tile) {
+                              int32_t* top1_dev, float* p1_dev, float* p2_dev, float* entropy_dev, int32_t tile) {
   if (!c) return DCL_ERR_INVALID_ARG;
   if (!x_dev || !w_dev || !top1_dev || !p1_dev || !p2_dev || R <= 0 || V <= 1)
     return fail(c, DCL_ERR_INVALID_ARG, "bad lmhead args");
   if (tile != 0 && tile != 256 && (tile & 0xff) != kTilePair) return fail(c, DCL_ERR_INVALID_ARG, "bad tile");
   const int nblk = gemm_lmhead_blocks(V);
-  float4* part = static_cast<float4*>(dev_alloc(c, sizeof(float4) * (size_t)R * nblk));
+  // {max, sum, id, second} partials, then (with entropy_dev) the entropy partials
+  float4* part = static_cast<float4*>(dev_alloc(c, (sizeof(float4) + (entropy_dev ? 4 : 0)) * (size_t)R * nblk));
   if (!part) return fail(c, DCL_ERR_OOM, "partials allocation failed");
+  float* upart = entropy_dev ? reinterpret_cast<float*>(part + (size_t)R * nblk) : nullptr;
   GemmPlan pl;
   EpiParams ep;
   ep.out = part;
+  ep.ent_part = upart;
   const char* why = nullptr;
   if (gemm_plan(&pl, x_dev, R, d, w_dev, V, EPI_LMHEAD, ep, c->num_sms, tile, &why)) {
     dev_free_one(c, part);
@@ -1036,7 +1071,12 @@ dcl_status dcl_op_lmhead_top2(dcl_ctx* c, const void* x_dev, const void* w_dev, 
     dev_free_one(c, part);
     return fail(c, DCL_ERR_CUDA, "LM-head GEMM: %s", cudaGetErrorString(e));
   }
-  CUDA_TRY(c, lmhead_combine_launch(part, R, nblk, top1_dev, p1_dev, p2_dev, nullptr, nullptr, c->stream));
+  ConfOut co;
+  co.top1 = top1_dev;
+  co.p1 = p1_dev;
+  co.p2 = p2_dev;
+  co.ent = entropy_dev;
+  CUDA_TRY(c, lmhead_combine_launch(part, upart, R, nblk, co, nullptr, nullptr, c->stream));
   s = check_device(c);
   dev_free_one(c, part);
   return s;

@@ -164,8 +164,9 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
   } else if constexpr (EPI == EPI_LMHEAD) {
     // Online softmax over this tile's columns: running max m (= top-1 value), sum of
     // exp(z - m), argmax (lowest column on ties: columns arrive in increasing order and
-    // only a strictly larger value replaces the leader), and the second largest value.
-    float m = -INFINITY, s = 0.f, t2 = -INFINITY;
+    // only a strictly larger value replaces the leader), the second largest value, and
+    // the entropy sum u = sum exp(z - m) * y with y = (z - m) log2(e).
+    float m = -INFINITY, s = 0.f, t2 = -INFINITY, u = 0.f;
     int id = -1;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
@@ -188,10 +189,19 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
       }
       if (cm > -INFINITY) {
         const float mb = cm * kLog2e;
-        float acc = s * exp2f(m * kLog2e - mb);
+        const float d = m * kLog2e - mb;  // -inf before the first live column
+        const float al = exp2f(d);
+        float acc = s * al;
+        float accu = s > 0.f ? al * fmaf(d, s, u) : 0.f;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], kLog2e, -mb));
+        for (int i = 0; i < 32; ++i) {
+          const float y = fmaf(v[i], kLog2e, -mb);
+          const float e = exp2f(y);
+          acc += e;
+          accu = fmaf(e, fmaxf(y, -200.f), accu);  // e = 0 below -149: the term's limit 0
+        }
         s = acc;
+        u = accu;
       }
       m = cm;
       id = cid;
@@ -201,6 +211,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
       const int nblk = (N + BN - 1) / BN;
       float4* part = reinterpret_cast<float4*>(ep.out);
       part[(size_t)row * nblk + n_blk] = make_float4(m, s, __int_as_float(id), t2);
+      if (ep.ent_part) ep.ent_part[(size_t)row * nblk + n_blk] = u;
     }
   }
 }
@@ -697,7 +708,7 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
     }
   } else if constexpr (EPI == EPI_LMHEAD) {
     // Online softmax over this tile's columns (see epilogue_tile); one float4 per row.
-    float m = -INFINITY, sum = 0.f, t2 = -INFINITY;
+    float m = -INFINITY, sum = 0.f, t2 = -INFINITY, u = 0.f;
     int id = -1;
 #pragma unroll 1
     for (int c = 0; c < 256; c += 32) {
@@ -720,10 +731,19 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       }
       if (cm > -INFINITY) {
         const float mb = cm * kLog2e;
-        float acc = sum * exp2f(m * kLog2e - mb);
+        const float d = m * kLog2e - mb;  // -inf before the first live column
+        const float al = exp2f(d);
+        float acc = sum * al;
+        float accu = sum > 0.f ? al * fmaf(d, sum, u) : 0.f;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) acc += exp2f(fmaf(v[i], kLog2e, -mb));
+        for (int i = 0; i < 32; ++i) {
+          const float y = fmaf(v[i], kLog2e, -mb);
+          const float e = exp2f(y);
+          acc += e;
+          accu = fmaf(e, fmaxf(y, -200.f), accu);  // e = 0 below -149: the term's limit 0
+        }
         sum = acc;
+        u = accu;
       }
       m = cm;
       id = cid;
@@ -733,6 +753,7 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       const int nblk = (N + 255) / 256;
       float4* part = reinterpret_cast<float4*>(ep.out);
       part[(size_t)row * nblk + n_blk] = make_float4(m, sum, __int_as_float(id), t2);
+      if (ep.ent_part) ep.ent_part[(size_t)row * nblk + n_blk] = u;
     }
   }
 }

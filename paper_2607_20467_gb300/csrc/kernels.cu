@@ -189,10 +189,13 @@ __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
 }
 
 // ------------------------------------------------------------------ softmax partial merge
-// A partial is {max, sum exp(z - max), argmax id, second largest z} over some columns.
+// A partial is {max m, sum exp(z - m), argmax id, second largest z, sum exp(z - m) * y}
+// over some columns, y = (z - m) log2(e) (the last one gives the entropy:
+// H = -sum P ln P = ln 2 * (log2(sum) - u / sum)).
 struct Part {
   float m, s, t2;
   int id;
+  float u = 0.f;
 };
 
 __device__ __forceinline__ void merge(Part& a, const Part& b) {
@@ -202,7 +205,11 @@ __device__ __forceinline__ void merge(Part& a, const Part& b) {
     return;
   }
   const float m = fmaxf(a.m, b.m);
-  const float s = a.s * exp2f((a.m - m) * kLog2e) + b.s * exp2f((b.m - m) * kLog2e);
+  const float da = (a.m - m) * kLog2e, db = (b.m - m) * kLog2e;  // <= 0, finite
+  const float ea = exp2f(da), eb = exp2f(db);
+  const float s = a.s * ea + b.s * eb;
+  // re-based to the new maximum: y' = y + d for every term
+  const float u = ea * fmaf(da, a.s, a.u) + eb * fmaf(db, b.s, b.u);
   if (b.m > a.m || (b.m == a.m && b.id < a.id)) {
     a.t2 = fmaxf(b.t2, a.m);
     a.id = b.id;
@@ -211,6 +218,7 @@ __device__ __forceinline__ void merge(Part& a, const Part& b) {
   }
   a.m = m;
   a.s = s;
+  a.u = u;
 }
 
 __device__ __forceinline__ Part shfl_part(const Part& a, int off) {
@@ -219,24 +227,32 @@ __device__ __forceinline__ Part shfl_part(const Part& a, int off) {
   b.s = __shfl_xor_sync(kFull, a.s, off);
   b.t2 = __shfl_xor_sync(kFull, a.t2, off);
   b.id = __shfl_xor_sync(kFull, a.id, off);
+  b.u = __shfl_xor_sync(kFull, a.u, off);
   return b;
 }
 
-__device__ __forceinline__ void write_conf(const Part& a, int32_t* top1, float* p1, float* p2, int r) {
-  top1[r] = a.id;
+__device__ __forceinline__ void write_conf(const Part& a, const ConfOut& o, int r) {
+  o.top1[r] = a.id;
   // p1 = exp(max - max) / sum.  The sum holds the max's own term exp(0) = 1, but that
   // term is evaluated as exp2 of a rounding residual and may come out a hair below 1, so
   // the probabilities are clamped to [0, 1] and p2 <= p1.
   const float inv = 1.0f / a.s;
   const float c1 = fminf(inv, 1.0f);
-  p1[r] = c1;
-  p2[r] = a.t2 == -INFINITY ? 0.f : fminf(exp2f((a.t2 - a.m) * kLog2e) * inv, c1);
+  if (o.p1) o.p1[r] = c1;
+  if (o.p2) o.p2[r] = a.t2 == -INFINITY ? 0.f : fminf(exp2f((a.t2 - a.m) * kLog2e) * inv, c1);
+  if (o.ent || o.mode) {
+    // H = -sum P ln P >= 0 (clamped: a near-certain row can round a hair below 0)
+    const float h = fmaxf(kLn2 * (log2f(a.s) - a.u * inv), 0.f);
+    if (o.ent) o.ent[r] = h;
+    if (o.conf) o.conf[r] = o.mode ? expf(-h) : c1;
+  } else if (o.conf && o.conf != o.p1) {
+    o.conf[r] = c1;
+  }
 }
 
 // LM row `row` (of *rows_dev) is written to slot slot[row] of top1 / p1 / p2.
-__global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows, int nblk,
-                                      int32_t* __restrict__ top1, float* __restrict__ p1,
-                                      float* __restrict__ p2, const int* __restrict__ rows_dev,
+__global__ void lmhead_combine_kernel(const float4* __restrict__ part, const float* __restrict__ upart, int rows,
+                                      int nblk, ConfOut out, const int* __restrict__ rows_dev,
                                       const int* __restrict__ slot) {
   pdl_wait();
   pdl_launch_dependents();
@@ -246,12 +262,13 @@ __global__ void lmhead_combine_kernel(const float4* __restrict__ part, int rows,
   if (row >= rows) return;
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
   for (int i = lane; i < nblk; i += 32) {
-    const float4 v = part[(size_t)row * nblk + i];
-    merge(a, Part{v.x, v.y, v.w, __float_as_int(v.z)});
+    const size_t j = (size_t)row * nblk + i;
+    const float4 v = part[j];
+    merge(a, Part{v.x, v.y, v.w, __float_as_int(v.z), upart ? upart[j] : 0.f});
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) merge(a, shfl_part(a, o));
-  if (lane == 0) write_conf(a, top1, p1, p2, slot ? slot[row] : row);
+  if (lane == 0) write_conf(a, out, slot ? slot[row] : row);
 }
 
 // ------------------------------------------------------------------ DCV on one sequence
@@ -298,7 +315,8 @@ __device__ int dcv_row(int32_t* xrow, const int32_t* ids, const float* c, int pb
 __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__ p,
                                   int32_t* __restrict__ k_out, int32_t* __restrict__ steps,
                                   const int32_t* __restrict__ ids, const float* __restrict__ c,
-                                  int N, int M, DcvParams prm, int32_t* done_count) {
+                                  const float* __restrict__ ent, float* __restrict__ jpde, int N, int M,
+                                  DcvParams prm, int32_t* done_count) {
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.x;
@@ -310,6 +328,21 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
   }
   // shift the [M]-sized generation arrays so they are indexed by absolute position
   const int K = dcv_row(x + (size_t)b * T, ids + (size_t)b * M - N, c + (size_t)b * M - N, pb, T, prm);
+  if (ent) {
+    // Eq. entropy_bound of the committed set U = [p, p + K): sum_U H - max_U H
+    const float* h = ent + (size_t)b * M - N + pb;
+    float sum = 0.f, mx = 0.f;
+    for (int i = threadIdx.x; i < K; i += 32) {
+      sum += h[i];
+      mx = fmaxf(mx, h[i]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      sum += __shfl_xor_sync(kFull, sum, o);
+      mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
+    }
+    if (threadIdx.x == 0) jpde[b] += K > 1 ? sum - mx : 0.f;
+  }
   if (threadIdx.x == 0) {
     k_out[b] = K;
     p[b] = pb + K;
@@ -322,22 +355,28 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
 template <int THREADS>
 __global__ void __launch_bounds__(THREADS) accept_stats_kernel(
     const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int P, int V,
-    int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2) {
+    int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2, int mode) {
   const int pos = blockIdx.x;  // b * P + i
   const int b = pos / P, i = pos % P;
   if (i < committed[b]) return;  // committed positions are never read
   const __nv_bfloat16* row = logits + (size_t)pos * V;
-  // per-thread online (max, sum, argmax, second) over a strided slice of the row
+  // per-thread online (max, sum, argmax, second, entropy sum) over a strided slice of the row
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
   auto take = [&](float v, int col) {
     if (v > a.m) {
-      a.s = a.s * exp2f((a.m - v) * kLog2e) + 1.f;
+      const float d = (a.m - v) * kLog2e;  // -inf for the first column
+      const float e = exp2f(d);
+      a.u = a.s > 0.f ? e * fmaf(d, a.s, a.u) : 0.f;
+      a.s = a.s * e + 1.f;
       a.t2 = a.m;
       a.m = v;
       a.id = col;
     } else if (a.m != -INFINITY) {
       if (v > a.t2) a.t2 = v;
-      a.s += exp2f((v - a.m) * kLog2e);
+      const float y = (v - a.m) * kLog2e;
+      const float e = exp2f(y);
+      a.s += e;
+      a.u = fmaf(e, fmaxf(y, -200.f), a.u);  // e = 0 below -149: the term's limit 0
     }
   };
   const bool vec = ((reinterpret_cast<uintptr_t>(row) & 15) == 0);
@@ -372,7 +411,14 @@ __global__ void __launch_bounds__(THREADS) accept_stats_kernel(
     Part v = threadIdx.x < THREADS / 32 ? red[threadIdx.x] : Part{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) merge(v, shfl_part(v, o));
-    if (threadIdx.x == 0) write_conf(v, ids, c1, c2, pos);
+    if (threadIdx.x == 0) {
+      ConfOut o;
+      o.top1 = ids;
+      o.p2 = c2;
+      o.conf = c1;
+      o.mode = mode;
+      write_conf(v, o, pos);
+    }
   }
 }
 
@@ -452,22 +498,23 @@ cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloa
   }
 }
 
-cudaError_t lmhead_combine_launch(const float4* part, int rows, int nblk, int32_t* top1, float* p1,
-                                  float* p2, const int* rows_dev, const int* slot, cudaStream_t stream) {
+cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int rows, int nblk, const ConfOut& o,
+                                  const int* rows_dev, const int* slot, cudaStream_t stream) {
   const int threads = 256;
   const int blocks = (rows * 32 + threads - 1) / threads;
-  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, rows, nblk, top1, p1, p2, rows_dev, slot);
+  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, upart, rows, nblk, o, rows_dev, slot);
 }
 
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
-                              const int32_t* ids, const float* c, int batch, int N, int M,
-                              const DcvParams& prm, int32_t* done_count, cudaStream_t stream) {
-  return launch_pdl(dcv_commit_kernel, batch, 32, 0, stream, x, p, k_out, steps, ids, c, N, M, prm, done_count);
+                              const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
+                              int N, int M, const DcvParams& prm, int32_t* done_count, cudaStream_t stream) {
+  return launch_pdl(dcv_commit_kernel, batch, 32, 0, stream, x, p, k_out, steps, ids, c, ent, jpde, N, M, prm,
+                    done_count);
 }
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
-                                int V, int32_t* ids, float* c1, float* c2, cudaStream_t stream) {
-  accept_stats_kernel<512><<<B * P, 512, 0, stream>>>(logits, committed, P, V, ids, c1, c2);
+                                int V, int32_t* ids, float* c1, float* c2, int mode, cudaStream_t stream) {
+  accept_stats_kernel<512><<<B * P, 512, 0, stream>>>(logits, committed, P, V, ids, c1, c2, mode);
   return cudaGetLastError();
 }
 

@@ -26,7 +26,7 @@ def ops():
     ctx.close()
 
 
-def _guarded(seed, B, P, V, taus):
+def _guarded(seed, B, P, V, taus, confidence=0):
     d = syn.accept_inputs(seed, B, P, V, V - 1)
     bits = d["logits_bf16"]
     for _ in range(50):
@@ -35,6 +35,8 @@ def _guarded(seed, B, P, V, taus):
         for b in range(B):
             for i in range(int(d["committed"][b]), P):
                 _, c1, _ = model.confidence(z[b, i][None])
+                if confidence:
+                    c1 = decode.entropy_confidence(model.entropy(z[b, i][None]))
                 if min(abs(c1[0] - t) for t in taus) < 1e-4:
                     bad.append((b, i))
         if not bad:
@@ -45,22 +47,26 @@ def _guarded(seed, B, P, V, taus):
     raise RuntimeError("could not clear the guard band")
 
 
-@pytest.mark.parametrize("B,P,V,L,contig", [(8, 32, 4096, 16, 0), (16, 32, 1000, 32, 0), (6, 40, 3001, 7, 1),
-                                            (64, 32, 126464, 16, 0), (64, 32, 126464, 32, 1)])
-def test_accept_bit_exact(ops, B, P, V, L, contig):
+@pytest.mark.parametrize("B,P,V,L,contig,conf", [(8, 32, 4096, 16, 0, 0), (16, 32, 1000, 32, 0, 0),
+                                                 (6, 40, 3001, 7, 1, 0), (64, 32, 126464, 16, 0, 0),
+                                                 (64, 32, 126464, 32, 1, 0), (16, 32, 4096, 16, 0, 1),
+                                                 (32, 32, 126464, 16, 0, 1)])
+def test_accept_bit_exact(ops, B, P, V, L, contig, conf):
+    """conf = 1: the thresholds see exp(-H) (marginal entropy); the guard band then keeps
+    exp(-H) 1e-4 away from them (H is summed in fp32 on the GPU, fp64 in the oracle)."""
     import paper_2607_20467_gb300 as dcl
-    tc, td = 0.7, 0.9
-    d, z = _guarded(B * 131 + P + L, B, P, V, (tc, td))
+    tc, td = (0.7, 0.9) if not conf else (0.5, 0.8)
+    d, z = _guarded(B * 131 + P + L, B, P, V, (tc, td), conf)
     logits = torch.from_numpy(d["logits_bf16"].view(np.int16)).cuda().view(torch.bfloat16)
     committed = torch.from_numpy(d["committed"]).cuda()
     x = torch.from_numpy(d["x"].copy()).cuda()
     k = torch.full((B,), -1, dtype=torch.int32, device="cuda")
     cfg = dcl.decode_config(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P,
-                            contiguous_drafts=contig)
+                            contiguous_drafts=contig, confidence=conf)
     ops.accept(logits, committed, x, cfg, k)
     torch.cuda.synchronize()
     ocfg = decode.DecodeConfig(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P,
-                               contiguous_drafts=bool(contig))
+                               contiguous_drafts=bool(contig), confidence=conf)
     K, x_out, _, _, _ = accept.accept(z, d["committed"], d["x"], ocfg, L)
     assert (k.cpu().numpy() == K).all()
     assert (x.cpu().numpy() == x_out).all()
@@ -74,4 +80,7 @@ def test_accept_rejects_bad_arguments(ops):
     assert st == dcl.DCL_ERR_INVALID_ARG
     st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 5000, 100, t.data_ptr(), t.data_ptr(), cfg,
                               t.data_ptr())
+    assert st == dcl.DCL_ERR_INVALID_ARG
+    bad = dcl.decode_config(gen_len=32, confidence=2)
+    st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 32, 100, t.data_ptr(), t.data_ptr(), bad, t.data_ptr())
     assert st == dcl.DCL_ERR_INVALID_ARG

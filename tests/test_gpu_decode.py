@@ -54,8 +54,9 @@ def ctx(dcl, weights):
     c.close()
 
 
-def _predict(w):
-    return lambda tokens: model.predict(TINY, w, tokens, rows=slice(N, T), bf16_operands=True)
+def _predict(w, with_entropy=False):
+    return lambda tokens: model.predict(TINY, w, tokens, rows=slice(N, T), bf16_operands=True,
+                                        with_entropy=with_entropy)
 
 
 def test_forward_parity(dcl, ctx, weights):
@@ -95,15 +96,16 @@ def test_forward_parity(dcl, ctx, weights):
             assert err.max() <= 3e-3, (layer, err.max())
 
 
-def _check_step(x0, p0, x1, k1, ids, c1, c2, cfg, L, tol):
+def _check_step(x0, p0, x1, k1, ids, c1, c2, cfg, L, tol, conf=None):
     """Check one GPU step (x0, p0) -> (x1, p0 + k1) of one row against the oracle's
-    predictions (ids, c1, c2 over the generation positions).  Decisions with a margin
-    above tol must match the oracle; the rest must be valid outcomes.  Returns
-    (number of decisions checked exactly, number of near ties)."""
+    predictions (ids, c1, c2 over the generation positions; conf, if given, is the
+    confidence the thresholds see instead of c1).  Decisions with a margin above tol
+    must match the oracle; the rest must be valid outcomes.  Returns (number of
+    decisions checked exactly, number of near ties)."""
     full_id = np.zeros(T, np.int64)
     full_c = np.zeros(T)
     gap = np.full(T, np.inf)
-    full_id[N:], full_c[N:], gap[N:] = ids, c1, c1 - c2
+    full_id[N:], full_c[N:], gap[N:] = ids, c1 if conf is None else conf, c1 - c2
     w_eff = min(L, T - p0)
     exact = near = 0
     # K: between the prefix lengths obtained with the threshold moved by -tol / +tol
@@ -151,34 +153,44 @@ def _check_step(x0, p0, x1, k1, ids, c1, c2, cfg, L, tol):
     return exact, near
 
 
-@pytest.mark.parametrize("seed,tau_c,tau_d,L,contig", [(0, 0.7, 0.98, 32, 0), (1, 0.5, 0.8, 16, 0),
-                                                       (2, 0.9, 0.6, 8, 1), (3, 0.3, 0.95, 64, 0)])
-def test_teacher_forced_steps(dcl, ctx, weights, seed, tau_c, tau_d, L, contig):
+@pytest.mark.parametrize("seed,tau_c,tau_d,L,contig,conf", [(0, 0.7, 0.98, 32, 0, 0), (1, 0.5, 0.8, 16, 0, 0),
+                                                            (2, 0.9, 0.6, 8, 1, 0), (3, 0.3, 0.95, 64, 0, 0),
+                                                            (4, 0.3, 0.6, 32, 0, 1), (5, 0.5, 0.9, 16, 1, 1)])
+def test_teacher_forced_steps(dcl, ctx, weights, seed, tau_c, tau_d, L, contig, conf):
     """Every state of the oracle's own trajectory is loaded into the GPU, one GPU step
-    runs, and the result is checked against the oracle's decision at that state."""
+    runs, and the result is checked against the oracle's decision at that state (conf
+    = 1: the thresholds see exp(-H); the step's Eq. entropy_bound is checked too)."""
     B = 2
     prompt = syn.prompt_ids(100 + seed, B, N, TINY.mask_id)
     cfg = dcl.decode_config(tau_commit=tau_c, tau_draft=tau_d, max_window=L, gen_len=M,
-                            contiguous_drafts=contig)
+                            contiguous_drafts=contig, confidence=conf)
     ocfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=tau_d, max_window=L, gen_len=M,
-                               contiguous_drafts=bool(contig))
-    ref = decode.generate(_predict(weights), prompt, ocfg, TINY.mask_id)
+                               contiguous_drafts=bool(contig), confidence=conf)
+    ref = decode.generate(_predict(weights, with_entropy=True), prompt, ocfg, TINY.mask_id)
     ctx.set_prompt(prompt, cfg)
     p = np.full(B, N, np.int64)
     exact = near = 0
     for s, (xin, pr) in enumerate(zip(ref["inputs"], ref["preds"])):
-        ctx.set_state(xin, p.astype(np.int32))
-        k = ctx.step(return_k=True)
+        ctx.set_state(xin, p.astype(np.int32))  # also clears the entropy-bound accumulators
+        _, st, _ = ctx.generate(max_steps=1, out=False, check=False)
         x1, p1 = ctx.get_state()
+        k = p1 - p
+        bound = 0.0
         for b in range(B):
             if p[b] >= T:
                 assert k[b] == 0 and (x1[b] == xin[b]).all() and p1[b] == p[b]
                 continue
             assert p1[b] == p[b] + k[b] and 1 <= k[b] <= min(L, T - p[b])
+            c = decode.entropy_confidence(pr[3, b]) if conf else None
             e, n = _check_step(xin[b], int(p[b]), x1[b], int(k[b]), pr[0, b], pr[1, b], pr[2, b],
-                               ocfg, L, E2E_TOL)
+                               ocfg, L, E2E_TOL, conf=c)
             exact += e
             near += n
+            H = pr[3, b][int(p[b]) - N:int(p[b]) - N + int(k[b])]
+            bound += decode.jpde_bound(H)
+        # Eq. entropy_bound of the sets the GPU committed, with the oracle's entropies:
+        # each H within the end-to-end tolerance scaled by H (|dH| <= 2 H |dz|)
+        assert abs(st.jpde_bound - bound) <= 0.05 * (bound + 1.0) * max(1, int(k.max())), (s, st.jpde_bound, bound)
         p = p + ref["k"][s]
     assert exact > 0
     print(f"teacher-forced: {exact} decisions exact, {near} near ties (|margin| <= {E2E_TOL})")
@@ -224,6 +236,50 @@ def test_free_running_generation(dcl, ctx, weights, seed):
     assert (out_g == ref["x"][0, N:]).all()
     assert len(states) - 1 == ref["n_iter"]
     print(f"seed {seed}: identical trajectories ({ref['n_iter']} steps)")
+
+
+def test_forward_entropy_parity(dcl, ctx, weights):
+    """The marginal entropy from the fused LM head against the oracle (bf16 operands), and
+    the confidence the thresholds see with confidence = 1: exp(-H) <= p1."""
+    prompt = syn.prompt_ids(13, 2, N, TINY.mask_id)
+    cfg = dcl.decode_config(tau_commit=0.5, tau_draft=0.9, max_window=32, gen_len=M, confidence=1)
+    ctx.set_prompt(prompt, cfg)
+    x = np.full((2, T), TINY.mask_id, np.int32)
+    x[:, :N] = prompt
+    x[:, N + 40:] = np.random.default_rng(1).integers(0, TINY.mask_id, (2, M - 40))
+    ctx.set_state(x, np.full(2, N, np.int32))
+    p1 = torch.zeros(2 * M, device="cuda")
+    conf = torch.zeros(2 * M, device="cuda")
+    ent = torch.zeros(2 * M, device="cuda")
+    ctx.forward_debug(p1=p1, conf=conf, entropy=ent)
+    xr = x.copy()
+    xr[:, N:N + 32] = TINY.mask_id
+    worst = 0.0
+    for b in range(2):
+        sl = slice(b * M, (b + 1) * M)
+        _, p1_o, _, H_o = _predict(weights, with_entropy=True)(xr[b])
+        gH, gc, gp1 = ent[sl].cpu().numpy(), conf[sl].cpu().numpy(), p1[sl].cpu().numpy()
+        worst = max(worst, float(np.abs(gH - H_o).max()))
+        # the end-to-end logit drift (up to ~0.1 on this model) moves H by <= 2 H |dz|
+        assert (np.abs(gH - H_o) <= 0.2 * H_o + 1e-3).all()
+        assert np.abs(gc - np.exp(-gH.astype(np.float64))).max() <= 1e-6
+        assert (gc <= gp1 + 1e-6).all()
+    print(f"entropy: max |H_gpu - H| = {worst:.2e}")
+
+
+def test_entropy_bound_of_sequential_decoding_is_zero(dcl, ctx, weights):
+    prompt = syn.prompt_ids(17, 2, N, TINY.mask_id)
+    cfg = dcl.decode_config(tau_commit=1.0, tau_draft=2.0, max_window=16, gen_len=M, confidence=1)
+    ctx.set_prompt(prompt, cfg)
+    out, st, _ = ctx.generate(max_steps=2 * M)
+    assert st.steps == M and st.tokens == 2 * M and st.jpde_bound == 0.0
+    cfg = dcl.decode_config(tau_commit=0.0, tau_draft=2.0, max_window=16, gen_len=M, confidence=1)
+    ctx.set_prompt(prompt, cfg)
+    _, st, _ = ctx.generate(max_steps=2 * M)
+    assert st.steps == M // 16 and st.jpde_bound > 0.0
+    ctx.restart()  # restart clears the accumulated bound: the same run gives the same total
+    _, st2, _ = ctx.generate(max_steps=2 * M)
+    assert st2.jpde_bound == st.jpde_bound
 
 
 def test_generate_counts_and_progress(dcl, ctx, weights):

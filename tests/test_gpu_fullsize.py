@@ -23,7 +23,8 @@ A 32-layer forward of an 8B model in fp64 is out of reach of a test, so:
   * a second generation of the same prompts through dcl_generate gives the same tokens.
 The same holds with the approximate prefix key / value cache on (a step's predictions
 then come from the computed suffix; dcl_forward_debug runs the same suffix without
-recording the refresh).  The rule is restated here in a few lines of numpy; the oracle
+recording the refresh), and with the entropy confidence (the thresholds then see
+exp(-H), which dcl_forward_debug returns beside p1; exp(-H) <= p1 is checked).  The rule is restated here in a few lines of numpy; the oracle
 is not fed GPU values.
 """
 import numpy as np
@@ -38,16 +39,19 @@ pytestmark = pytest.mark.gpu
 STD = 0.02
 TAU_C, TAU_D = 0.70, 0.98
 # name: (shape, batch, prompt, generation, window, weight seed, LM-head scale, steps checked,
-#        key / value cache)
+#        key / value cache, confidence)
 CONFIGS = {
-    "llada8b": ("llada8b", 1, 256, 256, 128, 1, 12.0, None, 0),
-    "llada8b-long": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 0),
-    "llada8b-long-b8": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 24, 0),
-    "dream7b": ("dream7b", 16, 384, 512, 256, 2, 12.8, 12, 0),
+    "llada8b": ("llada8b", 1, 256, 256, 128, 1, 12.0, None, 0, 0),
+    "llada8b-long": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 0, 0),
+    "llada8b-long-b8": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 24, 0, 0),
+    "dream7b": ("dream7b", 16, 384, 512, 256, 2, 12.8, 12, 0, 0),
     # the approximate prefix key / value cache (refresh at every 32-position block)
-    "llada8b-long-cache": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 1),
-    "llada8b-long-b8-cache": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 40, 1),
-    "dream7b-cache": ("dream7b", 16, 384, 512, 256, 2, 12.8, 40, 1),
+    "llada8b-long-cache": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 1, 0),
+    "llada8b-long-b8-cache": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 40, 1, 0),
+    "dream7b-cache": ("dream7b", 16, 384, 512, 256, 2, 12.8, 40, 1, 0),
+    # the thresholds see exp(-entropy) instead of the top-1 probability
+    "llada8b-entropy": ("llada8b", 1, 256, 256, 128, 1, 12.0, 48, 0, 1),
+    "dream7b-cache-entropy": ("dream7b", 16, 384, 512, 256, 2, 12.8, 12, 1, 1),
 }
 
 
@@ -60,20 +64,21 @@ def dcl():
 
 
 def _context(dcl, name):
-    shape, B, N, M, L, seed, lm_scale, _, cache = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, _, cache, conf = CONFIGS[name]
     sh = syn.SHAPES[shape]
     stream = torch.cuda.Stream()
     ctx = dcl.Context(sh, max_batch=B, max_seq=N + M, stream=stream.cuda_stream)
     ctx.init_random_weights(seed, STD, lm_scale, 0.0)
     prompt = syn.prompt_ids(1000, B, N, sh.mask_id)
-    cfg = dcl.decode_config(tau_commit=TAU_C, tau_draft=TAU_D, max_window=L, block_len=32, gen_len=M, kv_cache=cache)
+    cfg = dcl.decode_config(tau_commit=TAU_C, tau_draft=TAU_D, max_window=L, block_len=32, gen_len=M, kv_cache=cache,
+                            confidence=conf)
     ctx.set_prompt(prompt, cfg)
     return ctx, stream, prompt
 
 
 @pytest.mark.parametrize("name,layers", [("llada8b", (0, 1)), ("dream7b", (0,))])
 def test_first_blocks_match_oracle(dcl, name, layers):
-    shape, B, N, M, L, seed, lm_scale, _, _ = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, _, _, _ = CONFIGS[name]
     sh = syn.SHAPES[shape]
     T = N + M
     ctx, stream, prompt = _context(dcl, name)
@@ -127,7 +132,7 @@ def _expected_step(x0, p0, top1, c1, N, L, mask_id):
 
 @pytest.mark.parametrize("name", list(CONFIGS))
 def test_generation_follows_acceptance_rule(dcl, name):
-    shape, B, N, M, L, seed, lm_scale, check_steps, _ = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, check_steps, _, conf_kind = CONFIGS[name]
     sh = syn.SHAPES[shape]
     T = N + M
     ctx, stream, prompt = _context(dcl, name)
@@ -135,6 +140,8 @@ def test_generation_follows_acceptance_rule(dcl, name):
         top1 = torch.zeros(B * M, dtype=torch.int32, device="cuda")
         c1 = torch.zeros(B * M, device="cuda")
         c2 = torch.zeros(B * M, device="cuda")
+        cc = torch.zeros(B * M, device="cuda")
+        ent = torch.zeros(B * M, device="cuda")
         torch.cuda.synchronize()  # the buffers exist before the context's stream writes them
         steps = 0
         while True:
@@ -142,12 +149,22 @@ def test_generation_follows_acceptance_rule(dcl, name):
             if (p0 >= T).all():
                 break
             with torch.cuda.stream(stream):
-                ctx.forward_debug(None, top1, c1, c2)
+                ctx.forward_debug(None, top1, c1, c2, cc, ent)
             ids = top1.cpu().numpy().reshape(B, M)
-            conf = c1.cpu().numpy().reshape(B, M)
+            prob1 = c1.cpu().numpy().reshape(B, M)
             conf2 = c2.cpu().numpy().reshape(B, M)
+            conf = cc.cpu().numpy().reshape(B, M)  # what the thresholds see
+            H = ent.cpu().numpy().reshape(B, M)
             assert ((ids >= 0) & (ids < sh.vocab)).all()
-            assert (conf2 <= conf).all() and (conf <= 1.0).all() and (conf2 >= 0.0).all()
+            assert (conf2 <= prob1).all() and (prob1 <= 1.0).all() and (conf2 >= 0.0).all()
+            assert (H >= 0).all() and (H <= np.log(sh.vocab) + 1e-3).all()
+            if conf_kind:
+                assert np.abs(conf - np.exp(-H.astype(np.float64))).max() <= 1e-6
+                # exp(-H) <= p1 exactly; equality for a two-way tie at the top, where the
+                # fp32 sums of 1e5 terms (relative error ~1e-6 each) may flip it by ~1e-5
+                assert (conf <= prob1 + 1e-4).all(), float((conf - prob1).max())
+            else:
+                assert (conf == prob1).all()
             k = ctx.step(return_k=True)
             x1, p1 = ctx.get_state()
             for b in range(B):
