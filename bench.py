@@ -514,6 +514,61 @@ def _traffic_from_profiles(kernel):
     return None
 
 
+# Threshold / window grids of the paper's sensitivity ablations (App. F.1: tau_c at
+# tau_d = 0.98, tau_d at tau_c = 0.70, the maximum window L), plus the tau_c grid with
+# the entropy confidence (App. F.3 alternatives).
+SWEEPS = (
+    [("tau_commit", dict(tau_c=t, tau_d=0.98, window=None, confidence=0)) for t in (0.65, 0.68, 0.70, 0.72, 0.75, 0.80)]
+    + [("tau_draft", dict(tau_c=0.70, tau_d=t, window=None, confidence=0)) for t in (0.85, 0.88, 0.90, 0.92, 0.95, 0.98)]
+    + [("window", dict(tau_c=0.70, tau_d=0.98, window=w, confidence=0)) for w in (32, 64, 96, 128)]
+    + [("tau_commit_entropy", dict(tau_c=t, tau_d=0.98, window=None, confidence=1)) for t in (0.65, 0.70, 0.80)]
+)
+
+
+def run_sweep(args):
+    """Step counts and throughput over the ablation grids: whole generations through
+    dcl_generate (host clock around it, on-device restart between runs), one JSON line
+    per grid point.  Random weights: the curves show the decoding mechanics on this
+    hardware, not the paper's accuracy / TPS (those need trained weights)."""
+    import torch
+
+    import synthetic as syn
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2607_20467_gb300 as dcl
+
+    wl = WORKLOADS[args.workload]
+    shape = syn.SHAPES[wl["shape"]]
+    B, N, M = wl["batch"], wl["n_prompt"], wl["gen"]
+    stream = torch.cuda.Stream()
+    ctx = dcl.Context(shape, max_batch=B, max_seq=N + M, stream=stream.cuda_stream)
+    ctx.init_random_weights(wl["seed"], 0.02, wl["lm_scale"], 0.0)
+    prompt = syn.prompt_ids(1000, B, N, shape.mask_id)
+    for name, pt in SWEEPS:
+        window = pt["window"] or wl["window"]
+        cfg = dcl.decode_config(tau_commit=pt["tau_c"], tau_draft=pt["tau_d"], max_window=window,
+                                block_len=wl["block"], gen_len=M, kv_cache=int(wl.get("cache", 0)),
+                                confidence=pt["confidence"])
+        ctx.set_prompt(prompt, cfg)
+        ctx.generate(max_steps=4 * M, out=False)  # warm-up (graph capture for this config)
+        secs, st = [], None
+        for _ in range(max(1, args.e2e_iters)):
+            ctx.restart()
+            torch.cuda.synchronize()
+            t = time.perf_counter()
+            _, st, _ = ctx.generate(max_steps=4 * M, out=False)
+            secs.append(time.perf_counter() - t)
+        sec = min(secs)
+        print(json.dumps({"sweep": name, "workload": args.workload, "tau_commit": pt["tau_c"],
+                          "tau_draft": pt["tau_d"], "window": window, "confidence": pt["confidence"],
+                          "steps": int(st.steps), "tokens": int(st.tokens),
+                          "steps_per_token": st.steps / max(1, st.tokens / B),
+                          "ms_per_step": 1e3 * sec / max(1, st.steps), "tokens_per_s": st.tokens / sec,
+                          "jpde_bound_per_token": st.jpde_bound / max(1, st.tokens)}), flush=True)
+    ctx.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -523,9 +578,13 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="llada8b")
     ap.add_argument("--e2e-iters", type=int, default=2)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="steps / throughput over the tau_c, tau_d, L (and entropy) grids, one JSON line each")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.sweep:
+        return run_sweep(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
