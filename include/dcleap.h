@@ -236,11 +236,14 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * segments each (S = 0: shared out over all CTA pairs) run by different pairs; rejected
  * with DCL_ERR_INVALID_ARG when the last round is full or a sharing pair would get no K
  * block; DCL_TILE_PAIR | DCL_TILE_MULTICAST clusters of two CTA pairs on consecutive
- * 256-row blocks that load each weight tile from L2 once (TMA multicast; M > 256).
+ * 256-row blocks that load each weight tile from L2 once (TMA multicast; M > 256);
+ * DCL_TILE_PAIR | DCL_TILE_HALVES whole tiles in full rounds, then every tile of a partial
+ * last round as two 256 x 128 pieces (no K split).
  * Partial sums are always combined in K order, so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
 #define DCL_TILE_STREAMK (1 << 16)
 #define DCL_TILE_MULTICAST (1 << 17)
+#define DCL_TILE_HALVES (1 << 18)
 
 /* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05
  * tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];

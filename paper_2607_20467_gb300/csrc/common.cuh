@@ -93,6 +93,7 @@ struct EpiParams {
 
 struct GemmPlan {
   CUtensorMap ta, tb;
+  CUtensorMap tbh;       // pair tiles: the weight seen in 64-row boxes (half-width pieces)
   CUtensorMap tc;        // pair tiles: the output (bf16 / fp32 boxes of 32 rows x 128 bytes)
   CUtensorMap tw;        // pair tiles with partials: the fp32 workspace [rows][256]
   CUtensorMap tv;        // QKV with ep.vt_heads > 0: v^T boxes [64 channels][32 tokens]
@@ -108,6 +109,7 @@ struct GemmPlan {
   size_t smem = 0;
   int splits = 1;          // split-K factor (pair tiles only)
   int streamk = 0;         // > 0: left-over pair tiles shared out by K over this many pairs
+  int halves = 0;          // 1: the left-over pair tiles run as two 256 x 128 pieces
   int ws_slots = 0;        // stream-K partial slots per left-over tile
   size_t flags_needed = 0; // ints of zero-initialised split counters the launch needs
   size_t ws_needed = 0;    // floats of workspace for split-K partials
@@ -125,6 +127,7 @@ struct GemmPlan {
 constexpr int kTilePair = 2;
 constexpr int kTileStreamK = 1 << 16;
 constexpr int kTileMulticast = 1 << 17;  // with kTilePair: clusters of two pairs sharing W tiles
+constexpr int kTileHalves = 1 << 18;     // with kTilePair: left-over tiles as two half-width pieces
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
                       int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
 // Attach the zero-initialised counters (>= flags_needed ints) and the workspace

@@ -595,19 +595,21 @@ __device__ __forceinline__ void store_bf16_box(const Src& s, Stage& o, const CUt
   o.issue(tmc, b, x, o.row0, false);
 }
 
-// The fused epilogues of a 256 x 256 pair tile, for one warp's 32-row band of one CTA
-// half.  All tcgen05.ld run warp-uniformly.
+// The fused epilogues of a pair tile (256 rows x W columns: W = 256, or 128 for piece
+// `piece` of a tile cut in two), for one warp's 32-row band of one CTA half.  A piece
+// covers output columns [n_blk * 256 + piece * W, + W); with SwiGLU it holds W/2 gate
+// columns and the W/2 matching up columns.  All tcgen05.ld run warp-uniformly.
 template <int EPI>
 __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUtensorMap* tmc, const CUtensorMap* tmv,
                                               const CUtensorMap* tmk, int row, int n_blk, int M, int N,
-                                              const EpiParams& ep) {
-  const int n0 = n_blk * 256;
+                                              const EpiParams& ep, int piece = 0, int W = 256) {
+  const int n0 = n_blk * 256 + piece * W;
   if constexpr (EPI == EPI_BF16) {
 #pragma unroll 1
-    for (int c = 0; c < 256 && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
+    for (int c = 0; c < W && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
   } else if constexpr (EPI == EPI_RESID_F32) {
 #pragma unroll 1
-    for (int c = 0; c < 256; c += 32) {
+    for (int c = 0; c < W; c += 32) {
       float v[32];
       src_cols(s, c, v);
       if (n0 + c >= N) break;
@@ -629,7 +631,7 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       const float* cs = ep.rope_cos + (size_t)pos * half;
       const float* sn = ep.rope_sin + (size_t)pos * half;
 #pragma unroll 1
-      for (int hb = 0; hb < 256; hb += hd) {
+      for (int hb = 0; hb < W; hb += hd) {
         // rotate-half pairs (j, j + half): hd 128 fills a box with rotated columns
         // [hb, hb + 64) and one with [hb + 64, hb + 128); hd 64 fills one box [hb, hb + 64)
         uint32_t b0, b1;
@@ -673,7 +675,7 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       // v columns leave transposed, as the attention's K-major operand: boxes of 64
       // channels x 32 tokens of vt [batch * G][hd][T]
 #pragma unroll 1
-      for (int c = 0; c < 256 && n0 + c < N; c += 64) {
+      for (int c = 0; c < W && n0 + c < N; c += 64) {
         const int cv = n0 + c - ep.rope_cols, g = cv / ep.head_dim, d0 = cv - g * ep.head_dim;
         const uint32_t b = o.acquire();
 #pragma unroll 1
@@ -687,24 +689,25 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       }
     } else {
 #pragma unroll 1
-      for (int c = 0; c < 256 && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
+      for (int c = 0; c < W && n0 + c < N; c += 64) store_bf16_box(s, o, tmc, c, n0 + c);
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
-    // columns [0, 128) of the tile are gate rows, [128, 256) the matching up rows
+    // columns [0, W/2) of the tile are gate rows, [W/2, W) the matching up rows
+    const int G2 = W >> 1;
 #pragma unroll 1
-    for (int c = 0; c < 128; c += 64) {
+    for (int c = 0; c < G2; c += 64) {
       const uint32_t b = o.acquire();
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
         float g[32], u[32];
         src_cols(s, c + 32 * h, g);
-        src_cols(s, 128 + c + 32 * h, u);
+        src_cols(s, G2 + c + 32 * h, u);
         float v[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = g[i] / (1.0f + __expf(-g[i])) * u[i];
         stage_bf16(b, o.lane, h, v);
       }
-      o.issue(tmc, b, n_blk * 128 + c, o.row0, false);
+      o.issue(tmc, b, n_blk * 128 + piece * G2 + c, o.row0, false);
     }
   } else if constexpr (EPI == EPI_LMHEAD) {
     // Online softmax over this tile's columns (see epilogue_tile); one float4 per row.
@@ -868,15 +871,39 @@ enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3 };
 struct Sched {
   int tiles, ku, C, splits;
   int streamk;  // 0: off; else the number of pairs (<= C) that share the left-over tiles
+  int halves;   // 1: the tiles of a partial last round run as two 256 x 128 pieces each
 };
 struct Item {
   int t, ku0, ku1, kind;
+  int piece = 0, width = 256;  // columns [piece * width, + width) of tile t
   int sp;     // IT_SPLIT: split index
   int rel;    // IT_PART / IT_LAST: stream-K tile index (0..R-1)
   int slot;   // IT_PART: partial slot; IT_LAST: number of earlier segments
 };
 
 __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& it) {
+  it.piece = 0;
+  it.width = 256;
+  if (s.halves) {
+    // full rounds of whole tiles, then every left-over tile as two half-width pieces on
+    // two consecutive pairs (same rows of A, neighbouring rows of W): the last round
+    // takes half as long and the pieces need no combination
+    const int full = s.tiles / s.C;
+    it.ku0 = 0;
+    it.ku1 = s.ku;
+    it.kind = IT_PLAIN;
+    if (idx < full) {
+      it.t = c + idx * s.C;
+      return true;
+    }
+    const int first = full * s.C;
+    const long w = (long)c + (long)(idx - full) * s.C;
+    if (w >= 2L * (s.tiles - first)) return false;
+    it.t = first + (int)(w >> 1);
+    it.piece = (int)(w & 1);
+    it.width = 128;
+    return true;
+  }
   if (s.splits > 1) {
     const long w = (long)c + (long)idx * s.C;
     if (w >= (long)s.tiles * s.splits) return false;
@@ -951,10 +978,10 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
 template <int EPI, bool MC>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
-                    const __grid_constant__ CUtensorMap tmc, const __grid_constant__ CUtensorMap tmw,
-                    const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmk, int M,
-                    int N, int K, EpiParams ep, int splits, int streamk, int ws_slots, int* flags, float* ws,
-                    int* err) {
+                    const __grid_constant__ CUtensorMap tmbh, const __grid_constant__ CUtensorMap tmc,
+                    const __grid_constant__ CUtensorMap tmw, const __grid_constant__ CUtensorMap tmv,
+                    const __grid_constant__ CUtensorMap tmk, int M, int N, int K, EpiParams ep, int splits,
+                    int streamk, int halves, int ws_slots, int* flags, float* ws, int* err) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -998,6 +1025,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_mbar_init();
     prefetch_tmap(&tma);
     prefetch_tmap(&tmb);
+    prefetch_tmap(&tmbh);
   }
   if (warp == 1) tmem_alloc_pair(holder, TMEM2_COLS);
   tc_fence_before();
@@ -1017,6 +1045,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   sc.C = gridDim.x / CL;
   sc.splits = splits;
   sc.streamk = streamk;
+  sc.halves = halves;
   // item tile -> (m block, n block); MC: pair pr takes the pr-th 256-row half of the unit
   auto tile_mn = [&](int t, int& m_blk, int& n_blk) {
     m_blk = MC ? 2 * (t % num_mh) + (int)pr : t % num_mh;
@@ -1034,7 +1063,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         int m_blk, n_blk;
         tile_mn(it.t, m_blk, n_blk);
         const int kb0 = it.ku0 * KA2, kb1 = it.ku1 * KA2;
-        const int wrow = n_blk * 256 + (int)rank * 128;  // this CTA's half of the weight tile
+        // this CTA's half of the weight rows of the item: 128 rows of a whole tile, or 64
+        // of a half-width piece (SwiGLU: the gate rows in the leader, the matching up rows
+        // in the peer, as for whole tiles)
+        const bool hw = it.width != 256;
+        const int wrow = n_blk * 256 +
+                         (!hw ? (int)rank * 128
+                              : (EPI == EPI_SWIGLU ? (int)rank * 128 + it.piece * 64 : it.piece * 128 + (int)rank * 64));
+        const CUtensorMap* tw_map = hw ? &tmbh : &tmb;
+        const uint32_t stage_tx = 2u * (uint32_t)(hw ? A2_STAGE_BYTES + B2_STAGE_BYTES / 2 : STAGE2_BYTES);
         for (int kb = kb0; kb < kb1 && kb < kb0 + kPrefetchAhead; ++kb) tma_prefetch_l2(&tmb, kb * BK, wrow);
         for (int kb = kb0; kb < kb1; kb += KA2) {
           for (int a = 0; a < KA2; ++a)
@@ -1052,11 +1089,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                 wrow + (int)pr * 64, full_leader, (uint16_t)((1u << crank) | (1u << (crank ^ 2u))));
           } else {
             const uint32_t full_leader = mapa_shared(full0 + 8 * stage, lead);
-            if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, 2 * STAGE2_BYTES);
+            if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, stage_tx);
             for (int a = 0; a < KA2; ++a) {
               tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, &tma, (kb + a) * BK,
                                m_blk * 256 + (int)rank * 128, full_leader);
-              tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, &tmb, (kb + a) * BK, wrow,
+              tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, tw_map, (kb + a) * BK, wrow,
                                full_leader);
             }
           }
@@ -1074,13 +1111,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
       // ------------------------------------------------ MMA issuer (leader CTA only)
-      constexpr uint32_t idesc = make_idesc(256, 256);
+      constexpr uint32_t idesc_full = make_idesc(256, 256);
+      constexpr uint32_t idesc_half = make_idesc(256, 128);
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
       Item it;
       for (int idx = 0; ok && next_item(idx, sc, cluster, it); ++idx) {
         const int kb0 = it.ku0 * KA2, kb1 = it.ku1 * KA2;
+        const uint32_t idesc = it.width == 256 ? idesc_full : idesc_half;
         const int ab = idx & 1;
         const uint32_t aph = (uint32_t)(idx >> 1) & 1u;
         if (!mbar_wait(tempty0 + 8 * ab, aph ^ 1u, abort_flag)) {
@@ -1153,7 +1192,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (phantom) {
         // nothing to store
       } else if (it.kind == IT_PLAIN) {
-        epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
+        epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep, it.piece, it.width);
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
         int* flag = flags + t * 2 + rank;
@@ -1319,8 +1358,8 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kern, p.ta, p.tb, p.tc, p.tw, p.tv, p.tk, p.M, p.N, p.K, p.ep, p.splits, p.streamk,
-                            p.ws_slots, p.flags, p.ws, err);
+  return cudaLaunchKernelEx(&cfg, kern, p.ta, p.tb, p.tbh, p.tc, p.tw, p.tv, p.tk, p.M, p.N, p.K, p.ep, p.splits,
+                            p.streamk, p.halves, p.ws_slots, p.flags, p.ws, err);
 }
 
 // Clusters of four CTA-pair CTAs that can be resident at once (0 if unknown).
@@ -1478,14 +1517,32 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     }
     mc = 1;
   }
+  // Half-width tail (on request, kTileHalves): whole tiles in full rounds, then each
+  // tile of a partial last round as two 256 x 128 pieces on two pairs, with no partial
+  // sums to combine (each output is still one MMA chain over all of K, so results are
+  // bit-identical to whole tiles).  Measured, a piece takes as long per K block as a
+  // whole tile: the six-stage operand ring, not the tensor core, sets the pace of a
+  // K block (about 1.7 us of load latency under full load over six 32 KB stages), so the
+  // planner does not pick it.
+  int halves = 0;
+  if (cg == 2 && pair_forced && (tile & kTileHalves)) {
+    if (streamk != 0 || mc != 0 || epi == EPI_LMHEAD || forced_splits > 1) {
+      *why = "gemm: half-width tail tiles exclude stream-K, multicast, K splits and the LM-head epilogue";
+      return cudaErrorInvalidValue;
+    }
+    halves = 1;
+    splits = 1;
+  }
   // each CTA loads 128 rows of A; of W a one-CTA tile loads bn rows, a pair CTA 128 (MC: 64)
   if (!encode_kmajor(&plan->ta, A, M, K, BM) ||
-      !encode_kmajor(&plan->tb, W, N, K, cg == 2 ? (mc ? 64 : 128) : bn)) {
+      !encode_kmajor(&plan->tb, W, N, K, cg == 2 ? (mc ? 64 : 128) : bn) ||
+      (cg == 2 && !encode_kmajor(&plan->tbh, W, N, K, 64))) {
     *why = "gemm: cuTensorMapEncodeTiled failed";
     return cudaErrorInvalidValue;
   }
   plan->splits = splits;
   plan->streamk = streamk;
+  plan->halves = halves;
   plan->ws_slots = 0;
   plan->flags_needed = 0;
   plan->ws_needed = 0;
@@ -1516,7 +1573,9 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
     plan->n_tiles = (int)pair_tiles;
     // stream-K: all pairs when there are plain rounds, else only the sharing ones (the
     // kernel derives the round stride from the grid)
-    const long items = streamk ? (pair_tiles >= pairs ? pairs : streamk) : pair_tiles * splits;
+    const long items = streamk  ? (pair_tiles >= pairs ? pairs : streamk)
+                       : halves ? (pair_tiles >= pairs ? pairs : std::min<long>(pairs, 2 * pair_tiles))
+                                : pair_tiles * splits;
     plan->grid = 2 * (int)(items < pairs ? items : pairs);
     if (mc) {  // units of two 256-row blocks, one per cluster of four
       const long units = (long)((((M + 255) / 256) + 1) / 2) * ((N + 255) / 256) * splits;

@@ -62,12 +62,13 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
-PAIR, SK, MC = 2, 1 << 16, 1 << 17
+PAIR, SK, MC, HALF = 2, 1 << 16, 1 << 17, 1 << 18
 # auto, one-CTA 128 / 256 columns, CTA pair (library's K schedule), CTA pair unsplit,
 # CTA pair with 2 / 3 K splits, CTA pair with stream-K over all pairs / in K halves,
-# clusters of two pairs sharing weight tiles (unsplit / 2 K splits)
+# clusters of two pairs sharing weight tiles (unsplit / 2 K splits), left-over tiles as
+# two half-width pieces
 TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK, PAIR | SK | (2 << 8),
-         PAIR | MC | (1 << 8), PAIR | MC | (2 << 8)]
+         PAIR | MC | (1 << 8), PAIR | MC | (2 << 8), PAIR | HALF]
 
 
 def _splits(tile):
@@ -156,6 +157,24 @@ def test_linear_split_k_is_deterministic(ops, tile, mode):
         outs.append(o)
     torch.cuda.synchronize()
     assert torch.equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("M,N,K,mode", [(512, 12288, 4096, 0), (512, 4096, 4096, 1), (300, 1280, 4096, 0),
+                                        (512, 4096, 12288, 1), (1, 128, 64, 0)])
+def test_linear_half_pieces_equal_whole_tiles(ops, M, N, K, mode):
+    """Half-width pieces accumulate each output over all of K in the same order as whole
+    tiles: the same bits (whole tiles forced by an unsplit pair tile), run after run."""
+    rng = np.random.default_rng(M + 3 * N + K)
+    a = _bf16(rng.normal(0, 1, (M, K)).astype(np.float32))
+    w = _bf16(rng.normal(0, K ** -0.5, (N, K)).astype(np.float32))
+    h0 = torch.from_numpy(rng.normal(0, 2, (M, N)).astype(np.float32)).cuda()
+    outs = []
+    for tile in (PAIR | (1 << 8), PAIR | HALF, PAIR | HALF):
+        o = h0.clone() if mode == 1 else torch.zeros(M, N, dtype=torch.bfloat16, device="cuda")
+        ops.op_linear(a, w, o, mode=mode, tile=tile)
+        outs.append(o)
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
 
 
 # ------------------------------------------------------------------ attention
