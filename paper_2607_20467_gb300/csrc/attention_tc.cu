@@ -13,9 +13,11 @@
 // O / l leaves through TMA.  Two passes cost one more Q K^T than an online softmax but
 // need no rescaling of the TMEM accumulator and give the exact row maximum.
 //
-// Roles (192 threads): warp 0 lane 0 TMA producer (Q once, then K / V^T blocks through a
+// Roles (320 threads): warp 0 lane 0 TMA producer (Q once, then K / V^T blocks through a
 // 2-stage ring in the order the MMAs consume them); warp 1 allocates TMEM and its lane 0
-// issues the MMAs; warps 2..5 run the softmax and the epilogue.  P is double-buffered so
+// issues the MMAs; warps 2..9 run the softmax and the epilogue, two warps per 32-row
+// band (TMEM lane quarter), each on one 64-column half of every S block: the row maxima
+// and sums of the two halves are combined through shared memory.  P is double-buffered so
 // that the softmax of block j + 1 overlaps the P V MMAs of block j.  V enters as V^T (a
 // K-major operand, kv contiguous), written by v_transpose_kernel from the q|k|v buffer.
 // Every wait is bounded (DERR_WAIT_TIMEOUT).
@@ -25,7 +27,8 @@
 namespace dcl {
 namespace {
 
-constexpr int AT_THREADS = 192;
+constexpr int AT_THREADS = 320;
+constexpr int AT_SOFTMAX = 8;  // softmax warps (2 .. 9)
 constexpr int AT_STAGES = 2;
 constexpr int AT_BOX = 128 * 128;  // one 128-row x 128-byte swizzle box
 
@@ -37,7 +40,8 @@ struct AttnCfg {
   static constexpr int VBOX = HD * 128;                // one V^T box: [HD rows][64 kv]
   static constexpr int P_BYTES = 2 * 2 * 2 * AT_BOX;   // 2 buffers of P_hi and P_lo, [128][128] each
   static constexpr int BARS = 256;
-  static constexpr size_t SMEM = 1024 + (size_t)Q_BYTES + AT_STAGES * STAGE_BYTES + P_BYTES + BARS;
+  static constexpr int RED = 2 * 128 * 4;              // per-half row maxima / sums [2][128]
+  static constexpr size_t SMEM = 1024 + (size_t)Q_BYTES + AT_STAGES * STAGE_BYTES + P_BYTES + BARS + RED;
   static constexpr uint32_t TMEM_COLS = 512;           // S double buffer (2 x 128) + O (HD)
 };
 
@@ -95,6 +99,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   const uint32_t holder = drain + 8;
   volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
+  float* red = reinterpret_cast<float*>(smem + (bars + C::BARS - base));  // [2][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -109,10 +114,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full0 + 8 * i, 1);
-      mbar_init(s_empty0 + 8 * i, 4);  // the 4 softmax warps
+      mbar_init(s_empty0 + 8 * i, AT_SOFTMAX);  // the softmax warps
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(p_full0 + 8 * i, 4);
+      mbar_init(p_full0 + 8 * i, AT_SOFTMAX);
       mbar_init(p_empty0 + 8 * i, 1);
     }
     mbar_init(o_full, 1);
@@ -271,10 +276,13 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       mbar_wait(drain, 0, &no_abort);
     }
   } else {
-    // ------------------------------------------------ softmax + epilogue (warps 2..5)
+    // ------------------------------------------------ softmax + epilogue (warps 2..9)
     const int q = warp & 3;             // TMEM lane quarter = 32-row band
+    const int hs = (warp - 2) >> 2;     // which 64-column half of each S block
+    const int co = 64 * hs;
     const int r = q * 32 + lane;        // query row within the tile
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    auto softmax_bar = []() { asm volatile("bar.sync 1, %0;" ::"n"(AT_SOFTMAX * 32) : "memory"); };
     const float scale2 = kLog2e * rsqrtf((float)HD);
     bool ok = true;
     int si = 0;
@@ -285,23 +293,23 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int valid = T - j * 128;
-      uint32_t v[4][32];  // the whole 128-column row, one wait
+      const int valid = T - j * 128 - co;  // live columns of this half
+      uint32_t v[2][32];  // this half of the row, one wait
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * c), v[c]);
+      for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + co + 32 * c), v[c]);
       tmem_ld_wait();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(s_empty0 + 8 * sb);
       float mm = -INFINITY;
-      if (valid >= 128) {
+      if (valid >= 64) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < 2; ++c)
 #pragma unroll
           for (int e = 0; e < 32; ++e) mm = fmaxf(mm, f32(v[c][e]));
       } else {
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < 2; ++c)
 #pragma unroll
           for (int e = 0; e < 32; ++e)
             if (32 * c + e < valid) mm = fmaxf(mm, f32(v[c][e]));
@@ -309,6 +317,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       m = fmaxf(m, mm * scale2);
       ++si;
     }
+    // the row maximum over both halves (every softmax warp reaches this point: a failed
+    // wait above is warp-uniform and skips no barrier, since ok stays false after it)
+    red[hs * 128 + r] = m;
+    softmax_bar();
+    m = fmaxf(red[r], red[128 + r]);
+    softmax_bar();  // every read is done before the sums reuse the slots
     float l = 0.f;
     for (int j = 0; ok && j < nb; ++j) {  // pass 2: P = exp2(s - m), l, P_hi / P_lo
       const int sb = si & 1, pb = j & 1;
@@ -320,11 +334,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       const int valid = T - j * 128;
       const uint32_t pbase = sP + (uint32_t)pb * 4 * AT_BOX;
       uint32_t v[2][32];
-      tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128), v[0]);
+      tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + co), v[0]);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 2 * hs; c < 2 * hs + 2; ++c) {
         tmem_ld_wait();
-        if (c + 1 < 4) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * (c + 1)), v[(c + 1) & 1]);
+        if (c + 1 < 2 * hs + 2) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * (c + 1)), v[(c + 1) & 1]);
         // P = hi + lo: hi = P with its low 16 bits cleared (a bf16 value), lo = P - hi
         // (exact) rounded to bf16, so P is carried to about 2^-16 relative
         uint32_t hb[32];
@@ -358,18 +372,21 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       ++si;
     }
+    // the row sum over both halves, half 0 + half 1 (a fixed order)
+    red[hs * 128 + r] = l;
+    softmax_bar();
+    l = red[r] + red[128 + r];
     if (ok) ok = mbar_wait(o_full, 0, abort_flag);
     ok = __all_sync(0xffffffffu, ok);
     if (ok) {
-      // epilogue: O / l -> bf16 -> TMA store (staged in this warp's part of the P
-      // buffers, free once every PV MMA has completed)
+      // epilogue: O / l -> bf16 -> TMA store, each warp one 64-column box of its band
+      // (staged in the P buffers, free once every PV MMA has completed)
       tc_fence_after();
       const float inv = 1.0f / l;
       const int row0 = qt * 128 + q * 32;
-      const uint32_t stg = sP + (uint32_t)q * (C::KB * 32 * 128);
 #pragma unroll 1
-      for (int c = 0; c < HD; c += 64) {
-        const uint32_t bx = stg + (uint32_t)(c >> 6) * (32 * 128);
+      for (int c = co; c < HD; c += 128) {
+        const uint32_t bx = sP + (uint32_t)((q * 2 + hs) * (32 * 128));
 #pragma unroll 1
         for (int hh = 0; hh < 2; ++hh) {
           uint32_t v[32];
