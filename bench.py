@@ -295,6 +295,24 @@ def _config(wl, args):
             "l2": "no flush needed: every step streams all weights (>> 129 MB L2)"}
 
 
+def _allreduce(v, op, dist, device):
+    """max or sum of a float over the ranks of `dist` (the value itself without one)."""
+    if dist is None:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def aggregate_replicas(ms, tokens, e2e_s, dist=None, device="cuda"):
+    """Whole-job numbers of N independent replicas (one per GPU, no data-path exchange):
+    the slowest rank's timed window (ms), the tokens every rank committed in it, and the
+    slowest rank's end-to-end generation time (s).  Timing only: the ranks share no data."""
+    return (_allreduce(ms, "max", dist, device), _allreduce(tokens, "sum", dist, device),
+            _allreduce(e2e_s, "max", dist, device))
+
+
 # ---------------------------------------------------------------------- our arm
 def run_ours(args):
     import torch
@@ -393,29 +411,13 @@ def run_ours(args):
         e2e_steps.append(int(st.steps))
         assert st.done == 1
 
-    # aggregate over ranks (timing only: max time, summed tokens)
-    def allmax(v):
-        if not dist:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
-    def allsum(v):
-        if not dist:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        return float(t.item())
-
-    ms_max = allmax(ms)
     # every step costs the same (full recompute), so a timed window of K steps is credited
     # the trajectory's average rate, B*M tokens per S steps: the window need not cover
     # whole generations for the value to equal whole-generation throughput
     per_step = B * M / S
     # (cached steps differ in cost: the window is credited the tokens it actually committed)
-    tokens_all = allsum(tokens if cached else args.steps * per_step)
-    e2e_mean = allmax(statistics.mean(e2e_s))
+    ms_max, tokens_all, e2e_mean = aggregate_replicas(ms, tokens if cached else args.steps * per_step,
+                                                      statistics.mean(e2e_s), dist, "cuda")
     peaks = _peaks()
     if cached:
         # the cached step's work varies (refresh or suffix): the trajectory's mean
