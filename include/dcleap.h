@@ -292,6 +292,14 @@ typedef enum {
   DCL_K_ROWPLAN = 11     /* the rows the step computes (full recompute or cache suffix) */
 } dcl_kernel_kind;
 
+/* Fault-handling self-test (the device waits of the GEMM and attention pipelines are
+ * bounded; this exercises that path without a fault): a one-thread kernel waits on
+ * something nothing signals - which = 0: a fresh mbarrier, 1: a zero counter in global
+ * memory - through the same bounded helpers, gives up after the 2 s wait limit and
+ * records the timeout.  Returns DCL_ERR_TIMEOUT (the expected outcome) and leaves the
+ * context usable; INVALID_ARG for another `which`.  Synchronises. */
+dcl_status dcl_selftest_wait_timeout(dcl_ctx* ctx, int32_t which);
+
 /* enable = 1 re-captures the step graph with a pair of timing events (CUDA event record
  * nodes on the context stream) around every kernel; 0 restores the plain graph.
  * Takes effect at once if a prompt is set, else at the next dcl_set_prompt. */

@@ -82,6 +82,7 @@ SIGNATURES = {
     "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I]),
     "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _I]),
     "dcl_op_generate": (_I, [_P, _P, ctypes.c_uint64, _I, ctypes.c_int64, ctypes.c_int64, _F, _F]),
+    "dcl_selftest_wait_timeout": (_I, [_P, _I]),
     "dcl_set_profiling": (_I, [_P, _I]),
     "dcl_profile_last_step": (_I, [_P, _P, _P, _I, _P]),
     "dcl_last_error": (ctypes.c_char_p, [_P]),
@@ -275,6 +276,10 @@ class Context:
 
     def op_generate(self, dst, seed, tid, start, count, std, mean=0.0):
         self._check(self._L.dcl_op_generate(self.ptr, _ptr(dst), seed, tid, start, count, std, mean))
+
+    def selftest_wait_timeout(self, which):
+        """Status of the bounded-wait self-test (DCL_ERR_TIMEOUT is the expected one)."""
+        return self._L.dcl_selftest_wait_timeout(self.ptr, which)
 
     def set_profiling(self, enable):
         self._check(self._L.dcl_set_profiling(self.ptr, int(bool(enable))))

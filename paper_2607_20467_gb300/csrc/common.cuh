@@ -140,6 +140,8 @@ cudaError_t gemm_bind_scratch(GemmPlan* plan, int* flags, float* ws);
 // (plan unchanged) when the shape does not allow it (T a multiple of 32 is needed).
 bool gemm_fuse_kv(GemmPlan* plan, void* kbuf, void* vt, int batch, int T, int H, int G, int hd, int Tp);
 cudaError_t gemm_launch(const GemmPlan& plan, int* err, cudaStream_t stream);
+// Bounded-wait self-test (which = 0: an mbarrier, 1: a global counter; flag = a zero int).
+cudaError_t wait_selftest_launch(int which, const int* flag, int* err, cudaStream_t stream);
 int gemm_lmhead_blocks(int vocab);  // number of 256-column partial records per row
 // cuTensorMapEncodeTiled through the runtime's driver entry point: dims / box in elements
 // (innermost first), strides in bytes for dimensions 1 .. rank-1; out-of-range elements

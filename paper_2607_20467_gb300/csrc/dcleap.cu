@@ -1094,6 +1094,22 @@ dcl_status dcl_op_generate(dcl_ctx* c, void* dst_dev, uint64_t seed, int32_t tid
   return DCL_OK;
 }
 
+dcl_status dcl_selftest_wait_timeout(dcl_ctx* c, int32_t which) {
+  if (!c) return DCL_ERR_INVALID_ARG;
+  if (which != 0 && which != 1) return fail(c, DCL_ERR_INVALID_ARG, "which must be 0 or 1");
+  int* flag = static_cast<int*>(dev_alloc(c, sizeof(int)));
+  if (!flag) return fail(c, DCL_ERR_OOM, "flag allocation failed");
+  cudaError_t e = cudaMemsetAsync(flag, 0, sizeof(int), c->stream);
+  if (e == cudaSuccess) e = wait_selftest_launch(which, flag, c->derr, c->stream);
+  if (e != cudaSuccess) {
+    dev_free_one(c, flag);
+    return fail(c, DCL_ERR_CUDA, "self-test launch: %s", cudaGetErrorString(e));
+  }
+  const dcl_status s = check_device(c);
+  dev_free_one(c, flag);
+  return s;
+}
+
 dcl_status dcl_set_profiling(dcl_ctx* c, int32_t enable) {
   if (!c) return DCL_ERR_INVALID_ARG;
   c->profiling = enable != 0;

@@ -1649,6 +1649,32 @@ cudaError_t gemm_bind_scratch(GemmPlan* p, int* flags, float* ws) {
   return cudaSuccess;
 }
 
+// Fault-handling self-test: one thread waits, through the same bounded helpers the
+// pipelines use, on something nothing will ever signal - a fresh mbarrier (which = 0) or
+// a zero counter in global memory (which = 1) - gives up after the wait limit, records
+// DERR_WAIT_TIMEOUT and returns, leaving the context usable.
+__global__ void wait_selftest_kernel(int which, const int* flag, int* err) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  bool ok;
+  if (which == 0) {
+    const uint32_t b = smem_u32(&bar);
+    mbar_init(b, 1);
+    fence_mbar_init();
+    ok = mbar_wait(b, 0, &abort_flag);  // phase 0 completes only after an arrival
+  } else {
+    ok = wait_flag_geq(flag, 1, &abort_flag);
+  }
+  if (!ok) report_error(err, DERR_WAIT_TIMEOUT);
+}
+
+cudaError_t wait_selftest_launch(int which, const int* flag, int* err, cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 32, 0, stream>>>(which, flag, err);
+  return cudaGetLastError();
+}
+
 cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
   if ((p.flags_needed && !p.flags) || (p.ws_needed && !p.ws)) return cudaErrorInvalidValue;
   if (p.cg == 2 && p.mc) {
