@@ -238,12 +238,16 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * block; DCL_TILE_PAIR | DCL_TILE_MULTICAST clusters of two CTA pairs on consecutive
  * 256-row blocks that load each weight tile from L2 once (TMA multicast; M > 256);
  * DCL_TILE_PAIR | DCL_TILE_HALVES whole tiles in full rounds, then every tile of a partial
- * last round as two 256 x 128 pieces (no K split).
+ * last round as two 256 x 128 pieces (no K split); DCL_TILE_PAIR | DCL_TILE_DSMEM clusters
+ * of two CTA pairs: whole tiles in full rounds, then every left-over tile split by K over
+ * one cluster's pairs, the upper half's fp32 sum added to the lower half's through
+ * distributed shared memory (K >= 128, at most one left-over tile per cluster).
  * Partial sums are always combined in K order, so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
 #define DCL_TILE_STREAMK (1 << 16)
 #define DCL_TILE_MULTICAST (1 << 17)
 #define DCL_TILE_HALVES (1 << 18)
+#define DCL_TILE_DSMEM (1 << 19)
 
 /* The dense contractions of the forward (Sec. 3.3 step (ii)): out = a @ w^T on the tcgen05
  * tensor cores.  a_dev bf16 [M][K], w_dev bf16 [N][K];

@@ -76,8 +76,9 @@ enum Epilogue : int {
 struct EpiParams {
   void* out = nullptr;
   int ldo = 0;
-  const float* rope_cos = nullptr;  // [T][head_dim/2]
+  const float* rope_cos = nullptr;  // [head_dim/2][rope_T], positions contiguous
   const float* rope_sin = nullptr;
+  int rope_T = 0;                   // positions in the tables (row length)
   int rope_cols = 0;
   int head_dim = 0;
   int seq_T = 1;                    // rows per sequence (position = row % seq_T)
@@ -110,6 +111,7 @@ struct GemmPlan {
   int splits = 1;          // split-K factor (pair tiles only)
   int streamk = 0;         // > 0: left-over pair tiles shared out by K over this many pairs
   int halves = 0;          // 1: the left-over pair tiles run as two 256 x 128 pieces
+  int ds = 0;              // 1: four-CTA clusters, left-over tiles split by K over two pairs (DSMEM sum)
   int ws_slots = 0;        // stream-K partial slots per left-over tile
   size_t flags_needed = 0; // ints of zero-initialised split counters the launch needs
   size_t ws_needed = 0;    // floats of workspace for split-K partials
@@ -128,6 +130,7 @@ constexpr int kTilePair = 2;
 constexpr int kTileStreamK = 1 << 16;
 constexpr int kTileMulticast = 1 << 17;  // with kTilePair: clusters of two pairs sharing W tiles
 constexpr int kTileHalves = 1 << 18;     // with kTilePair: left-over tiles as two half-width pieces
+constexpr int kTileDsmem = 1 << 19;      // with kTilePair: left-over tiles split by K over a cluster's pairs
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
                       int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
 // Attach the zero-initialised counters (>= flags_needed ints) and the workspace
@@ -234,6 +237,8 @@ cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, c
 cudaError_t generate_launch(__nv_bfloat16* dst, uint64_t seed, int tid, int64_t start,
                             int64_t count, float std, float mean, int64_t cols, int blk,
                             int blk_stride, int blk_off, cudaStream_t stream);
+// cos / sin of the rotate-half angles t * theta^(-2j/hd), computed in double on the host,
+// laid out [hd/2][T] (positions contiguous).
 cudaError_t rope_table_build(float* cos_dev, float* sin_dev, int T, int hd, float theta,
                              cudaStream_t stream);
 

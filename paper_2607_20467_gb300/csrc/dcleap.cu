@@ -305,8 +305,8 @@ dcl_status build_graph(dcl_ctx* c) {
 // environment variable DCL_GEMM_TILES, e.g. "o=128,down=pair:2" (128 / 256 = one-CTA tile
 // width, pair[:S] = CTA-pair tile with S K-splits, pair:sk[:S] = CTA-pair tile with the
 // stream-K schedule, S segments per left-over tile, pair:mc[:S] = pairs sharing weight
-// tiles by multicast, S K-splits, pair:h = left-over tiles as half-width pieces); 0 = let
-// the planner choose.
+// tiles by multicast, S K-splits, pair:h = left-over tiles as half-width pieces, pair:ds =
+// left-over tiles split by K over a cluster's two pairs); 0 = let the planner choose.
 int tile_override(const char* name) {
   const char* env = getenv("DCL_GEMM_TILES");
   if (!env) return 0;
@@ -319,6 +319,7 @@ int tile_override(const char* name) {
       if (strncmp(v, "pair:sk", 7) == 0) return kTilePair | kTileStreamK | ((v[7] == ':' ? atoi(v + 8) : 0) << 8);
       if (strncmp(v, "pair:mc", 7) == 0) return kTilePair | kTileMulticast | ((v[7] == ':' ? atoi(v + 8) : 0) << 8);
       if (strcmp(v, "pair:h") == 0 || strncmp(v, "pair:h,", 7) == 0) return kTilePair | kTileHalves;
+      if (strncmp(v, "pair:ds", 7) == 0) return kTilePair | kTileDsmem;
       if (strncmp(v, "pair", 4) == 0) return kTilePair | ((v[4] == ':' ? atoi(v + 5) : 0) << 8);
       return atoi(v);
     }
@@ -362,6 +363,7 @@ dcl_status build_plans(dcl_ctx* c) {
     e0.ldo = nqkv;
     e0.rope_cos = c->rope_cos;
     e0.rope_sin = c->rope_sin;
+    e0.rope_T = c->max_seq;
     e0.rope_cols = (H + G) * hd;
     e0.head_dim = hd;
     e0.seq_T = c->T;

@@ -116,8 +116,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
     if (n0 < ep.rope_cols) {
       const int hd = ep.head_dim, half = hd >> 1;
       const int pos = live ? row % ep.seq_T : 0;
-      const float* cs = ep.rope_cos + (size_t)pos * half;
-      const float* sn = ep.rope_sin + (size_t)pos * half;
+      const float* cs = ep.rope_cos + pos;  // [half][rope_T]: a warp's rows read one line
+      const float* sn = ep.rope_sin + pos;
 #pragma unroll 1
       for (int hb = 0; hb < BN; hb += hd) {
 #pragma unroll 1
@@ -129,7 +129,8 @@ __device__ __forceinline__ void epilogue_tile(uint32_t taddr, int row, int n_blk
             float a[32], b[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const float c = __ldg(cs + j0 + i), s = __ldg(sn + j0 + i);
+              const size_t jt = (size_t)(j0 + i) * ep.rope_T;
+              const float c = __ldg(cs + jt), s = __ldg(sn + jt);
               a[i] = lo[i] * c - hi[i] * s;
               b[i] = hi[i] * c + lo[i] * s;
             }
@@ -408,11 +409,15 @@ constexpr int BOX_BYTES = 32 * 128;                 // one staging box: 32 rows 
 constexpr int STG2_BYTES = 4 * 2 * BOX_BYTES;       // 4 epilogue warps x 2 boxes
 constexpr int FIX_BOXES = RING2_BYTES / (4 * BOX_BYTES);  // stream-K fix-up boxes per warp
 constexpr int BARS2_BYTES = 640;
-static_assert(16 * STAGES2 + 48 + 8 * 4 * FIX_BOXES <= BARS2_BYTES, "barrier area");
+static_assert(16 * STAGES2 + 48 + 8 * 4 * FIX_BOXES + 40 <= BARS2_BYTES, "barrier area");
 static_assert(FIX_BOXES >= 2, "fix-up needs two boxes per warp");
 constexpr size_t SMEM2 = 1024 + (size_t)RING2_BYTES + STG2_BYTES + BARS2_BYTES;
 static_assert(SMEM2 <= 232448, "shared memory per CTA");
 constexpr int TMEM2_COLS = 512;
+// DSMEM split: the received fp32 half-sum rows, padded by 16 bytes so that eight lanes'
+// 16-byte accesses to eight consecutive rows fall in distinct bank groups
+constexpr int DS_ROW_BYTES = 256 * 4 + 16;
+static_assert(128 * DS_ROW_BYTES <= RING2_BYTES, "the received sum lives in the operand ring");
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
@@ -473,6 +478,36 @@ __device__ __forceinline__ void umma_commit_pair(uint32_t bar, uint16_t cta_mask
 }
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+// Bulk copy of `bytes` (a multiple of 16) from this CTA's shared memory to another CTA's
+// (dst and bar: shared::cluster addresses from mapa), completing on that CTA's barrier.
+__device__ __forceinline__ void bulk_copy_to_cluster(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "r"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+// Bounded wait for a phase completed by arrivals released at cluster scope (data that
+// other CTAs of the cluster wrote into this CTA's shared memory is visible afterwards).
+__device__ __forceinline__ bool mbar_try_wait_acq_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(1000000u)
+      : "memory");
+  return ok != 0;
+}
+__device__ __noinline__ bool mbar_wait_acq_cluster(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait_acq_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait_acq_cluster(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
+  }
 }
 // This lane's row of a staging box: 32 fp32 values, or 32 bf16 values into half h
 // (columns 32h .. 32h + 31) of a 64-column bf16 box.
@@ -547,11 +582,24 @@ struct Src {
   size_t part_stride = 0;       // floats between consecutive splits' partials
   int nparts = 0;
   int row = 0;                  // this thread's row within the CTA's 128-row half
+  uint32_t dpart = 0;           // DSMEM split: the other K half's sum in this CTA's shared
+                                // memory, row r at dpart + r * DS_ROW_BYTES (0: none)
 };
 __device__ __forceinline__ void src_cols(const Src& s, int col, float (&v)[32]) {
   uint32_t r[32];
   tmem_ld32(s.taddr + col, r);
-  if (s.has_sum) {
+  if (s.dpart) {
+    tmem_ld_wait();
+    const uint32_t a = s.dpart + (uint32_t)(s.row * DS_ROW_BYTES + col * 4);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float4 t = ld_shared_v4(a + 16 * k);
+      v[4 * k] = f32(r[4 * k]) + t.x;  // K lower half (own) + K upper half (received)
+      v[4 * k + 1] = f32(r[4 * k + 1]) + t.y;
+      v[4 * k + 2] = f32(r[4 * k + 2]) + t.z;
+      v[4 * k + 3] = f32(r[4 * k + 3]) + t.w;
+    }
+  } else if (s.has_sum) {
     uint32_t q[32];
     tmem_ld32(s.tsum + col, q);
     tmem_ld_wait();
@@ -628,47 +676,45 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       const int hd = ep.head_dim, half = hd >> 1;
       const int pos = row < M ? (ep.row_pos ? ep.row_pos[row] : row % ep.seq_T) : 0;
       const bool to_k = ep.k_store && n0 >= ep.k_col0;  // k columns go to the key store
-      const float* cs = ep.rope_cos + (size_t)pos * half;
-      const float* sn = ep.rope_sin + (size_t)pos * half;
+      // tables [half][rope_T]: the 32 consecutive positions of a band read one 128-byte line
+      const float* cs = ep.rope_cos + pos;
+      const float* sn = ep.rope_sin + pos;
 #pragma unroll 1
       for (int hb = 0; hb < W; hb += hd) {
-        // rotate-half pairs (j, j + half): hd 128 fills a box with rotated columns
-        // [hb, hb + 64) and one with [hb + 64, hb + 128); hd 64 fills one box [hb, hb + 64)
-        uint32_t b0, b1;
-        if (hd == 128) {  // both boxes free
-          if (o.lane == 0) bulk_wait_read<0>();
-          __syncwarp();
-          b0 = o.box0 + (uint32_t)(o.n & 1) * BOX_BYTES;
-          b1 = o.box0 + (uint32_t)((o.n + 1) & 1) * BOX_BYTES;
-        } else {
-          b0 = b1 = o.acquire();
-        }
+        // rotate-half pairs (j, j + half).  hd 128: box `part` 0 holds the rotated columns
+        // [hb, hb + 64) = x_j c - x_{j+64} s, part 1 holds [hb + 64, hb + 128) = x_{j+64} c
+        // + x_j s; each part re-reads both source halves from TMEM so that one box at a
+        // time is staged and the stores stay pipelined (a head never waits for every store
+        // in flight, which under a concurrent mainloop cost ~20 us per tile).  hd 64: one
+        // box [hb, hb + 64) holds both halves.
+        const int nparts = hd == 128 ? 2 : 1;
 #pragma unroll 1
-        for (int j0 = 0; j0 < half; j0 += 32) {
-          float lo[32], hi[32];
-          src_cols(s, hb + j0, lo);
-          src_cols(s, hb + half + j0, hi);
+        for (int part = 0; part < nparts; ++part) {
+          const uint32_t b = o.acquire();
+#pragma unroll 1
+          for (int j0 = 0; j0 < half; j0 += 32) {
+            float lo[32], hi[32];
+            src_cols(s, hb + j0, lo);
+            src_cols(s, hb + half + j0, hi);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float c = __ldg(cs + j0 + i), sv = __ldg(sn + j0 + i);
-            const float x = lo[i], y = hi[i];
-            lo[i] = x * c - y * sv;
-            hi[i] = y * c + x * sv;
+            for (int i = 0; i < 32; ++i) {
+              const size_t jt = (size_t)(j0 + i) * ep.rope_T;
+              const float c = __ldg(cs + jt), sv = __ldg(sn + jt);
+              const float x = lo[i], y = hi[i];
+              lo[i] = x * c - y * sv;
+              hi[i] = y * c + x * sv;
+            }
+            if (hd == 128) {
+              stage_bf16(b, o.lane, j0 >> 5, part == 0 ? lo : hi);
+            } else {
+              stage_bf16(b, o.lane, 0, lo);
+              stage_bf16(b, o.lane, 1, hi);
+            }
           }
-          if (hd == 128) {
-            stage_bf16(b0, o.lane, j0 >> 5, lo);
-            stage_bf16(b1, o.lane, j0 >> 5, hi);
-          } else {
-            stage_bf16(b0, o.lane, 0, lo);
-            stage_bf16(b0, o.lane, 1, hi);
-          }
-        }
-        if (to_k) {
-          o.issue3(tmk, b0, n0 + hb - ep.k_col0, t0, bz);
-          if (hd == 128) o.issue3(tmk, b1, n0 + hb + 64 - ep.k_col0, t0, bz);
-        } else {
-          o.issue(tmc, b0, n0 + hb, o.row0, false);
-          if (hd == 128) o.issue(tmc, b1, n0 + hb + 64, o.row0, false);
+          if (to_k)
+            o.issue3(tmk, b, n0 + hb + 64 * part - ep.k_col0, t0, bz);
+          else
+            o.issue(tmc, b, n0 + hb + 64 * part, o.row0, false);
         }
       }
     } else if (ep.vt_heads > 0) {
@@ -867,11 +913,13 @@ __device__ __noinline__ bool fixup_to_tmem(const CUtensorMap* tmw, int y0, int s
 //              (the tile's last segment: it waits for the other segments' partials, sums
 //              them in K order and runs the epilogue), so no pair waits on a pair that is
 //              itself waiting.
-enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3 };
+enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3, IT_DS_RECV = 4, IT_DS_SEND = 5 };
 struct Sched {
   int tiles, ku, C, splits;
   int streamk;  // 0: off; else the number of pairs (<= C) that share the left-over tiles
   int halves;   // 1: the tiles of a partial last round run as two 256 x 128 pieces each
+  int ds;       // 1: the tiles of a partial last round are split by K over the two pairs
+                //    of a 4-CTA cluster, the upper half's sum sent through DSMEM
 };
 struct Item {
   int t, ku0, ku1, kind;
@@ -884,6 +932,35 @@ struct Item {
 __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& it) {
   it.piece = 0;
   it.width = 256;
+  if (s.ds) {
+    // c = pair index (pairs 2k and 2k + 1 form cluster k): full rounds of whole tiles,
+    // then left-over tile `first + k` on cluster k, K lower half on its first pair (which
+    // receives the other half's sum and runs the epilogue), upper half on its second
+    const int full = s.tiles / s.C;
+    if (idx < full) {
+      it.t = c + idx * s.C;
+      it.ku0 = 0;
+      it.ku1 = s.ku;
+      it.kind = IT_PLAIN;
+      return true;
+    }
+    const int first = full * s.C, k = c >> 1;
+    if (2 * (s.tiles - first) > s.C) {  // (fewer rows than planned) more left-over tiles
+      it.t = c + idx * s.C;            // than clusters: whole tiles, round robin
+      it.ku0 = 0;
+      it.ku1 = s.ku;
+      it.kind = IT_PLAIN;
+      return it.t < s.tiles;
+    }
+    if (idx > full || first + k >= s.tiles) return false;
+    it.t = first + k;
+    const int mid = s.ku >> 1;
+    const bool upper = (c & 1) != 0;
+    it.ku0 = upper ? mid : 0;
+    it.ku1 = upper ? s.ku : mid;
+    it.kind = upper ? IT_DS_SEND : IT_DS_RECV;
+    return true;
+  }
   if (s.halves) {
     // full rounds of whole tiles, then every left-over tile as two half-width pieces on
     // two consecutive pairs (same rows of A, neighbouring rows of W): the last round
@@ -975,7 +1052,7 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
 // weights cross from L2 once per cluster.  Every load completes on its destination pair's
 // leader barrier (64 KB per stage, as without multicast); a stage is refilled once both
 // pairs' MMAs have released it (empty counts the two leaders' commits).
-template <int EPI, bool MC>
+template <int EPI, bool MC, bool DS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
                     const __grid_constant__ CUtensorMap tmbh, const __grid_constant__ CUtensorMap tmc,
@@ -997,18 +1074,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t drain = tempty0 + 16;
   const uint32_t holder = drain + 8;
   const uint32_t fix0 = holder + 8;  // 4 x FIX_BOXES stream-K fix-up barriers
+  const uint32_t ds_go = fix0 + 8 * 4 * FIX_BOXES;  // DS: the receiver's ring is free (4 warps)
+  const uint32_t ds_data0 = ds_go + 8;              // DS: + 8 q, band q's rows have arrived (tx bytes)
   volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
 
   static_assert(!MC || KA2 == 1, "the multicast variant stages one K block per ring stage");
-  constexpr int CL = MC ? 4 : 2;  // CTAs per cluster
+  static_assert(!(MC && DS), "one four-CTA scheme at a time");
+  constexpr int CL = (MC || DS) ? 4 : 2;  // CTAs per cluster
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t crank = cluster_ctarank();
   const uint32_t rank = crank & 1u;             // 0: leader of the pair (issues the MMAs), 1: peer
-  const uint32_t pr = MC ? (crank >> 1) : 0u;   // which pair of the cluster
+  const uint32_t pr = (MC || DS) ? (crank >> 1) : 0u;  // which pair of the cluster
   const uint32_t lead = crank & ~1u;            // cluster rank of this pair's leader
   const uint16_t pair_mask = (uint16_t)(0x3u << lead);
-  const int cluster = blockIdx.x / CL;
+  // the scheduler's unit: the cluster (pairs and MC), or the pair (DS: 2 per cluster)
+  const int cluster = DS ? (int)(blockIdx.x >> 1) : (int)(blockIdx.x / CL);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
@@ -1021,6 +1102,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(tempty0 + 8, 8);
     mbar_init(drain, 1);
     for (int b = 0; b < 4 * FIX_BOXES; ++b) mbar_init(fix0 + 8 * b, 1);
+    mbar_init(ds_go, 4);
+    for (int b = 0; b < 4; ++b) mbar_init(ds_data0 + 8 * b, 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tma);
@@ -1042,10 +1125,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   Sched sc;
   sc.tiles = num_mh * num_n;
   sc.ku = (K + BK * KA2 - 1) / (BK * KA2);
-  sc.C = gridDim.x / CL;
+  sc.C = DS ? gridDim.x / 2 : gridDim.x / CL;
   sc.splits = splits;
   sc.streamk = streamk;
   sc.halves = halves;
+  sc.ds = DS ? 1 : 0;
   // item tile -> (m block, n block); MC: pair pr takes the pr-th 256-row half of the unit
   auto tile_mn = [&](int t, int& m_blk, int& n_blk) {
     m_blk = MC ? 2 * (t % num_mh) + (int)pr : t % num_mh;
@@ -1193,6 +1277,52 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // nothing to store
       } else if (it.kind == IT_PLAIN) {
         epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep, it.piece, it.width);
+      } else if (it.kind == IT_DS_RECV) {
+        // this pair's MMAs are done (tfull): the operand ring is free for the other K
+        // half's sum, which the other pair of the cluster writes into it; then the
+        // epilogue adds it to this accumulator (lower half + upper half, a fixed order)
+        const uint32_t partner = crank ^ 2u;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(ds_data0 + 8 * q, 32 * DS_ROW_BYTES);  // this band's rows
+          mbar_arrive_cluster(mapa_shared(ds_go, partner));
+        }
+        if (!mbar_wait_acq_cluster(ds_data0 + 8 * q, 0, abort_flag)) {
+          *abort_flag = 1;
+          report_error(err, DERR_WAIT_TIMEOUT);
+        }
+        __syncwarp();
+        s.dpart = sA;
+        if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
+      } else if (it.kind == IT_DS_SEND) {
+        // the K upper half: each lane writes its accumulator row into this CTA's own ring
+        // (free: this pair's MMAs are done), then, once the receiving pair's ring is free,
+        // one bulk copy per warp moves the band's 32 rows into the same place there
+        const uint32_t partner = crank ^ 2u;
+        const uint32_t own = sA + (uint32_t)(row_local * DS_ROW_BYTES);
+#pragma unroll 1
+        for (int c = 0; c < 256; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(s.taddr + c, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            st_shared_v4(own + (uint32_t)((c + 4 * k) * 4), r[4 * k], r[4 * k + 1], r[4 * k + 2], r[4 * k + 3]);
+        }
+        fence_proxy_async_smem();  // the rows are read by the bulk copy (async proxy)
+        __syncwarp();
+        if (!mbar_wait_acq_cluster(ds_go, 0, abort_flag)) {
+          *abort_flag = 1;
+          report_error(err, DERR_WAIT_TIMEOUT);
+        }
+        __syncwarp();
+        if (lane == 0 && !*abort_flag) {
+          const uint32_t band = sA + (uint32_t)(q * 32 * DS_ROW_BYTES);
+          bulk_copy_to_cluster(mapa_shared(band, partner), band, 32 * DS_ROW_BYTES,
+                               mapa_shared(ds_data0 + 8 * q, partner));
+          bulk_commit();
+          bulk_wait_read<0>();  // this CTA's rows were read (the ring is not touched again)
+        }
+        __syncwarp();
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
         int* flag = flags + t * 2 + rank;
@@ -1335,10 +1465,10 @@ cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
   return launch_pdl(kern, p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream, p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
 }
 
-template <int EPI, bool MC>
+template <int EPI, bool MC, bool DS = false>
 cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   static bool attr_set = false;
-  auto kern = gemm_tc2_kernel<EPI, MC>;
+  auto kern = gemm_tc2_kernel<EPI, MC, DS>;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2);
     if (e != cudaSuccess) return e;
@@ -1351,7 +1481,7 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = MC ? 4 : 2;
+  attr[0].val.clusterDim.x = (MC || DS) ? 4 : 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1366,7 +1496,7 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
 int mc_max_clusters() {
   static int n = -1;
   if (n < 0) {
-    auto kern = gemm_tc2_kernel<EPI_BF16, true>;
+    auto kern = gemm_tc2_kernel<EPI_BF16, true, false>;
     n = 0;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2) == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
@@ -1568,6 +1698,46 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
       return cudaErrorInvalidValue;
     }
   }
+  // DSMEM split (kTileDsmem, or chosen by the planner): four-CTA clusters; whole tiles in
+  // full rounds over all pairs, then each left-over tile split by K over the two pairs of
+  // one cluster, the upper half's fp32 sum written straight into the lower pair's idle
+  // operand ring (distributed shared memory, no global partials) and added there before
+  // the epilogue.  The last round then costs about half a tile.
+  int ds = 0, ds_clusters = 0;
+  if (cg == 2) {
+    const bool ds_forced = pair_forced && (tile & kTileDsmem);
+    const bool ds_ok = streamk == 0 && mc == 0 && halves == 0 && epi != EPI_LMHEAD && units >= 2 &&
+                       (ds_forced ? forced_splits <= 1 : true);
+    const int cl4 = ds_ok ? std::min(num_sms / 4, mc_max_clusters()) : 0;
+    long full = 0, rest = 0;
+    if (cl4 >= 1) {
+      full = pair_tiles / (2L * cl4);
+      rest = pair_tiles % (2L * cl4);
+    }
+    const bool fits = cl4 >= 1 && rest <= cl4;
+    if (ds_forced && !fits) {
+      *why = "gemm: the DSMEM split needs four-CTA clusters, no other schedule, K >= 128 and at most one "
+             "left-over tile per cluster";
+      return cudaErrorInvalidValue;
+    }
+    if (fits) {
+      const double c_plain = (double)((pair_tiles + pairs - 1) / pairs);
+      const double c_ds = (double)full + (rest ? 0.56 : 0.0);
+      const double c_split = splits > 1 ? 0.5 * (double)((pair_tiles * splits + pairs - 1) / pairs) + 0.15 : 1e9;
+      const char* env = getenv("DCL_GEMM_DS");
+      const bool allowed = !(env && env[0] == '0');
+      // (the planner's own choice: tile 0, or a bare pair tile with no other flag or split)
+      const bool auto_sched = tile == 0 || tile == kTilePair;
+      if (ds_forced || (allowed && auto_sched && rest > 0 && c_ds < c_plain - 0.05 && c_ds < c_split)) {
+        ds = 1;
+        splits = 1;
+        ds_clusters = full > 0 ? cl4 : (int)rest;
+        if (ds_clusters < 1) ds_clusters = 1;
+      }
+    }
+  }
+  plan->ds = ds;
+  if (ds) plan->splits = 1;
   plan->mc = mc;
   if (cg == 2) {
     plan->n_tiles = (int)pair_tiles;
@@ -1582,6 +1752,7 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
       const long cl = std::min<long>(num_sms / 4, mc_clusters);
       plan->grid = 4 * (int)(units < cl ? units : cl);
     }
+    if (ds) plan->grid = 4 * ds_clusters;
     plan->smem = SMEM2;
     if (splits > 1) {
       plan->flags_needed = (size_t)plan->n_tiles * 2;
@@ -1684,6 +1855,15 @@ cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
       case EPI_QKV_ROPE: return launch_t2<EPI_QKV_ROPE, true>(p, err, stream);
       case EPI_SWIGLU: return launch_t2<EPI_SWIGLU, true>(p, err, stream);
       case EPI_LMHEAD: return launch_t2<EPI_LMHEAD, true>(p, err, stream);
+    }
+    return cudaErrorInvalidValue;
+  }
+  if (p.cg == 2 && p.ds) {
+    switch (p.epi) {
+      case EPI_BF16: return launch_t2<EPI_BF16, false, true>(p, err, stream);
+      case EPI_RESID_F32: return launch_t2<EPI_RESID_F32, false, true>(p, err, stream);
+      case EPI_QKV_ROPE: return launch_t2<EPI_QKV_ROPE, false, true>(p, err, stream);
+      case EPI_SWIGLU: return launch_t2<EPI_SWIGLU, false, true>(p, err, stream);
     }
     return cudaErrorInvalidValue;
   }

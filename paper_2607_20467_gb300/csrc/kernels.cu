@@ -547,8 +547,8 @@ cudaError_t rope_table_build(float* cos_dev, float* sin_dev, int T, int hd, floa
   for (int t = 0; t < T; ++t)
     for (int j = 0; j < half; ++j) {
       const double ang = (double)t * pow((double)theta, -2.0 * j / hd);
-      hc[(size_t)t * half + j] = (float)cos(ang);
-      hc[(size_t)T * half + (size_t)t * half + j] = (float)sin(ang);
+      hc[(size_t)j * T + t] = (float)cos(ang);  // [half][T]: positions contiguous
+      hc[(size_t)T * half + (size_t)j * T + t] = (float)sin(ang);
     }
   e = cudaMemcpyAsync(cos_dev, hc, sizeof(float) * (size_t)T * half, cudaMemcpyHostToDevice, stream);
   if (e == cudaSuccess)

@@ -62,13 +62,13 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
-PAIR, SK, MC, HALF = 2, 1 << 16, 1 << 17, 1 << 18
+PAIR, SK, MC, HALF, DS = 2, 1 << 16, 1 << 17, 1 << 18, 1 << 19
 # auto, one-CTA 128 / 256 columns, CTA pair (library's K schedule), CTA pair unsplit,
 # CTA pair with 2 / 3 K splits, CTA pair with stream-K over all pairs / in K halves,
 # clusters of two pairs sharing weight tiles (unsplit / 2 K splits), left-over tiles as
 # two half-width pieces
 TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK, PAIR | SK | (2 << 8),
-         PAIR | MC | (1 << 8), PAIR | MC | (2 << 8), PAIR | HALF]
+         PAIR | MC | (1 << 8), PAIR | MC | (2 << 8), PAIR | HALF, PAIR | DS]
 
 
 def _splits(tile):
@@ -92,6 +92,8 @@ def _streamk_possible(M, N, K, segments):
 
 def _unsupported(M, N, K, tile):
     """True when the tile choice cannot run this shape (then the call must be refused)."""
+    if tile & DS:  # (and at most one left-over tile per cluster: every shape here has <= 32)
+        return K // 64 < 2
     if tile & SK:
         return not _streamk_possible(M, N, K, (tile >> 8) & 0xff)
     return K // 64 < _splits(tile) or not _rows_ok(M, tile)
@@ -139,7 +141,8 @@ def test_linear_residual(ops, M, N, K, tile):
 
 @pytest.mark.parametrize("tile,mode", [(PAIR | (3 << 8), 1), (PAIR | (2 << 8), 0), (0, 1), (0, 0),
                                        (PAIR | SK, 0), (PAIR | SK, 1), (PAIR | SK | (2 << 8), 1),
-                                       (PAIR | MC | (2 << 8), 1), (PAIR | MC | (3 << 8), 0)])
+                                       (PAIR | MC | (2 << 8), 1), (PAIR | MC | (3 << 8), 0),
+                                       (PAIR | DS, 1), (PAIR | DS, 0)])
 def test_linear_split_k_is_deterministic(ops, tile, mode):
     """Split-K and stream-K partial sums are combined in K order: two runs give the same
     bits."""
