@@ -105,7 +105,9 @@ def test_cache_changes_the_result_only_through_stale_keys(dcl, weights):
         out, st, status = a.generate(max_steps=4 * M)
         assert st.done == 1
         x, p = a.get_state()
-        assert (p == T).all() and (x[:, N:] != TINY.mask_id).all() and (x[:, :N] == prompt).all()
+        # (a committed token may be the MASK id itself when that was the prediction; random
+        # weights make that about 1 / V likely per position)
+        assert (p == T).all() and (x[:, N:] == TINY.mask_id).mean() < 0.01 and (x[:, :N] == prompt).all()
         a.restart()
         out2, st2, _ = a.generate(max_steps=4 * M)
         assert (out2 == out).all() and st2.steps == st.steps
