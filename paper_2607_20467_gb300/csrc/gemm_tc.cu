@@ -408,16 +408,19 @@ constexpr int RING2_BYTES = STAGES2 * STAGE2_BYTES;
 constexpr int BOX_BYTES = 32 * 128;                 // one staging box: 32 rows x 128 bytes
 constexpr int STG2_BYTES = 4 * 2 * BOX_BYTES;       // 4 epilogue warps x 2 boxes
 constexpr int FIX_BOXES = RING2_BYTES / (4 * BOX_BYTES);  // stream-K fix-up boxes per warp
-constexpr int BARS2_BYTES = 640;
-static_assert(16 * STAGES2 + 48 + 8 * 4 * FIX_BOXES + 40 <= BARS2_BYTES, "barrier area");
+constexpr int BARS2_BYTES = 768;
+static_assert(16 * STAGES2 + 48 + 8 * 4 * FIX_BOXES + 8 + 8 * 16 <= BARS2_BYTES, "barrier area");
 static_assert(FIX_BOXES >= 2, "fix-up needs two boxes per warp");
 constexpr size_t SMEM2 = 1024 + (size_t)RING2_BYTES + STG2_BYTES + BARS2_BYTES;
 static_assert(SMEM2 <= 232448, "shared memory per CTA");
 constexpr int TMEM2_COLS = 512;
-// DSMEM split: the received fp32 half-sum rows, padded by 16 bytes so that eight lanes'
-// 16-byte accesses to eight consecutive rows fall in distinct bank groups
-constexpr int DS_ROW_BYTES = 256 * 4 + 16;
-static_assert(128 * DS_ROW_BYTES <= RING2_BYTES, "the received sum lives in the operand ring");
+// DSMEM split: the received fp32 half sum moves in 64-column chunks per 32-row band, each
+// a contiguous block of 32 rows padded by 16 bytes (eight lanes' 16-byte accesses to
+// eight consecutive rows fall in distinct bank groups), block (band, chunk) at
+// (band * 4 + chunk) * DS_BLOCK_BYTES
+constexpr int DS_ROW_BYTES = 64 * 4 + 16;
+constexpr int DS_BLOCK_BYTES = 32 * DS_ROW_BYTES;
+static_assert(16 * DS_BLOCK_BYTES <= RING2_BYTES, "the received sum lives in the operand ring");
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
@@ -583,14 +586,30 @@ struct Src {
   int nparts = 0;
   int row = 0;                  // this thread's row within the CTA's 128-row half
   uint32_t dpart = 0;           // DSMEM split: the other K half's sum in this CTA's shared
-                                // memory, row r at dpart + r * DS_ROW_BYTES (0: none)
+                                // memory, in (band, chunk) blocks (0: none)
+  uint32_t dbar = 0;            // DSMEM split: this band's 4 chunk barriers
+  mutable uint32_t dready = 0;  // chunks waited for so far
+  volatile int* dabort = nullptr;
+  int* derr = nullptr;
 };
+// DSMEM split: the received 64-column chunk has arrived (bounded wait, once per chunk;
+// warp-uniform)
+__device__ __forceinline__ void ds_chunk_ready(const Src& s, int chunk) {
+  if (s.dready & (1u << chunk)) return;
+  if (!mbar_wait_acq_cluster(s.dbar + 8 * chunk, 0, s.dabort)) {
+    *s.dabort = 1;
+    report_error(s.derr, DERR_WAIT_TIMEOUT);
+  }
+  s.dready |= 1u << chunk;
+}
 __device__ __forceinline__ void src_cols(const Src& s, int col, float (&v)[32]) {
   uint32_t r[32];
   tmem_ld32(s.taddr + col, r);
   if (s.dpart) {
+    ds_chunk_ready(s, col >> 6);
     tmem_ld_wait();
-    const uint32_t a = s.dpart + (uint32_t)(s.row * DS_ROW_BYTES + col * 4);
+    const uint32_t a = s.dpart + (uint32_t)((((s.row >> 5) * 4 + (col >> 6)) * 32 + (s.row & 31)) * DS_ROW_BYTES +
+                                            (col & 63) * 4);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       const float4 t = ld_shared_v4(a + 16 * k);
@@ -1077,7 +1096,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t holder = drain + 8;
   const uint32_t fix0 = holder + 8;  // 4 x FIX_BOXES stream-K fix-up barriers
   const uint32_t ds_go = fix0 + 8 * 4 * FIX_BOXES;  // DS: the receiver's ring is free (4 warps)
-  const uint32_t ds_data0 = ds_go + 8;              // DS: + 8 q, band q's rows have arrived (tx bytes)
+  const uint32_t ds_data0 = ds_go + 8;              // DS: + 8 (4 q + c), chunk c of band q arrived
   volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
 
@@ -1105,7 +1124,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(drain, 1);
     for (int b = 0; b < 4 * FIX_BOXES; ++b) mbar_init(fix0 + 8 * b, 1);
     mbar_init(ds_go, 4);
-    for (int b = 0; b < 4; ++b) mbar_init(ds_data0 + 8 * b, 1);
+    for (int b = 0; b < 16; ++b) mbar_init(ds_data0 + 8 * b, 1);
     *abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tma);
@@ -1283,47 +1302,58 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // this pair's MMAs are done (tfull): the operand ring is free for the other K
         // half's sum, which the other pair of the cluster writes into it; then the
         // epilogue adds it to this accumulator (lower half + upper half, a fixed order)
+        // The sum arrives in four 64-column chunks per band; the epilogue waits for each
+        // chunk when it first reads it, so it overlaps the rest of the transfer.
         const uint32_t partner = crank ^ 2u;
         if (lane == 0) {
-          mbar_arrive_expect_tx(ds_data0 + 8 * q, 32 * DS_ROW_BYTES);  // this band's rows
+          for (int c = 0; c < 4; ++c) mbar_arrive_expect_tx(ds_data0 + 8 * (4 * q + c), DS_BLOCK_BYTES);
           mbar_arrive_cluster(mapa_shared(ds_go, partner));
-        }
-        if (!mbar_wait_acq_cluster(ds_data0 + 8 * q, 0, abort_flag)) {
-          *abort_flag = 1;
-          report_error(err, DERR_WAIT_TIMEOUT);
         }
         __syncwarp();
         s.dpart = sA;
+        s.dbar = ds_data0 + 8 * (4 * q);
+        s.dready = 0;
+        s.dabort = abort_flag;
+        s.derr = err;
         if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
+        // every chunk has landed before this CTA may leave (one the epilogue skipped too)
+        for (int c = 0; c < 4; ++c) ds_chunk_ready(s, c);
       } else if (it.kind == IT_DS_SEND) {
         // the K upper half: each lane writes its accumulator row into this CTA's own ring
         // (free: this pair's MMAs are done), then, once the receiving pair's ring is free,
         // one bulk copy per warp moves the band's 32 rows into the same place there
         const uint32_t partner = crank ^ 2u;
-        const uint32_t own = sA + (uint32_t)(row_local * DS_ROW_BYTES);
+        bool go = false;
 #pragma unroll 1
-        for (int c = 0; c < 256; c += 32) {
-          uint32_t r[32];
-          tmem_ld32(s.taddr + c, r);
-          tmem_ld_wait();
+        for (int chunk = 0; chunk < 4; ++chunk) {
+          const uint32_t blk = sA + (uint32_t)((4 * q + chunk) * DS_BLOCK_BYTES);
+          const uint32_t own = blk + (uint32_t)(lane * DS_ROW_BYTES);
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            uint32_t r[32];
+            tmem_ld32(s.taddr + 64 * chunk + 32 * h, r);
+            tmem_ld_wait();
 #pragma unroll
-          for (int k = 0; k < 8; ++k)
-            st_shared_v4(own + (uint32_t)((c + 4 * k) * 4), r[4 * k], r[4 * k + 1], r[4 * k + 2], r[4 * k + 3]);
+            for (int k = 0; k < 8; ++k)
+              st_shared_v4(own + (uint32_t)((32 * h + 4 * k) * 4), r[4 * k], r[4 * k + 1], r[4 * k + 2], r[4 * k + 3]);
+          }
+          fence_proxy_async_smem();  // the rows are read by the bulk copy (async proxy)
+          __syncwarp();
+          if (!go) {
+            if (!mbar_wait_acq_cluster(ds_go, 0, abort_flag)) {
+              *abort_flag = 1;
+              report_error(err, DERR_WAIT_TIMEOUT);
+            }
+            go = true;
+            __syncwarp();
+          }
+          if (lane == 0 && !*abort_flag) {
+            bulk_copy_to_cluster(mapa_shared(blk, partner), blk, DS_BLOCK_BYTES,
+                                 mapa_shared(ds_data0 + 8 * (4 * q + chunk), partner));
+            bulk_commit();
+          }
         }
-        fence_proxy_async_smem();  // the rows are read by the bulk copy (async proxy)
-        __syncwarp();
-        if (!mbar_wait_acq_cluster(ds_go, 0, abort_flag)) {
-          *abort_flag = 1;
-          report_error(err, DERR_WAIT_TIMEOUT);
-        }
-        __syncwarp();
-        if (lane == 0 && !*abort_flag) {
-          const uint32_t band = sA + (uint32_t)(q * 32 * DS_ROW_BYTES);
-          bulk_copy_to_cluster(mapa_shared(band, partner), band, 32 * DS_ROW_BYTES,
-                               mapa_shared(ds_data0 + 8 * q, partner));
-          bulk_commit();
-          bulk_wait_read<0>();  // this CTA's rows were read (the ring is not touched again)
-        }
+        if (lane == 0) bulk_wait_read<0>();  // this CTA's rows were read (the ring is not touched again)
         __syncwarp();
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
