@@ -43,17 +43,6 @@ struct Cfg {
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
 };
 
-// Bring a box of the tensor into L2 ahead of its load (no shared memory, no barrier).
-__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* tm, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(tm)),
-               "r"(x), "r"(y)
-               : "memory");
-}
-#ifndef DCL_PF_AHEAD
-#define DCL_PF_AHEAD 0
-#endif
-constexpr int kPrefetchAhead = DCL_PF_AHEAD;  // K blocks of weights requested into L2 ahead
 
 __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
@@ -277,10 +266,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
         const int m_blk = t % num_m, n_blk = t / num_m;
-        for (int kb = 0; kb < num_kb && kb < kPrefetchAhead; ++kb)
-          tma_prefetch_l2(&tmb, kb * BK, n_blk * BN);
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (kb + kPrefetchAhead < num_kb) tma_prefetch_l2(&tmb, (kb + kPrefetchAhead) * BK, n_blk * BN);
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
             ok = false;
             break;
@@ -1177,10 +1163,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                               : (EPI == EPI_SWIGLU ? (int)rank * 128 + it.piece * 64 : it.piece * 128 + (int)rank * 64));
         const CUtensorMap* tw_map = hw ? &tmbh : &tmb;
         const uint32_t stage_tx = 2u * (uint32_t)(hw ? A2_STAGE_BYTES + B2_STAGE_BYTES / 2 : STAGE2_BYTES);
-        for (int kb = kb0; kb < kb1 && kb < kb0 + kPrefetchAhead; ++kb) tma_prefetch_l2(&tmb, kb * BK, wrow);
         for (int kb = kb0; kb < kb1; kb += KA2) {
-          for (int a = 0; a < KA2; ++a)
-            if (kb + a + kPrefetchAhead < kb1) tma_prefetch_l2(&tmb, (kb + a + kPrefetchAhead) * BK, wrow);
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
             ok = false;
             break;

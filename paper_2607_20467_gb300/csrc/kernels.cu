@@ -192,10 +192,10 @@ __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
 // A partial is {max m, sum exp(z - m), argmax id, second largest z, sum exp(z - m) * y}
 // over some columns, y = (z - m) log2(e) (the last one gives the entropy:
 // H = -sum P ln P = ln 2 * (log2(sum) - u / sum)).
-struct Part {
+struct Part {  // (aggregate: brace-initialised parts leave u = 0)
   float m, s, t2;
   int id;
-  float u = 0.f;
+  float u;
 };
 
 __device__ __forceinline__ void merge(Part& a, const Part& b) {
@@ -205,8 +205,8 @@ __device__ __forceinline__ void merge(Part& a, const Part& b) {
     return;
   }
   const float m = fmaxf(a.m, b.m);
-  const float da = (a.m - m) * kLog2e, db = (b.m - m) * kLog2e;  // <= 0, finite
-  const float ea = exp2f(da), eb = exp2f(db);
+  const float da = (a.m - m) * kLog2e, db = (b.m - m) * kLog2e;  // <= 0, finite; one is 0
+  const float ea = da == 0.f ? 1.f : exp2f(da), eb = db == 0.f ? 1.f : exp2f(db);
   const float s = a.s * ea + b.s * eb;
   // re-based to the new maximum: y' = y + d for every term
   const float u = ea * fmaf(da, a.s, a.u) + eb * fmaf(db, b.s, b.u);
@@ -251,24 +251,34 @@ __device__ __forceinline__ void write_conf(const Part& a, const ConfOut& o, int 
 }
 
 // LM row `row` (of *rows_dev) is written to slot slot[row] of top1 / p1 / p2.
-__global__ void lmhead_combine_kernel(const float4* __restrict__ part, const float* __restrict__ upart, int rows,
-                                      int nblk, ConfOut out, const int* __restrict__ rows_dev,
-                                      const int* __restrict__ slot) {
+// One CTA of COMBINE_THREADS per row: each thread merges a strided share of the row's
+// partials, then warps and the CTA merge in a fixed order (deterministic).
+constexpr int COMBINE_THREADS = 128;
+__global__ void __launch_bounds__(COMBINE_THREADS) lmhead_combine_kernel(
+    const float4* __restrict__ part, const float* __restrict__ upart, int rows, int nblk, ConfOut out,
+    const int* __restrict__ rows_dev, const int* __restrict__ slot) {
   pdl_wait();
   pdl_launch_dependents();
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
+  const int row = blockIdx.x;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   if (rows_dev) rows = min(rows, *rows_dev);
   if (row >= rows) return;
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
-  for (int i = lane; i < nblk; i += 32) {
+  for (int i = threadIdx.x; i < nblk; i += COMBINE_THREADS) {
     const size_t j = (size_t)row * nblk + i;
     const float4 v = part[j];
     merge(a, Part{v.x, v.y, v.w, __float_as_int(v.z), upart ? upart[j] : 0.f});
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) merge(a, shfl_part(a, o));
-  if (lane == 0) write_conf(a, out, slot ? slot[row] : row);
+  __shared__ Part red[COMBINE_THREADS / 32];
+  if (lane == 0) red[w] = a;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    Part t = red[0];
+    for (int k = 1; k < COMBINE_THREADS / 32; ++k) merge(t, red[k]);
+    write_conf(t, out, slot ? slot[row] : row);
+  }
 }
 
 // ------------------------------------------------------------------ DCV on one sequence
@@ -500,9 +510,8 @@ cudaError_t rmsnorm_launch(const float* x, const __nv_bfloat16* gain, __nv_bfloa
 
 cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int rows, int nblk, const ConfOut& o,
                                   const int* rows_dev, const int* slot, cudaStream_t stream) {
-  const int threads = 256;
-  const int blocks = (rows * 32 + threads - 1) / threads;
-  return launch_pdl(lmhead_combine_kernel, blocks, threads, 0, stream, part, upart, rows, nblk, o, rows_dev, slot);
+  return launch_pdl(lmhead_combine_kernel, rows, COMBINE_THREADS, 0, stream, part, upart, rows, nblk, o, rows_dev,
+                    slot);
 }
 
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
