@@ -45,13 +45,13 @@ WORKLOADS = {
     # the same architecture, long generation: prompt 512, gen 1024, batch 1
     "llada8b-long": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
                          seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
-    # the same, batch 8 (BASELINE config 4, full recompute)
+    # the same, batch 8, full recompute
     "llada8b-long-b8": dict(shape="llada8b", batch=8, n_prompt=512, gen=1024, block=32, window=512,
                             seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98),
     # Dream-7B shape (GQA 28 / 4 heads), batch 16, prompt 384, gen 512, full recompute
     "dream7b": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
                     seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98),
-    # the same three with the approximate prefix key / value cache (BASELINE configs 4 / 5)
+    # the same three with the approximate prefix key / value cache (refresh every 32 positions)
     "llada8b-long-cache": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
                                seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=1),
     "llada8b-long-b8-cache": dict(shape="llada8b", batch=8, n_prompt=512, gen=1024, block=32, window=512,
