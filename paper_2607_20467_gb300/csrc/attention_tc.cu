@@ -2,22 +2,20 @@
 // every position attends to every position of its sequence), on the tcgen05 tensor
 // cores of sm_103a.
 //
-// One CTA = 128 query rows of one (sequence, head); the key axis is walked in blocks of
-// 128 in two passes:
-//   pass 1: S_j = Q K_j^T into TMEM, row maxima m (softmax warps, one query row per
-//           thread);
-//   pass 2: S_j again; P_j = exp2(S_j * log2(e)/sqrt(hd) - m) with the row sum l kept in
-//           fp32; P_j is written to shared memory as a bf16 pair hi + lo (hi = P with its
-//           low 16 bits cleared, lo = bf16(P - hi): about 16 significant bits together)
-//           and O += P_hi V_j + P_lo V_j accumulates in TMEM.
-// O / l leaves through TMA.  Two passes cost one more Q K^T than an online softmax but
-// need no rescaling of the TMEM accumulator and give the exact row maximum.
+// One CTA = 128 query rows of one (sequence, head); the key axis is walked once, in
+// blocks of 128: S_j = Q K_j^T into TMEM (double-buffered), then per row a running
+// maximum m, P_j = exp2(S_j * log2(e)/sqrt(hd) - m) with the row sum l kept in fp32, P_j
+// written to shared memory as a bf16 pair hi + lo (hi = P with its low 16 bits cleared,
+// lo = bf16(P - hi): about 16 significant bits together), and O += P_hi V_j + P_lo V_j
+// in TMEM.  m moves only when a block's maximum exceeds it by more than 8 (P stays below
+// 2^8); l and O are then scaled by the same factor, so O / l is unchanged.  O / l leaves
+// through TMA.
 //
 // Roles (320 threads): warp 0 lane 0 TMA producer (Q once, then K / V^T blocks through a
 // 2-stage ring in the order the MMAs consume them); warp 1 allocates TMEM and its lane 0
 // issues the MMAs; warps 2..9 run the softmax and the epilogue, two warps per 32-row
-// band (TMEM lane quarter), each on one 64-column half of every S block: the row maxima
-// and sums of the two halves are combined through shared memory.  P is double-buffered so
+// band (TMEM lane quarter), each on one 64-column half of every S block: the block
+// maxima and the final sums of the two halves are combined through shared memory.  P is double-buffered so
 // that the softmax of block j + 1 overlaps the P V MMAs of block j.  V enters as V^T (a
 // K-major operand, kv contiguous), written by v_transpose_kernel from the q|k|v buffer.
 // Every wait is bounded (DERR_WAIT_TIMEOUT).
@@ -153,19 +151,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       long issued = 0;
       mbar_arrive_expect_tx(q_full, C::Q_BYTES);
       for (int bx = 0; bx < C::KB; ++bx) tma_load_2d(sQ + bx * AT_BOX, &tq, h * HD + bx * 64, q_off + qt * 128, q_full);
-      // consumption order: K_0 .. K_{nb-1} (pass 1); K_0, K_1, then per j: K_{j+2}, V_j
-      // (pass 2; K only while j + 2 < nb)
-      const int n_loads = 3 * nb;
+      // consumption order: K_0, K_1, then per j: K_{j+2}, V_j (K only while j + 2 < nb)
+      const int n_loads = 2 * nb;
       const int head = nb < 2 ? nb : 2, npairs = nb > 2 ? nb - 2 : 0;
       for (int u = 0; u < n_loads && ok; ++u) {
         bool is_v;
         int j;
-        if (u < nb) {
+        if (u < head) {
           is_v = false, j = u;
-        } else if (u - nb < head) {
-          is_v = false, j = u - nb;
         } else {
-          const int r = u - nb - head;
+          const int r = u - head;
           if (r < 2 * npairs) {
             is_v = (r & 1) != 0;
             j = (r >> 1) + (is_v ? 0 : 2);
@@ -259,8 +254,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         umma_commit(p_empty0 + 8 * pb);
         return true;
       };
-      for (int j = 0; ok && j < nb; ++j) ok = issue_s();  // pass 1
-      if (ok) ok = issue_s();                              // pass 2: S_0, S_1
+      if (ok) ok = issue_s();  // S_0, S_1
       if (ok && nb > 1) ok = issue_s();
       for (int j = 0; ok && j < nb; ++j) {  // S_{j+2} (its buffer frees with P_j) before PV_j
         if (j + 2 < nb) ok = issue_s();
@@ -284,75 +278,90 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     auto softmax_bar = []() { asm volatile("bar.sync 1, %0;" ::"n"(AT_SOFTMAX * 32) : "memory"); };
     const float scale2 = kLog2e * rsqrtf((float)HD);
+    // One pass over the key blocks with a running maximum.  Per block: this half's 64
+    // columns of S from TMEM, the block's row maximum combined with the partner warp's
+    // half through shared memory, then P = exp2(S scale - m) against the running maximum
+    // m.  m is raised only when a block's maximum exceeds it by more than 8 (so P <= 2^8,
+    // exact in fp32 and in the hi / lo split); l and this warp's half of O are then scaled
+    // by 2^(m_old - m_new) once the previous P V product has completed.  O and l carry
+    // the same factor, so O / l is the softmax of the exact-maximum form.
     bool ok = true;
-    int si = 0;
-    float m = -INFINITY;
-    for (int j = 0; ok && j < nb; ++j) {  // pass 1: row maxima
-      const int sb = si & 1;
-      ok = mbar_wait(s_full0 + 8 * sb, ((uint32_t)si >> 1) & 1u, abort_flag);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc_fence_after();
-      const int valid = T - j * 128 - co;  // live columns of this half
-      uint32_t v[2][32];  // this half of the row, one wait
-#pragma unroll
-      for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + co + 32 * c), v[c]);
-      tmem_ld_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_empty0 + 8 * sb);
-      float mm = -INFINITY;
-      if (valid >= 64) {
-#pragma unroll
-        for (int c = 0; c < 2; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e) mm = fmaxf(mm, f32(v[c][e]));
-      } else {
-#pragma unroll
-        for (int c = 0; c < 2; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (32 * c + e < valid) mm = fmaxf(mm, f32(v[c][e]));
-      }
-      m = fmaxf(m, mm * scale2);
-      ++si;
-    }
-    // the row maximum over both halves (every softmax warp reaches this point: a failed
-    // wait above is warp-uniform and skips no barrier, since ok stays false after it)
-    red[hs * 128 + r] = m;
-    softmax_bar();
-    m = fmaxf(red[r], red[128 + r]);
-    softmax_bar();  // every read is done before the sums reuse the slots
-    float l = 0.f;
-    for (int j = 0; ok && j < nb; ++j) {  // pass 2: P = exp2(s - m), l, P_hi / P_lo
-      const int sb = si & 1, pb = j & 1;
-      ok = mbar_wait(s_full0 + 8 * sb, ((uint32_t)si >> 1) & 1u, abort_flag);
+    float m = -INFINITY, l = 0.f;
+    const uint32_t band_bar_id = 2u + (uint32_t)q;  // the two warps of this 32-row band
+    auto band_bar = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(band_bar_id) : "memory"); };
+    for (int j = 0; j < nb; ++j) {  // (no early exit: both warps of a band meet at every barrier)
+      const int sb = j & 1, pb = j & 1;
+      if (ok) ok = mbar_wait(s_full0 + 8 * sb, ((uint32_t)j >> 1) & 1u, abort_flag);
       if (ok && j >= 2) ok = mbar_wait(p_empty0 + 8 * pb, ((uint32_t)(j - 2) >> 1) & 1u, abort_flag);  // PV_{j-2} read it
       ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc_fence_after();
-      const int valid = T - j * 128;
-      const uint32_t pbase = sP + (uint32_t)pb * 4 * AT_BOX;
+      const int valid = T - j * 128 - co;  // live columns of this half
       uint32_t v[2][32];
-      tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + co), v[0]);
+      float mm = -INFINITY;
+      if (ok) {
+        tc_fence_after();
 #pragma unroll
-      for (int c = 2 * hs; c < 2 * hs + 2; ++c) {
+        for (int c = 0; c < 2; ++c) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + co + 32 * c), v[c]);
         tmem_ld_wait();
-        if (c + 1 < 2 * hs + 2) tmem_ld32(tmem + lane_off + (uint32_t)(sb * 128 + 32 * (c + 1)), v[(c + 1) & 1]);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(s_empty0 + 8 * sb);  // the S buffer is free for S_{j+2}
+        if (valid >= 64) {
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; ++e) mm = fmaxf(mm, f32(v[c][e]));
+        } else {
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (32 * c + e < valid) mm = fmaxf(mm, f32(v[c][e]));
+        }
+      }
+      red[hs * 128 + r] = mm * scale2;
+      band_bar();
+      const float mb = fmaxf(red[r], red[128 + r]);
+      band_bar();  // both halves read before the next block writes the slots
+      if (!ok) continue;
+      const bool raise = mb > m + 8.f;  // always at the first block (m = -inf)
+      if (j > 0 && __any_sync(0xffffffffu, raise)) {
+        // rescale l and this warp's O columns; P V_{j-1} must have completed first
+        if (!mbar_wait(p_empty0 + 8 * ((j - 1) & 1), ((uint32_t)(j - 1) >> 1) & 1u, abort_flag)) ok = false;
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) continue;
+        tc_fence_after();
+        const float f = raise ? ex2_approx(m - mb) : 1.f;
+#pragma unroll 1
+        for (int c = co; c < HD && c < co + 64; c += 32) {
+          uint32_t ov[32];
+          tmem_ld32(tmem + lane_off + 256u + (uint32_t)c, ov);
+          tmem_ld_wait();
+          float o[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = f32(ov[e]) * f;
+          tmem_st32(tmem + lane_off + 256u + (uint32_t)c, o);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        l *= f;
+      }
+      if (raise) m = mb;
+      const uint32_t box = sP + (uint32_t)pb * 4 * AT_BOX + (uint32_t)hs * AT_BOX;
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
         // P = hi + lo: hi = P with its low 16 bits cleared (a bf16 value), lo = P - hi
         // (exact) rounded to bf16, so P is carried to about 2^-16 relative
         uint32_t hb[32];
         float lo[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-          float p = ex2_approx(fmaf(f32(v[c & 1][e]), scale2, -m));
-          if (valid < 128 && 32 * c + e >= valid) p = 0.f;
-          l += p;
-          hb[e] = __float_as_uint(p) & 0xFFFF0000u;
-          lo[e] = p - __uint_as_float(hb[e]);
+          float pv = ex2_approx(fmaf(f32(v[c][e]), scale2, -m));
+          if (32 * c + e >= valid) pv = 0.f;
+          l += pv;
+          hb[e] = __float_as_uint(pv) & 0xFFFF0000u;
+          lo[e] = pv - __uint_as_float(hb[e]);
         }
-        const uint32_t box = pbase + (uint32_t)(c >> 1) * AT_BOX;
-        const int k0 = (c & 1) * 4;
+        const int k0 = c * 4;
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           st_shared_v4(box + swz(r, k0 + k), __byte_perm(hb[8 * k], hb[8 * k + 1], 0x7632),
@@ -366,11 +375,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       tc_fence_before();
       fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(s_empty0 + 8 * sb);
-        mbar_arrive(p_full0 + 8 * pb);
-      }
-      ++si;
+      if (lane == 0) mbar_arrive(p_full0 + 8 * pb);
     }
     // the row sum over both halves, half 0 + half 1 (a fixed order)
     red[hs * 128 + r] = l;
