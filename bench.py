@@ -16,6 +16,14 @@ committed in exactly those K steps.  Per-kernel times come from a second pass of
 same steps with timing events captured around every kernel.  `e2e` runs whole
 generations through the public API (prompt from pinned host memory, result read back).
 
+Under full recompute the line also carries `ms_per_step_at_p`: one step timed from the
+trajectory's states at p - N = 0, M/4, M/2, 3M/4 (set back each time), so that the step
+cost is read at fixed positions as well as over the trajectory.
+
+--workload accept times the acceptance pass alone (dcl_accept on seeded bf16 logits
+[64][32][126464], window 16) against the HBM roofline of the uncommitted logit rows it
+must read.
+
 --impl reference times the CPU oracle (tests' reference implementation) on a bounded
 sample of the same step on the host cores.
 """
@@ -65,6 +73,10 @@ WORKLOADS = {
     # 2-layer test model (latency-bound)
     "tiny": dict(shape="tiny", batch=1, n_prompt=32, gen=64, block=32, window=32,
                  seed=0, lm_scale=40.0, tau_c=0.70, tau_d=0.98),
+    # the acceptance pass alone on given bf16 logits: 64 sequences x 32 block positions x
+    # vocabulary 126464, window 16 (so that the draft region is exercised)
+    "accept": dict(kind="accept", batch=64, positions=32, vocab=126464, window=16, seed=7,
+                   tau_c=0.70, tau_d=0.98),
 }
 
 
@@ -313,6 +325,15 @@ def aggregate_replicas(ms, tokens, e2e_s, dist=None, device="cuda"):
             _allreduce(e2e_s, "max", dist, device))
 
 
+def _gpu_uuid(torch, local):
+    """The GPU's UUID as nvidia-smi names it (None when torch does not report one)."""
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        return None
+
+
 # ---------------------------------------------------------------------- our arm
 def run_ours(args):
     import torch
@@ -344,12 +365,22 @@ def run_ours(args):
                             block_len=wl["block"], gen_len=M, kv_cache=cached)
     ctx.set_prompt(prompt, cfg)
 
-    # one generation step by step: the trajectory (tokens committed per step) + warm-up
+    # one generation step by step: the trajectory (tokens committed per step) + warm-up.
+    # Under full recompute the states at p - N = 0, M/4, M/2, 3M/4 (the slowest row; the
+    # first state at or past each mark) are kept for the fixed-state step timings.
+    marks = [] if cached else [0, M // 4, M // 2, 3 * M // 4]
+    snaps = []
     ks, kper = [], []
+    p_host = np.full(B, N, np.int64)
     while sum(ks) < B * M and len(ks) < 4 * M:
+        if marks and int(p_host.min()) - N >= marks[0]:
+            snaps.append(ctx.get_state())
+            while marks and int(p_host.min()) - N >= marks[0]:
+                marks.pop(0)
         kr = ctx.step(return_k=True)
         kper.append(kr.copy())
         ks.append(int(kr.sum()))
+        p_host += kr
     S = len(ks)
     ctx.restart()
     for _ in range(args.warmup):
@@ -379,13 +410,7 @@ def run_ours(args):
         assert int((p - N).sum()) == sum(ks[:j]), "step trajectory did not replay deterministically"
         return t0.elapsed_time(t1), tokens
 
-    uuid = None
-    try:
-        uuid = str(torch.cuda.get_device_properties(local).uuid)
-        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
-    except Exception:
-        uuid = None
-    sampler = ClockSampler(uuid)
+    sampler = ClockSampler(_gpu_uuid(torch, local))
     sampler.start()
     ms, tokens = timed(args.steps)
     clocks = sampler.stop()
@@ -395,6 +420,21 @@ def run_ours(args):
     ms_prof, _ = timed(min(args.steps, max(3, S)))
     kern_ms, kern_kind = ctx.profile_last_step()
     ctx.set_profiling(False)
+
+    # one step from each kept state (set_state, then one step between CUDA events), median
+    # of 5: the step's cost at fixed positions, apart from the trajectory's dynamics
+    at_p = []
+    for xs, ps in snaps:
+        t = []
+        for _ in range(5):
+            ctx.set_state(xs, ps)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            ctx.step()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            t.append(e0.elapsed_time(e1))
+        at_p.append({"p_minus_n": int(ps.min()) - N, "ms": statistics.median(t)})
 
     # e2e through the public API: set_prompt (pinned host prompt) + generate (pinned out)
     pin_prompt = torch.from_numpy(prompt.copy()).pin_memory().numpy()
@@ -481,6 +521,7 @@ def run_ours(args):
                      "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
                      "avg_launch_ms": avg_ms, "flops_per_launch": flops_launch},
         "kernels": table,
+        "ms_per_step_at_p": at_p or None,
         "ms_per_step_profiled": ms_prof / min(args.steps, max(3, S)),
         "gpu_launches": args.steps * len(kern_ms),
         "clocks": clocks,
@@ -496,6 +537,198 @@ def run_ours(args):
     ctx.close()
     if dist:
         dist.destroy_process_group()
+    return 0
+
+
+# ---------------------------------------------------------------------- acceptance pass alone
+ACCEPT_METRIC = ("uncommitted block positions decided/s by the acceptance pass on bf16 logits, 1×GB300; "
+                 "% HBM roofline")
+
+
+def _accept_config(wl, args):
+    return {"workload": f"acceptance pass alone: bf16 logits [{wl['batch']}][{wl['positions']}][{wl['vocab']}] "
+                        f"(top-1 probability from a Beta mixture, committed prefixes uniform in "
+                        f"0..{wl['positions']}), window {wl['window']}, tau_commit {wl['tau_c']}, "
+                        f"tau_draft {wl['tau_d']}",
+            "global_batch": wl["batch"] * max(1, args.gpus), "seq_len": wl["positions"],
+            "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single",
+            "l2": "no flush needed: every call streams the uncommitted logit rows (240 MB > 129 MB L2)"}
+
+
+def _accept_data(wl, rank=0, nseq=None):
+    """Seeded inputs of the acceptance pass (logits of the first `nseq` sequences only when
+    given) and the number of uncommitted positions among those sequences."""
+    import synthetic as syn
+    V, P = wl["vocab"], wl["positions"]
+    nseq = nseq or wl["batch"]
+    only = None if nseq == wl["batch"] else {(b, i) for b in range(nseq) for i in range(P)}
+    d = syn.accept_inputs(wl["seed"] + rank, wl["batch"], P, V, V - 1, rows=only)
+    rows = int(np.clip(P - d["committed"][:nseq], 0, None).sum())
+    return d, rows
+
+
+def _accept_oracle_seconds(wl, d, nseq=None):
+    """The oracle's acceptance pass over the first `nseq` sequences (all by default), one
+    call (fp64 numpy); the bf16 -> float conversion is not timed."""
+    import synthetic as syn
+    from oracle import accept, decode
+    nseq = nseq or wl["batch"]
+    z = syn.bf16_to_f32(d["logits_bf16"][:nseq])
+    cfg = decode.DecodeConfig(tau_commit=wl["tau_c"], tau_draft=wl["tau_d"], max_window=wl["window"],
+                              gen_len=wl["positions"])
+    t0 = time.perf_counter()
+    accept.accept(z, d["committed"][:nseq], d["x"][:nseq], cfg, wl["window"])
+    return time.perf_counter() - t0
+
+
+def run_accept(args):
+    """dcl_accept on the config's logits: K calls back to back on the context stream.
+
+    A call is the two launches of the acceptance pass (softmax statistics of every
+    uncommitted position, then the contiguous commit and drafts); its algorithmic bytes
+    are the uncommitted logit rows, each read once.  Repeated calls see the same inputs
+    and write the same outputs (K depends on the logits and the committed prefix only)."""
+    import torch
+
+    wl = WORKLOADS[args.workload]
+    rank, world, local = _env_int("RANK", 0), _env_int("WORLD_SIZE", 1), _env_int("LOCAL_RANK", 0)
+    dist = None
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if local == 0:
+        import __graft_entry__
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    import paper_2607_20467_gb300 as dcl
+
+    B, P, V = wl["batch"], wl["positions"], wl["vocab"]
+    d, rows = _accept_data(wl, rank)
+    stream = torch.cuda.Stream()
+    ctx = dcl.Context(None, 1, 1, stream=stream.cuda_stream)
+    cfg = dcl.decode_config(tau_commit=wl["tau_c"], tau_draft=wl["tau_d"], max_window=wl["window"], gen_len=P)
+    host_logits = torch.from_numpy(d["logits_bf16"].view(np.int16)).pin_memory()
+    host_committed = torch.from_numpy(d["committed"]).pin_memory()
+    host_x = torch.from_numpy(d["x"].copy()).pin_memory()
+    with torch.cuda.stream(stream):
+        logits = host_logits.to("cuda", non_blocking=True).view(torch.bfloat16)
+        committed = host_committed.to("cuda", non_blocking=True)
+        x = host_x.to("cuda", non_blocking=True)
+        k = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    stream.synchronize()
+
+    for _ in range(args.warmup):
+        ctx.accept(logits, committed, x, cfg, k)
+    stream.synchronize()
+    k_ref, x_ref = k.clone(), x.clone()
+    torch.cuda.synchronize()
+
+    if dist:
+        dist.barrier()
+    sampler = ClockSampler(_gpu_uuid(torch, local))
+    sampler.start()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        ctx.accept(logits, committed, x, cfg, k)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    if dist:
+        dist.barrier()
+    ms = t0.elapsed_time(t1)
+    assert torch.equal(k, k_ref) and torch.equal(x, x_ref), "repeated acceptance calls differ"
+
+    # e2e: host logits / state in, K and x out, through the same call
+    out_k = torch.zeros(B, dtype=torch.int32).pin_memory()
+    out_x = torch.zeros((B, P), dtype=torch.int32).pin_memory()
+    e2e = []
+    for _ in range(args.e2e_iters):
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t = time.perf_counter()
+        with torch.cuda.stream(stream):
+            logits.view(torch.int16).copy_(host_logits, non_blocking=True)
+            committed.copy_(host_committed, non_blocking=True)
+            x.copy_(host_x, non_blocking=True)
+            ctx.accept(logits, committed, x, cfg, k)
+            out_k.copy_(k, non_blocking=True)
+            out_x.copy_(x, non_blocking=True)
+        stream.synchronize()
+        e2e.append(time.perf_counter() - t)
+    assert torch.equal(out_k, k_ref.cpu()) and torch.equal(out_x, x_ref.cpu())
+
+    rows_all = _allreduce(float(rows * args.steps), "sum", dist, "cuda")
+    ms_max = _allreduce(ms, "max", dist, "cuda")
+    e2e_s = _allreduce(statistics.mean(e2e), "max", dist, "cuda")
+    e2e_rows = _allreduce(float(rows), "sum", dist, "cuda")
+    peaks = _peaks()
+    ms_call = ms / args.steps
+    algo_bytes = rows * V * 2
+    achieved = algo_bytes / (ms_call / 1e3) / 1e9
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        s = _accept_oracle_seconds(wl, d)
+        cpu = {"value": rows / s, "unit": "positions/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"the whole workload once ({rows} uncommitted positions of {B * P}); fp64 numpy, "
+                         "bf16 -> float conversion untimed", "ms_per_step": 1e3 * s}
+    line = {
+        "metric": ACCEPT_METRIC, "value": rows_all / (ms_max / 1e3), "unit": "positions/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": f"synthetic: seeded bf16 logits (seed {wl['seed']}), random drafts and committed prefixes",
+        "config": _accept_config(wl, argparse.Namespace(gpus=world)),
+        "uncommitted_positions": rows,
+        "roofline": {"kernel": "accept (statistics + commit launches, timed together)", "bound": "hbm",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                     "peak_source": f"{peaks['source']} HBM copy (kernel timed alone)",
+                     "avg_launch_ms": ms_call, "bytes_per_launch": algo_bytes,
+                     "t_roof_ms": 1e3 * algo_bytes / (peaks["hbm_gbs"] * 1e9)},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clocks,
+        "e2e": {"value": e2e_rows / e2e_s, "unit": "positions/s",
+                "h2d_bytes_per_step": host_logits.numel() * 2 + 4 * B + 4 * B * P,
+                "d2h_bytes_per_step": 4 * B + 4 * B * P,
+                "step": "logits, committed prefixes and x copied in, one dcl_accept call, K and x copied out",
+                "ms_per_step": 1e3 * e2e_s},
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+    ctx.close()
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_accept_reference(args):
+    if _env_int("RANK", 0) != 0:
+        return 0
+    wl = WORKLOADS[args.workload]
+    nseq = wl["batch"]  # the whole workload per step (~1 s of CPU work)
+    d, rows = _accept_data(wl)
+    for _ in range(args.warmup):
+        _accept_oracle_seconds(wl, d, nseq)
+    secs = [_accept_oracle_seconds(wl, d, nseq) for _ in range(args.steps)]
+    s = statistics.mean(secs)
+    v = rows / s
+    line = {
+        "impl": "reference", "metric": ACCEPT_METRIC, "value": v, "unit": "positions/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * s, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": _accept_config(wl, args),
+        "cpu_baseline": {"value": v, "unit": "positions/s", "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": f"the whole workload per step ({nseq} sequences, {rows} uncommitted "
+                                   "positions); fp64 numpy, bf16 -> float conversion untimed",
+                         "cpu_seconds_timed": sum(secs)},
+        "e2e": {"value": v, "unit": "positions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
     return 0
 
 
@@ -585,11 +818,14 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    accept_only = WORKLOADS[args.workload].get("kind") == "accept"
     if args.sweep:
+        if accept_only:
+            ap.error("--sweep runs the decoding workloads only")
         return run_sweep(args)
     if args.impl == "reference":
-        return run_reference(args)
-    return run_ours(args)
+        return run_accept_reference(args) if accept_only else run_reference(args)
+    return run_accept(args) if accept_only else run_ours(args)
 
 
 if __name__ == "__main__":

@@ -362,54 +362,83 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
 }
 
 // ------------------------------------------------------------------ block acceptance
-template <int THREADS>
-__global__ void __launch_bounds__(THREADS) accept_stats_kernel(
+// One column into a thread's online partial (columns arrive in increasing order).  ENT
+// keeps the entropy sum u (needed only for the entropy confidence).
+template <bool ENT>
+__device__ __forceinline__ void take1(Part& a, float v, int col) {
+  if (v > a.m) {
+    const float d = (a.m - v) * kLog2e;  // -inf for the first column
+    const float e = exp2f(d);
+    if (ENT) a.u = a.s > 0.f ? e * fmaf(d, a.s, a.u) : 0.f;
+    a.s = a.s * e + 1.f;
+    a.t2 = a.m;
+    a.m = v;
+    a.id = col;
+  } else if (a.m != -INFINITY) {
+    if (v > a.t2) a.t2 = v;
+    const float y = (v - a.m) * kLog2e;
+    const float e = exp2f(y);
+    a.s += e;
+    if (ENT) a.u = fmaf(e, fmaxf(y, -200.f), a.u);  // e = 0 below -149: the term's limit 0
+  }
+}
+
+// Eight consecutive columns (one 16-byte vector).  When none of them exceeds the running
+// maximum, every column takes take1's second branch: the same operations in the same
+// order, without a compare and branch per column.
+template <bool ENT>
+__device__ __forceinline__ void take8(Part& a, const uint4& q, int col) {
+  const float v[8] = {bf16_lo(q.x), bf16_hi(q.x), bf16_lo(q.y), bf16_hi(q.y),
+                      bf16_lo(q.z), bf16_hi(q.z), bf16_lo(q.w), bf16_hi(q.w)};
+  const float cm = fmaxf(fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3])), fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7])));
+  if (cm > a.m || a.m == -INFINITY) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) take1<ENT>(a, v[k], col + k);
+    return;
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    a.t2 = fmaxf(a.t2, v[k]);
+    const float y = (v[k] - a.m) * kLog2e;
+    const float e = exp2f(y);
+    a.s += e;
+    if (ENT) a.u = fmaf(e, fmaxf(y, -200.f), a.u);
+  }
+}
+
+// One CTA of THREADS per position: thread t takes the 16-byte vectors t, t + THREADS, ...
+// of the row, ACC_AHEAD of them loaded before any is used (several loads in flight per
+// thread: with one, the latency of each load paced the thread).  256 threads and at
+// most 32 registers keep eight CTAs, so that ~1200 rows, resident on the 152 SMs at once.
+constexpr int ACC_THREADS = 256;
+constexpr int ACC_AHEAD = 4;
+template <int THREADS, bool ENT>
+__global__ void __launch_bounds__(THREADS, 2048 / THREADS) accept_stats_kernel(
     const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int P, int V,
     int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2, int mode) {
   const int pos = blockIdx.x;  // b * P + i
   const int b = pos / P, i = pos % P;
   if (i < committed[b]) return;  // committed positions are never read
   const __nv_bfloat16* row = logits + (size_t)pos * V;
-  // per-thread online (max, sum, argmax, second, entropy sum) over a strided slice of the row
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
-  auto take = [&](float v, int col) {
-    if (v > a.m) {
-      const float d = (a.m - v) * kLog2e;  // -inf for the first column
-      const float e = exp2f(d);
-      a.u = a.s > 0.f ? e * fmaf(d, a.s, a.u) : 0.f;
-      a.s = a.s * e + 1.f;
-      a.t2 = a.m;
-      a.m = v;
-      a.id = col;
-    } else if (a.m != -INFINITY) {
-      if (v > a.t2) a.t2 = v;
-      const float y = (v - a.m) * kLog2e;
-      const float e = exp2f(y);
-      a.s += e;
-      a.u = fmaf(e, fmaxf(y, -200.f), a.u);  // e = 0 below -149: the term's limit 0
-    }
-  };
   const bool vec = ((reinterpret_cast<uintptr_t>(row) & 15) == 0);
   int done = 0;
   if (vec) {
     const uint4* r4 = reinterpret_cast<const uint4*>(row);
     const int n8 = V / 8;
-    for (int j = threadIdx.x; j < n8; j += THREADS) {
-      const uint4 v = __ldcs(r4 + j);  // streamed once: do not keep in L2
-      const int col = j * 8;
-      take(bf16_lo(v.x), col + 0);
-      take(bf16_hi(v.x), col + 1);
-      take(bf16_lo(v.y), col + 2);
-      take(bf16_hi(v.y), col + 3);
-      take(bf16_lo(v.z), col + 4);
-      take(bf16_hi(v.z), col + 5);
-      take(bf16_lo(v.w), col + 6);
-      take(bf16_hi(v.w), col + 7);
+    int j = threadIdx.x;
+    for (; j + (ACC_AHEAD - 1) * THREADS < n8; j += ACC_AHEAD * THREADS) {
+      uint4 q[ACC_AHEAD];
+#pragma unroll
+      for (int t = 0; t < ACC_AHEAD; ++t) q[t] = __ldcs(r4 + j + t * THREADS);
+#pragma unroll
+      for (int t = 0; t < ACC_AHEAD; ++t) take8<ENT>(a, q[t], (j + t * THREADS) * 8);
     }
+    for (; j < n8; j += THREADS) take8<ENT>(a, __ldcs(r4 + j), j * 8);  // streamed once
     done = n8 * 8;
   }
   const unsigned short* r2 = reinterpret_cast<const unsigned short*>(row);
-  for (int j = done + threadIdx.x; j < V; j += THREADS) take(__uint_as_float((uint32_t)r2[j] << 16), j);
+  for (int j = done + threadIdx.x; j < V; j += THREADS) take1<ENT>(a, __uint_as_float((uint32_t)r2[j] << 16), j);
   // a thread's columns arrive in increasing order, so its argmax is its lowest maximal
   // column; merge() breaks ties between threads by the lower id
 #pragma unroll
@@ -523,7 +552,12 @@ cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* s
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
                                 int V, int32_t* ids, float* c1, float* c2, int mode, cudaStream_t stream) {
-  accept_stats_kernel<512><<<B * P, 512, 0, stream>>>(logits, committed, P, V, ids, c1, c2, mode);
+  if (mode)
+    accept_stats_kernel<ACC_THREADS, true><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, P, V, ids, c1, c2,
+                                                                             mode);
+  else
+    accept_stats_kernel<ACC_THREADS, false><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, P, V, ids, c1, c2,
+                                                                              mode);
   return cudaGetLastError();
 }
 

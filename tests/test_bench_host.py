@@ -1,0 +1,75 @@
+"""Host-side arithmetic of bench.py: the algorithmic work a step is credited with, the
+rows a cached step computes, and the inputs and bounds of the acceptance workload.
+"""
+import os
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+import synthetic as syn  # noqa: E402
+
+
+def test_step_work_of_the_llada8b_shape():
+    """Batch 1, prompt 256, gen 256: 7.147 TFLOP of linear layers, 0.137 of attention
+    (4 T^2 h H per layer), 0.265 of LM head over the 256 generation rows; 13.96 GB of layer
+    weights plus the 1.036 GB LM head streamed once per step."""
+    _, total, bytes_ = bench.step_work(syn.SHAPES["llada8b"], 1, 256, 256)
+    linear = sum(v for k, v in total.items() if k.startswith("gemm") and k != "gemm_lmhead")
+    assert linear == pytest.approx(7.147e12, rel=1e-3)
+    assert total["attention"] == pytest.approx(4 * 512 ** 2 * 128 * 32 * 32, rel=1e-12)
+    assert total["attention"] == pytest.approx(0.137e12, rel=5e-3)  # a 3-digit figure
+    assert total["gemm_lmhead"] == pytest.approx(0.265e12, rel=2e-3)
+    assert sum(total.values()) == pytest.approx(7.55e12, rel=2e-3)
+    lm = 2.0 * 126464 * 4096
+    assert lm == pytest.approx(1.036e9, rel=1e-3)
+    assert bytes_ - lm == pytest.approx(13.96e9 + 2 * 512 * 4096, rel=2e-3)
+
+
+def test_cached_rows_follow_the_refresh_rule():
+    """N = 4, M = 8, block 4: step 1 refreshes (all 12 rows, 8 at generation positions),
+    step 2 stays in the block [4, 8) and computes rows 4.., step 3 crosses into the next
+    block and refreshes again; a finished row computes nothing."""
+    out = bench.cached_rows([np.array([1]), np.array([3]), np.array([4])], 4, 8, 4)
+    assert out == [(12, 8), (8, 8), (12, 8)]
+    out = bench.cached_rows([np.array([8, 1]), np.array([0, 1])], 4, 8, 4)
+    assert out == [(24, 16), (8, 8)]
+
+
+def test_accept_inputs_and_their_uncommitted_rows():
+    wl = bench.WORKLOADS["accept"]
+    d, rows = bench._accept_data(wl, 0, nseq=2)
+    P, V = wl["positions"], wl["vocab"]
+    assert d["logits_bf16"].shape == (wl["batch"], P, V)
+    assert rows == int((P - d["committed"][:2]).sum())
+    # only the sampled sequences carry logits; their realised top-1 sits at the drawn index
+    assert not d["logits_bf16"][2:].any()
+    for b in range(2):
+        for i in range(P):
+            z = syn.bf16_to_f32(d["logits_bf16"][b, i])
+            assert int(np.argmax(z)) == int(d["top_index"][b, i])
+    assert bench._accept_oracle_seconds(wl, d, 2) > 0
+    cfg = bench._accept_config(wl, type("A", (), {"gpus": 1})())
+    assert cfg["global_batch"] == 64 and cfg["seq_len"] == 32 and cfg["parallelism"] == "single"
+
+
+def test_accept_algorithmic_bytes():
+    """The acceptance pass must read every uncommitted logit row once: for the seeded
+    workload 948 of the 2048 positions, 948 x 126464 x 2 B = 239.8 MB (35.3 us at the
+    measured 6793.8 GB/s)."""
+    wl = bench.WORKLOADS["accept"]
+    d, rows = bench._accept_data(wl, 0, nseq=1)  # committed prefixes of all 64 sequences
+    total = int((wl["positions"] - d["committed"]).sum())
+    assert total == 948
+    assert total * wl["vocab"] * 2 == pytest.approx(239.8e6, rel=1e-3)
+
+
+def test_sweep_refuses_the_acceptance_workload():
+    r = subprocess.run([sys.executable, "bench.py", "--workload", "accept", "--sweep"], cwd=ROOT,
+                       capture_output=True, text=True, timeout=120)
+    assert r.returncode == 2 and "decoding workloads" in r.stderr
