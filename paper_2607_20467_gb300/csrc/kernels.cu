@@ -11,6 +11,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "tc_ptx.cuh"
 
 namespace dcl {
 namespace {
@@ -383,24 +384,44 @@ __device__ __forceinline__ void take1(Part& a, float v, int col) {
   }
 }
 
-// Eight consecutive columns (one 16-byte vector).  When none of them exceeds the running
-// maximum, every column takes take1's second branch: the same operations in the same
-// order, without a compare and branch per column.
+// Eight consecutive columns (one 16-byte vector), without a branch per column: the
+// vector's maximum first (a new running maximum rescales s and u once, and takes the
+// lowest column holding it as the argmax), then every column adds exp2((z - m) log2 e)
+// on the special-function unit.  The argmax's own term is exp2 of the rounding residual
+// of the fused multiply-add, within an ulp of 1 (write_conf clamps p1 and p2).  A vector
+// holding an infinity takes the exact column-by-column path.
 template <bool ENT>
 __device__ __forceinline__ void take8(Part& a, const uint4& q, int col) {
   const float v[8] = {bf16_lo(q.x), bf16_hi(q.x), bf16_lo(q.y), bf16_hi(q.y),
                       bf16_lo(q.z), bf16_hi(q.z), bf16_lo(q.w), bf16_hi(q.w)};
   const float cm = fmaxf(fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3])), fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7])));
-  if (cm > a.m || a.m == -INFINITY) {
+  if (!(fabsf(cm) < INFINITY)) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) take1<ENT>(a, v[k], col + k);
     return;
   }
+  if (cm > a.m) {
+    int k0 = 7;
+#pragma unroll
+    for (int k = 6; k >= 0; --k) k0 = v[k] == cm ? k : k0;  // lowest column holding the maximum
+    float s2 = -INFINITY;  // largest of the other seven
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s2 = k == k0 ? s2 : fmaxf(s2, v[k]);
+    const float d = (a.m - cm) * kLog2e;  // -inf before the first vector
+    const float e = exp2f(d);
+    if (ENT) a.u = a.s > 0.f ? e * fmaf(d, a.s, a.u) : 0.f;
+    a.s *= e;
+    a.t2 = fmaxf(a.m, s2);
+    a.m = cm;
+    a.id = col + k0;
+  } else {
+    a.t2 = fmaxf(a.t2, cm);
+  }
+  const float ml = a.m * kLog2e;
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
-    a.t2 = fmaxf(a.t2, v[k]);
-    const float y = (v[k] - a.m) * kLog2e;
-    const float e = exp2f(y);
+    const float y = fmaf(v[k], kLog2e, -ml);
+    const float e = ex2_approx(y);
     a.s += e;
     if (ENT) a.u = fmaf(e, fmaxf(y, -200.f), a.u);
   }
