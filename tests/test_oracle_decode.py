@@ -283,3 +283,38 @@ def test_contiguous_drafts_subset_of_default():
         decode.commit_and_draft(xb, p, ids, c, cfg_b, L)
         changed_b = xb != x0
         assert (xa[changed_b] == xb[changed_b]).all()
+
+
+def test_remask_sets_exactly_the_clipped_window():
+    """Eq. remasking: positions [p, p + L) become MASK, clipped to the sequence end; nothing
+    else changes (checked against a per-position rule on every p and L of a short row)."""
+    T, mask = 12, 99
+    base = np.arange(T, dtype=np.int32)
+    for p in range(T + 1):
+        for L in range(1, T + 3):
+            x = base.copy()
+            decode.remask(x, p, L, mask)
+            for i in range(T):
+                assert x[i] == (mask if p <= i < p + L else base[i])
+
+
+def test_prefix_end_is_the_start_of_the_current_block():
+    """N + Bk floor((p - N) / Bk): the largest block boundary (counted from N) not above p."""
+    for N in (0, 3, 32):
+        for Bk in (1, 4, 32):
+            for p in range(N, N + 5 * Bk + 3):
+                pe = decode.prefix_end(p, N, Bk)
+                assert N <= pe <= p < pe + Bk
+                assert (pe - N) % Bk == 0
+
+
+def test_decision_confidence_modes():
+    p1 = np.array([0.9, 0.5, 0.2])
+    H = np.array([0.0, np.log(2.0), np.log(5.0)])
+    np.testing.assert_array_equal(decode.decision_confidence(p1, None, decode.DecodeConfig(gen_len=3)), p1)
+    c = decode.decision_confidence(p1, H, decode.DecodeConfig(gen_len=3, confidence=1))
+    np.testing.assert_allclose(c, [1.0, 0.5, 0.2], rtol=1e-15)  # exp(-ln k) = 1/k
+    with pytest.raises(ValueError):
+        decode.decision_confidence(p1, None, decode.DecodeConfig(gen_len=3, confidence=1))
+    with pytest.raises(ValueError):
+        decode.decision_confidence(p1, H, decode.DecodeConfig(gen_len=3, confidence=2))
