@@ -152,6 +152,14 @@ def cached_rows(kper, N, M, block):
     return out
 
 
+def k_histogram(kper):
+    """{K: number of (step, row) pairs that committed K tokens} over a trajectory's per-row
+    K values; rows that had finished (K = 0) are left out."""
+    k = np.concatenate([np.asarray(v).ravel() for v in kper]) if kper else np.zeros(0, np.int64)
+    k = k[k > 0]
+    return {str(int(v)): int(n) for v, n in zip(*np.unique(k, return_counts=True))}
+
+
 # ---------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -512,6 +520,7 @@ def run_ours(args):
         "config": _config(wl, argparse.Namespace(gpus=world)),
         "steps_per_token": S / M,
         "trajectory_steps": S,
+        "k_histogram": k_histogram(kper),
         "tokens_in_timed_window": tokens,
         "step_roofline": {"flops": step_flops, "bytes": step_bytes, "t_roof_ms": 1e3 * t_roof,
                           "frac": 1e3 * t_roof / ms_step, "peak_tflops": peak,

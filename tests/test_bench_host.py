@@ -73,3 +73,12 @@ def test_sweep_refuses_the_acceptance_workload():
     r = subprocess.run([sys.executable, "bench.py", "--workload", "accept", "--sweep"], cwd=ROOT,
                        capture_output=True, text=True, timeout=120)
     assert r.returncode == 2 and "decoding workloads" in r.stderr
+
+
+def test_k_histogram_counts_active_rows_only():
+    kper = [np.array([3, 1]), np.array([1, 2]), np.array([0, 2]), np.array([0, 5])]
+    assert bench.k_histogram(kper) == {"1": 2, "2": 2, "3": 1, "5": 1}
+    assert bench.k_histogram([]) == {}
+    # the histogram's tokens are the trajectory's tokens
+    h = bench.k_histogram(kper)
+    assert sum(int(k) * n for k, n in h.items()) == sum(int(v.sum()) for v in kper)
