@@ -50,7 +50,7 @@ def _guarded(seed, B, P, V, taus, confidence=0):
 @pytest.mark.parametrize("B,P,V,L,contig,conf", [(8, 32, 4096, 16, 0, 0), (16, 32, 1000, 32, 0, 0),
                                                  (6, 40, 3001, 7, 1, 0), (64, 32, 126464, 16, 0, 0),
                                                  (64, 32, 126464, 32, 1, 0), (16, 32, 4096, 16, 0, 1),
-                                                 (32, 32, 126464, 16, 0, 1)])
+                                                 (32, 32, 126464, 16, 0, 1), (3, 4096, 1000, 2048, 0, 0)])
 def test_accept_bit_exact(ops, B, P, V, L, contig, conf):
     """conf = 1: the thresholds see exp(-H) (marginal entropy); the guard band then keeps
     exp(-H) 1e-4 away from them (H is summed in fp32 on the GPU, fp64 in the oracle)."""
@@ -81,6 +81,9 @@ def test_accept_rejects_bad_arguments(ops):
     st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 5000, 100, t.data_ptr(), t.data_ptr(), cfg,
                               t.data_ptr())
     assert st == dcl.DCL_ERR_INVALID_ARG
+    for B, P, V in ((0, 32, 100), (1, 0, 100), (1, 32, 1), (1 << 10, 1 << 11, 100)):  # empty, degenerate, > 2^20
+        st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), B, P, V, t.data_ptr(), t.data_ptr(), cfg, t.data_ptr())
+        assert st == dcl.DCL_ERR_INVALID_ARG
     bad = dcl.decode_config(gen_len=32, confidence=2)
     st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 32, 100, t.data_ptr(), t.data_ptr(), bad, t.data_ptr())
     assert st == dcl.DCL_ERR_INVALID_ARG
