@@ -82,3 +82,14 @@ def test_k_histogram_counts_active_rows_only():
     # the histogram's tokens are the trajectory's tokens
     h = bench.k_histogram(kper)
     assert sum(int(k) * n for k, n in h.items()) == sum(int(v.sum()) for v in kper)
+
+
+def test_l2_note_follows_the_weight_bytes():
+    assert "streams all weights" in bench._l2_note(bench.WORKLOADS["llada8b"])
+    assert "stay in the 129 MB L2" in bench._l2_note(bench.WORKLOADS["tiny"])
+
+
+def test_oracle_whole_generation_of_the_tiny_workload():
+    """The tiny workload's CPU baseline runs the oracle's Algorithm 1 to completion."""
+    s, steps, n = bench.oracle_generation(bench.WORKLOADS["tiny"], 0.0)
+    assert s > 0 and n == 1 and 1 <= steps <= 64
