@@ -189,9 +189,13 @@ dcl_status dcl_debug_hidden(dcl_ctx* ctx, int32_t layer, float* h_dev);
  *   committed_dev int32 [B]: c_b positions already committed (left-aligned), so the
  *                 window starts at p = c_b; rows with c_b >= P are left unchanged.
  *   x_dev         int32 [B][P], in/out: receives the committed ids and new drafts.
- *   cfg           thresholds, max_window (0 = P/2), min_commit, contiguous_drafts.
+ *   cfg           thresholds, max_window (0 = P/2), min_commit, contiguous_drafts,
+ *                 confidence (0: top-1 probability, 1: exp(-H) of the marginal entropy).
  *   k_dev         int32 [B] out: K of every row.
- * Async; P <= 4096, B*P <= 1<<20.  Errors: INVALID_ARG, CUDA. */
+ * Committed c_b and repeated calls: K depends on the logits and c_b only, so a second
+ * call on its own output writes the same x.  Async on the context stream; 1 <= B,
+ * 1 <= P <= 4096, B*P <= 1<<20, V >= 2.  Errors: INVALID_ARG (NULL pointer, sizes,
+ * confidence not 0/1), OOM (scratch), CUDA. */
 dcl_status dcl_accept(dcl_ctx* ctx, const void* logits_dev, int32_t B, int32_t P, int32_t V,
                       const int32_t* committed_dev, int32_t* x_dev, const dcl_decode_config* cfg,
                       int32_t* k_dev);
