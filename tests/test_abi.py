@@ -64,3 +64,14 @@ def test_product_path_never_imports_the_oracle():
                 src = open(os.path.join(dirpath, fn)).read()
                 assert not re.search(r"^\s*(from|import)\s+oracle\b", src, re.M), fn
                 assert "oracle/" not in src, fn
+
+
+def test_missing_library_fails_loudly(built, monkeypatch, tmp_path):
+    """With libdcleap.so absent the binding raises instead of falling back to anything."""
+    pkg = built
+    monkeypatch.setattr(pkg, "LIB_PATH", str(tmp_path / "libdcleap.so"))
+    monkeypatch.setattr(pkg, "_lib", None)
+    with pytest.raises(ImportError, match="no CPU fallback"):
+        pkg.lib()
+    with pytest.raises(ImportError):
+        pkg.Context(None, 1, 1)
