@@ -1,0 +1,198 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case plants one mistake in the oracle (on the CPU, by replacing one of its functions
+for the duration of the test) of the kind a reader could make when restating the paper:
+a dropped term, a wrong sign, index or axis, a transposed operand, `>=` for `>`.  The
+named pin tests, run against the planted oracle, must fail.  Nothing here touches the
+CUDA path.
+"""
+import numpy as np
+import pytest
+
+from oracle import decode, model
+
+import test_oracle_decode as tdec
+import test_oracle_entropy as tent
+import test_oracle_model as tmod
+
+ROOT_GOLDEN = __import__("os").path.join(__import__("os").path.dirname(__file__), "golden")
+
+
+# ----------------------------------------------------------------- planted mistakes
+
+def _rms_no_mean(x, gain, eps):  # sum of squares instead of their mean
+    x = np.asarray(x, dtype=np.float64)
+    return x / np.sqrt(np.sum(x * x, axis=-1, keepdims=True) + eps) * np.asarray(gain, np.float64)
+
+
+def _rms_eps_outside(x, gain, eps):  # eps added after the square root
+    x = np.asarray(x, dtype=np.float64)
+    return x / (np.sqrt(np.mean(x * x, axis=-1, keepdims=True)) + eps) * np.asarray(gain, np.float64)
+
+
+def _rope_wrong_sign(x, angles):  # rotation by -angle
+    half = x.shape[-1] // 2
+    c, s = np.cos(angles)[:, None, :], np.sin(angles)[:, None, :]
+    x1, x2 = x[..., :half], x[..., half:]
+    return np.concatenate([x1 * c + x2 * s, x2 * c - x1 * s], axis=-1)
+
+
+def _rope_interleaved(x, angles):  # pairs (2j, 2j + 1) instead of (j, j + hd/2)
+    c, s = np.cos(angles)[:, None, :], np.sin(angles)[:, None, :]
+    x1, x2 = x[..., 0::2], x[..., 1::2]
+    out = np.empty_like(x)
+    out[..., 0::2] = x1 * c - x2 * s
+    out[..., 1::2] = x2 * c + x1 * s
+    return out
+
+
+def _rope_angles_wrong_freq(n_pos, head_dim, theta):  # theta^(-j/hd) instead of theta^(-2j/hd)
+    j = np.arange(head_dim // 2, dtype=np.float64)
+    return np.outer(np.arange(n_pos, dtype=np.float64), theta ** (-1.0 * j / head_dim))
+
+
+def _attention_variant(causal=False, scale=True, gqa_mod=False, softmax_axis=1):
+    def att(q, k, v):
+        T, H, hd = q.shape
+        G = k.shape[1]
+        rep = H // G
+        out = np.empty((T, H, hd))
+        for h in range(H):
+            g = h % G if gqa_mod else h // rep
+            s = q[:, h, :] @ k[:, g, :].T
+            if scale:
+                s = s / np.sqrt(hd)
+            if causal:
+                s = s + np.triu(np.full((T, T), -np.inf), 1)
+            s = s - s.max(axis=softmax_axis, keepdims=True)
+            w = np.exp(s)
+            w = w / w.sum(axis=softmax_axis, keepdims=True)
+            out[:, h, :] = w @ v[:, g, :]
+        return out.reshape(T, H * hd)
+    return att
+
+
+def _silu_sigmoid(x):  # sigmoid instead of x * sigmoid
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def _block_without_mlp_residual(shape, lw, h, angles, bf16_operands=False):
+    T = h.shape[0]
+    H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    f = lambda a: np.asarray(a, np.float64)  # noqa: E731
+    xn = model.rms_norm(h, lw["attn_norm"], shape.rms_eps)
+    q = model.apply_rope((xn @ f(lw["wq"]).T).reshape(T, H, hd), angles)
+    k = model.apply_rope((xn @ f(lw["wk"]).T).reshape(T, G, hd), angles)
+    v = (xn @ f(lw["wv"]).T).reshape(T, G, hd)
+    h = h + model.attention(q, k, v) @ f(lw["wo"]).T
+    xn = model.rms_norm(h, lw["mlp_norm"], shape.rms_eps)
+    a = model.silu(xn @ f(lw["w_gate"]).T) * (xn @ f(lw["w_up"]).T)
+    return a @ f(lw["w_down"]).T  # the residual h dropped
+
+
+def _block_gate_up_swapped(shape, lw, h, angles, bf16_operands=False):
+    lw = dict(lw, w_gate=lw["w_up"], w_up=lw["w_gate"])
+    return _ORIG["block"](shape, lw, h, angles, bf16_operands)
+
+
+def _confidence_p2_includes_top(z):
+    ids, p1, _ = _ORIG["confidence"](z)
+    return ids, p1, p1.copy()  # the "second" is the top itself
+
+
+def _confidence_last_argmax(z):  # ties to the highest index
+    z = np.asarray(z, dtype=np.float64)
+    ids = z.shape[-1] - 1 - np.argmax(z[..., ::-1], axis=-1)
+    _, p1, p2 = _ORIG["confidence"](z)
+    return ids, p1, p2
+
+
+def _entropy_log2(z):  # bits instead of nats
+    return _ORIG["entropy"](z) / np.log(2.0)
+
+
+def _exceeds_ge(c, tau):  # c >= tau instead of c > tau
+    return np.asarray(c, dtype=np.float32) >= np.float32(tau)
+
+
+def _commit_drafts_from_p_plus_k(x, p, ids, c, cfg, window):  # future region from p + K
+    T = x.shape[0]
+    w_eff = min(window, T - p)
+    K = min(max(decode.window_length(c[p:p + w_eff], cfg.tau_commit), cfg.min_commit), w_eff)
+    x[p:p + K] = ids[p:p + K]
+    lo = p + K
+    ok = decode.exceeds(c[lo:T], cfg.tau_draft)
+    seg = x[lo:T]
+    seg[ok] = ids[lo:T][ok]
+    return K
+
+
+def _remask_shifted(x, p, window, mask_id):  # one position late
+    x[p + 1:min(p + 1 + window, x.shape[0])] = mask_id
+
+
+def _jpde_sum_only(H_set):  # the max term dropped
+    H_set = np.asarray(H_set, dtype=np.float64)
+    return float(H_set.sum()) if H_set.size >= 2 else 0.0
+
+
+_ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy}
+
+
+# ------------------------------------------------------ planted mistake -> its pins
+CASES = [
+    ("rms_norm sum not mean", model, "rms_norm", _rms_no_mean,
+     [tmod.test_rms_norm_unit_rms_and_library, tmod.test_tiny_forward_matches_torch_restatement]),
+    ("rms_norm eps outside sqrt", model, "rms_norm", _rms_eps_outside,
+     [tmod.test_rms_norm_unit_rms_and_library]),
+    ("rope wrong sign", model, "apply_rope", _rope_wrong_sign,
+     [tmod.test_rope_is_complex_rotation, tmod.test_tiny_forward_matches_torch_restatement]),
+    ("rope interleaved pairs", model, "apply_rope", _rope_interleaved,
+     [tmod.test_rope_is_complex_rotation, tmod.test_tiny_forward_matches_torch_restatement]),
+    ("rope frequency exponent", model, "rope_angles", _rope_angles_wrong_freq,
+     [tmod.test_rope_is_complex_rotation, tmod.test_tiny_forward_matches_torch_restatement]),
+    ("attention causal", model, "attention", _attention_variant(causal=True),
+     [tmod.test_attention_matches_library_non_causal_gqa, tmod.test_attention_special_cases,
+      tmod.test_forward_is_bidirectional]),
+    ("attention unscaled", model, "attention", _attention_variant(scale=False),
+     [tmod.test_attention_matches_library_non_causal_gqa]),
+    ("attention GQA head map", model, "attention", _attention_variant(gqa_mod=True),
+     [tmod.test_attention_matches_library_non_causal_gqa, tmod.test_gqa_forward_matches_torch_restatement]),
+    ("attention softmax over queries", model, "attention", _attention_variant(softmax_axis=0),
+     [tmod.test_attention_matches_library_non_causal_gqa]),
+    ("silu as sigmoid", model, "silu", _silu_sigmoid,
+     [tmod.test_silu_matches_library, tmod.test_tiny_forward_matches_torch_restatement]),
+    ("block drops the MLP residual", model, "block", _block_without_mlp_residual,
+     [tmod.test_tiny_forward_matches_torch_restatement]),
+    ("block swaps gate and up", model, "block", _block_gate_up_swapped,
+     [tmod.test_tiny_forward_matches_torch_restatement]),
+    ("p2 includes the top-1", model, "confidence", _confidence_p2_includes_top,
+     [tmod.test_confidence_matches_library_softmax]),
+    ("argmax ties to the highest id", model, "confidence", _confidence_last_argmax,
+     [tmod.test_confidence_tie_gives_equal_top2]),
+    ("entropy in bits", model, "entropy", _entropy_log2,
+     [lambda: tent.test_entropy_uniform_is_log_v(8), tent.test_entropy_matches_scipy_on_random_rows]),
+    (">= instead of >", decode, "exceeds", _exceeds_ge,
+     [tdec.test_window_length_equals_first_failure_brute_force]),
+    ("drafts from p + K", decode, "commit_and_draft", _commit_drafts_from_p_plus_k,
+     [lambda: tdec.test_golden_scripted_trajectories(ROOT_GOLDEN)]),
+    ("remask one late", decode, "remask", _remask_shifted,
+     [tdec.test_remask_sets_exactly_the_clipped_window, lambda: tdec.test_golden_scripted_trajectories(ROOT_GOLDEN)]),
+    ("entropy bound without the max", decode, "jpde_bound", _jpde_sum_only,
+     [tent.test_jpde_bound_special_cases]),
+]
+
+
+@pytest.mark.parametrize("name,mod,attr,bad,pins", CASES, ids=[c[0] for c in CASES])
+def test_planted_mistake_fails_its_pins(monkeypatch, name, mod, attr, bad, pins):
+    monkeypatch.setattr(mod, attr, bad)
+    for pin in pins:
+        with pytest.raises(AssertionError):
+            pin()
+
+
+@pytest.mark.parametrize("name,mod,attr,bad,pins", CASES, ids=[c[0] for c in CASES])
+def test_pins_pass_on_the_oracle_as_written(name, mod, attr, bad, pins):
+    """The same pins pass without the planted mistake (so the failures above are caused by it)."""
+    for pin in pins:
+        pin()
