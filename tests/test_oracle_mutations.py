@@ -9,8 +9,11 @@ CUDA path.
 import numpy as np
 import pytest
 
-from oracle import decode, model
+from oracle import accept, decode, model
 
+import synthetic as syn
+import test_oracle_accept as tacc
+import test_oracle_cache as tcache
 import test_oracle_decode as tdec
 import test_oracle_entropy as tent
 import test_oracle_model as tmod
@@ -136,7 +139,41 @@ def _jpde_sum_only(H_set):  # the max term dropped
     return float(H_set.sum()) if H_set.size >= 2 else 0.0
 
 
-_ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy}
+def _forward_rows_rope_at_row_index(shape, weights, tokens, pos, kv_store, bf16_operands=False):
+    """Suffix rows rotated by their index in the suffix, not their position in the sequence."""
+    pos = np.asarray(pos, dtype=np.int64)
+    h = np.asarray(weights["embed"], np.float64)[np.asarray(tokens)[pos]]
+    angles = model.rope_angles(len(pos), shape.head_dim, shape.rope_theta)
+    for lw, kv in zip(weights["layers"], kv_store):
+        h = model.block_rows(shape, lw, h, pos, kv, angles, bf16_operands)
+    return model.rms_norm(h, weights["final_norm"], shape.rms_eps)
+
+
+def _block_rows_no_store(shape, lw, h, pos, kv, angles, bf16_operands=False):
+    """The rows' fresh keys / values never reach the store their queries attend to."""
+    n = h.shape[0]
+    H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    f = lambda a: np.asarray(a, np.float64)  # noqa: E731
+    xn = model.rms_norm(h, lw["attn_norm"], shape.rms_eps)
+    q = model.apply_rope((xn @ f(lw["wq"]).T).reshape(n, H, hd), angles)
+    h = h + model.attention(q, kv[0], kv[1]) @ f(lw["wo"]).T
+    xn = model.rms_norm(h, lw["mlp_norm"], shape.rms_eps)
+    a = model.silu(xn @ f(lw["w_gate"]).T) * (xn @ f(lw["w_up"]).T)
+    return h + a @ f(lw["w_down"]).T
+
+
+def _accept_window_from_zero(logits, committed, x, cfg, window):
+    """The window taken from position 0 instead of the committed prefix."""
+    return _ORIG["accept"](logits, np.zeros_like(committed), x, cfg, window)
+
+
+def _prefix_end_unaligned(p, n_prompt, block_len):  # p itself, not the block boundary
+    return p
+
+
+_ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy,
+         "accept": accept.accept}
+_TINY_W = syn.model_weights(syn.SHAPES["tiny"], 0, lm_head_scale=40.0, norm_gain_std=0.1)
 
 
 # ------------------------------------------------------ planted mistake -> its pins
@@ -180,6 +217,15 @@ CASES = [
      [tdec.test_remask_sets_exactly_the_clipped_window, lambda: tdec.test_golden_scripted_trajectories(ROOT_GOLDEN)]),
     ("entropy bound without the max", decode, "jpde_bound", _jpde_sum_only,
      [tent.test_jpde_bound_special_cases]),
+    ("cache: RoPE at the row index", model, "forward_rows", _forward_rows_rope_at_row_index,
+     [lambda: tcache.test_suffix_with_fresh_store_equals_full_forward(_TINY_W, tcache.N + 32)]),
+    ("cache: fresh keys not stored", model, "block_rows", _block_rows_no_store,
+     [lambda: tcache.test_all_rows_equal_full_forward(_TINY_W, False)]),
+    ("acceptance window from position 0", accept, "accept", _accept_window_from_zero,
+     [tacc.test_accept_matches_brute_force]),
+    ("prefix end not block-aligned", decode, "prefix_end", _prefix_end_unaligned,
+     [tdec.test_prefix_end_is_the_start_of_the_current_block,
+      lambda: tcache.test_refresh_exactly_at_block_changes(_TINY_W)]),
 ]
 
 
