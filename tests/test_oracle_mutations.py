@@ -171,8 +171,29 @@ def _prefix_end_unaligned(p, n_prompt, block_len):  # p itself, not the block bo
     return p
 
 
+def _forward_without_final_norm(shape, weights, tokens, bf16_operands=False, upto_layer=None):
+    h = np.asarray(weights["embed"], np.float64)[np.asarray(tokens)]
+    if upto_layer == -1:
+        return h
+    angles = model.rope_angles(len(tokens), shape.head_dim, shape.rope_theta)
+    for li, lw in enumerate(weights["layers"]):
+        h = model.block(shape, lw, h, angles, bf16_operands)
+        if upto_layer == li:
+            return h
+    return h  # the final RMSNorm dropped
+
+
+def _entropy_confidence_wrong_sign(H):  # exp(+H)
+    return np.exp(np.asarray(H, dtype=np.float64))
+
+
+def _commit_drafts_ignore_chain(x, p, ids, c, cfg, window):  # App. E flag ignored
+    import dataclasses
+    return _ORIG["commit_and_draft"](x, p, ids, c, dataclasses.replace(cfg, contiguous_drafts=False), window)
+
+
 _ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy,
-         "accept": accept.accept}
+         "accept": accept.accept, "commit_and_draft": decode.commit_and_draft}
 _TINY_W = syn.model_weights(syn.SHAPES["tiny"], 0, lm_head_scale=40.0, norm_gain_std=0.1)
 
 
@@ -223,6 +244,13 @@ CASES = [
      [lambda: tcache.test_all_rows_equal_full_forward(_TINY_W, False)]),
     ("acceptance window from position 0", accept, "accept", _accept_window_from_zero,
      [tacc.test_accept_matches_brute_force]),
+    ("forward without the final RMSNorm", model, "forward_hidden", _forward_without_final_norm,
+     [tmod.test_tiny_forward_matches_torch_restatement, tmod.test_gqa_forward_matches_torch_restatement]),
+    ("entropy confidence exp(+H)", decode, "entropy_confidence", _entropy_confidence_wrong_sign,
+     [tent.test_entropy_shift_invariance_bounds_and_order, tdec.test_decision_confidence_modes]),
+    ("contiguous drafts ignored", decode, "commit_and_draft", _commit_drafts_ignore_chain,
+     [lambda: tdec.test_golden_scripted_trajectories(ROOT_GOLDEN),
+      lambda: tdec.test_golden_after_states_step_by_step(ROOT_GOLDEN)]),
     ("prefix end not block-aligned", decode, "prefix_end", _prefix_end_unaligned,
      [tdec.test_prefix_end_is_the_start_of_the_current_block,
       lambda: tcache.test_refresh_exactly_at_block_changes(_TINY_W)]),
