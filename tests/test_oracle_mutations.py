@@ -6,6 +6,9 @@ a dropped term, a wrong sign, index or axis, a transposed operand, `>=` for `>`.
 named pin tests, run against the planted oracle, must fail.  Nothing here touches the
 CUDA path.
 """
+import os
+from dataclasses import replace
+
 import numpy as np
 import pytest
 
@@ -18,7 +21,7 @@ import test_oracle_decode as tdec
 import test_oracle_entropy as tent
 import test_oracle_model as tmod
 
-ROOT_GOLDEN = __import__("os").path.join(__import__("os").path.dirname(__file__), "golden")
+ROOT_GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
 
 
 # ----------------------------------------------------------------- planted mistakes
@@ -188,8 +191,7 @@ def _entropy_confidence_wrong_sign(H):  # exp(+H)
 
 
 def _commit_drafts_ignore_chain(x, p, ids, c, cfg, window):  # App. E flag ignored
-    import dataclasses
-    return _ORIG["commit_and_draft"](x, p, ids, c, dataclasses.replace(cfg, contiguous_drafts=False), window)
+    return _ORIG["commit_and_draft"](x, p, ids, c, replace(cfg, contiguous_drafts=False), window)
 
 
 _ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy,
