@@ -93,3 +93,18 @@ def test_oracle_whole_generation_of_the_tiny_workload():
     """The tiny workload's CPU baseline runs the oracle's Algorithm 1 to completion."""
     s, steps, n = bench.oracle_generation(bench.WORKLOADS["tiny"], 0.0)
     assert s > 0 and n == 1 and 1 <= steps <= 64
+
+
+def test_step_work_of_a_cached_suffix_step():
+    """LLaDA-8B shape, prompt 512 + gen 1024, a cached step over 32 suffix rows: 6.98e9
+    linear weights per row (2 flops each), attention 4 q T h H per layer, and the stored
+    keys / values of all T = 1536 positions read once: 0.524 MB per position = 805 MB."""
+    sh = syn.SHAPES["llada8b"]
+    _, total, b_cached = bench.step_work(sh, 1, 512, 1024, rows=32, lm_rows=32, cached=True)
+    _, _, b_plain = bench.step_work(sh, 1, 512, 1024, rows=32, lm_rows=32, cached=False)
+    linear = sum(v for k, v in total.items() if k.startswith("gemm") and k != "gemm_lmhead")
+    assert linear == pytest.approx(2 * 6.98e9 * 32, rel=1e-3)
+    assert total["attention"] == 4.0 * 32 * 1536 * 4096 * 32
+    assert total["gemm_lmhead"] == 2.0 * 32 * 4096 * 126464
+    assert b_cached - b_plain == pytest.approx(0.524e6 * 1536, rel=1e-3)
+    assert b_cached - b_plain == pytest.approx(805e6, rel=1e-3)
