@@ -239,9 +239,7 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * tiles of a partly filled last round of the persistent grid are cut into about S K
  * segments each (S = 0: shared out over all CTA pairs) run by different pairs; rejected
  * with DCL_ERR_INVALID_ARG when the last round is full or a sharing pair would get no K
- * block; DCL_TILE_PAIR | DCL_TILE_MULTICAST clusters of two CTA pairs on consecutive
- * 256-row blocks that load each weight tile from L2 once (TMA multicast; M > 256);
- * DCL_TILE_PAIR | DCL_TILE_HALVES whole tiles in full rounds, then every tile of a partial
+ * block; DCL_TILE_PAIR | DCL_TILE_HALVES whole tiles in full rounds, then every tile of a partial
  * last round as two 256 x 128 pieces (no K split); DCL_TILE_PAIR | DCL_TILE_DSMEM clusters
  * of two CTA pairs: whole tiles in full rounds, then every left-over tile split by K over
  * one cluster's pairs, the upper half's fp32 sum added to the lower half's through
@@ -249,7 +247,6 @@ dcl_status dcl_op_rmsnorm(dcl_ctx* ctx, const float* x_dev, const void* gain_dev
  * Partial sums are always combined in K order, so every choice is deterministic. */
 #define DCL_TILE_PAIR 2
 #define DCL_TILE_STREAMK (1 << 16)
-#define DCL_TILE_MULTICAST (1 << 17)
 #define DCL_TILE_HALVES (1 << 18)
 #define DCL_TILE_DSMEM (1 << 19)
 

@@ -102,7 +102,6 @@ struct GemmPlan {
   int M = 0, N = 0, K = 0;
   int bn = 256;          // output columns per tile
   int cg = 1;            // 1: one CTA per 128 x bn tile; 2: a CTA pair per 256 x 256 tile
-  int mc = 0;            // cg 2: clusters of two pairs sharing the weight tile by multicast
   int epi = EPI_BF16;
   EpiParams ep;
   int grid = 0;
@@ -124,11 +123,9 @@ struct GemmPlan {
 // that width; kTilePair forces the CTA-pair 256 x 256 tile, kTilePair | (S << 8) that
 // tile with S K splits (S = 0: the planner chooses, S = 1: unsplit),
 // kTilePair | kTileStreamK | (S << 8) the pair tile with the stream-K schedule, each
-// left-over tile cut into about S K segments (S = 0: shared out over all pairs),
-// kTilePair | kTileMulticast clusters of two pairs that load each weight tile once.
+// left-over tile cut into about S K segments (S = 0: shared out over all pairs).
 constexpr int kTilePair = 2;
 constexpr int kTileStreamK = 1 << 16;
-constexpr int kTileMulticast = 1 << 17;  // with kTilePair: clusters of two pairs sharing W tiles
 constexpr int kTileHalves = 1 << 18;     // with kTilePair: left-over tiles as two half-width pieces
 constexpr int kTileDsmem = 1 << 19;      // with kTilePair: left-over tiles split by K over a cluster's pairs
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,

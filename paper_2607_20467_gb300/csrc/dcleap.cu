@@ -304,8 +304,8 @@ dcl_status build_graph(dcl_ctx* c) {
 // Tile of one of the step's GEMMs ("qkv", "o", "gateup", "down", "lmhead") forced by the
 // environment variable DCL_GEMM_TILES, e.g. "o=128,down=pair:2" (128 / 256 = one-CTA tile
 // width, pair[:S] = CTA-pair tile with S K-splits, pair:sk[:S] = CTA-pair tile with the
-// stream-K schedule, S segments per left-over tile, pair:mc[:S] = pairs sharing weight
-// tiles by multicast, S K-splits, pair:h = left-over tiles as half-width pieces, pair:ds =
+// stream-K schedule, S segments per left-over tile, pair:h = left-over tiles as
+// half-width pieces, pair:ds =
 // left-over tiles split by K over a cluster's two pairs); 0 = let the planner choose.
 int tile_override(const char* name) {
   const char* env = getenv("DCL_GEMM_TILES");
@@ -317,7 +317,6 @@ int tile_override(const char* name) {
     if (len > n && strncmp(s, name, n) == 0 && s[n] == '=') {
       const char* v = s + n + 1;
       if (strncmp(v, "pair:sk", 7) == 0) return kTilePair | kTileStreamK | ((v[7] == ':' ? atoi(v + 8) : 0) << 8);
-      if (strncmp(v, "pair:mc", 7) == 0) return kTilePair | kTileMulticast | ((v[7] == ':' ? atoi(v + 8) : 0) << 8);
       if (strcmp(v, "pair:h") == 0 || strncmp(v, "pair:h,", 7) == 0) return kTilePair | kTileHalves;
       if (strncmp(v, "pair:ds", 7) == 0) return kTilePair | kTileDsmem;
       if (strncmp(v, "pair", 4) == 0) return kTilePair | ((v[4] == ':' ? atoi(v + 5) : 0) << 8);

@@ -429,17 +429,6 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar_cluster)
       : "memory");
 }
-// The box lands at the same shared-memory offset in every CTA of cta_mask; each
-// destination's bytes complete on the mbarrier at bar's offset in the leader of that
-// destination's CTA pair (bar: the address of the issuing pair leader's barrier).
-__device__ __forceinline__ void tma_load_2d_pair_mc(uint32_t dst, const CUtensorMap* tm, int x, int y,
-                                                    uint32_t bar_cluster, uint16_t cta_mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar_cluster), "h"(cta_mask)
-      : "memory");
-}
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t holder, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(holder), "r"(ncols)
                : "memory");
@@ -1052,14 +1041,7 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
 // + r holds row r of CTA `rank`'s half of the tile (S slots per tile).  Items that are
 // waited on never wait themselves before they publish, and every CTA is resident (grid <=
 // SMs, one CTA per SM), so every wait ends.
-//
-// MC (a cluster of 4 = two CTA pairs on the two 256-row halves of a 512-row block, same
-// weight tile): each CTA loads its own A rows and half of its pair-half of the weight
-// tile, multicast to itself and to the CTA with the same role in the other pair, so the
-// weights cross from L2 once per cluster.  Every load completes on its destination pair's
-// leader barrier (64 KB per stage, as without multicast); a stage is refilled once both
-// pairs' MMAs have released it (empty counts the two leaders' commits).
-template <int EPI, bool MC, bool DS>
+template <int EPI, bool DS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
                     const __grid_constant__ CUtensorMap tmbh, const __grid_constant__ CUtensorMap tmc,
@@ -1086,22 +1068,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile uint32_t* holder_ptr = reinterpret_cast<volatile uint32_t*>(smem + (holder - base));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + (holder + 4 - base));
 
-  static_assert(!MC || KA2 == 1, "the multicast variant stages one K block per ring stage");
-  static_assert(!(MC && DS), "one four-CTA scheme at a time");
-  constexpr int CL = (MC || DS) ? 4 : 2;  // CTAs per cluster
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t crank = cluster_ctarank();
   const uint32_t rank = crank & 1u;             // 0: leader of the pair (issues the MMAs), 1: peer
-  const uint32_t pr = (MC || DS) ? (crank >> 1) : 0u;  // which pair of the cluster
   const uint32_t lead = crank & ~1u;            // cluster rank of this pair's leader
   const uint16_t pair_mask = (uint16_t)(0x3u << lead);
-  // the scheduler's unit: the cluster (pairs and MC), or the pair (DS: 2 per cluster)
-  const int cluster = DS ? (int)(blockIdx.x >> 1) : (int)(blockIdx.x / CL);
+  // the scheduler's unit: the pair (one cluster, or half of a DS cluster)
+  const int cluster = (int)(blockIdx.x >> 1);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
       mbar_init(full0 + 8 * s, 1);             // the pair leader's producer arrives (+ tx bytes)
-      mbar_init(empty0 + 8 * s, MC ? 2 : 1);   // MMA commits of the pairs that read the stage
+      mbar_init(empty0 + 8 * s, 1);            // the pair's MMA commit
     }
     mbar_init(tfull0, 1);
     mbar_init(tfull0 + 8, 1);
@@ -1120,7 +1098,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (warp == 1) tmem_alloc_pair(holder, TMEM2_COLS);
   tc_fence_before();
   __syncthreads();
-  cluster_sync_all();  // the peer's barriers exist before any remote arrive / multicast
+  cluster_sync_all();  // the peer's barriers exist before any remote arrive
   tc_fence_after();
   const uint32_t tmem_base = *holder_ptr;
   pdl_wait();  // the previous kernel of the step has completed
@@ -1128,19 +1106,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (ep.m_dev) M = min(M, *ep.m_dev);  // the step's row count (written by an earlier kernel)
   const int num_m = (M + 255) / 256;
   const int num_n = (N + 255) / 256;
-  const int num_mh = MC ? (num_m + 1) >> 1 : num_m;  // MC: units of two 256-row blocks
   Sched sc;
-  sc.tiles = num_mh * num_n;
+  sc.tiles = num_m * num_n;
   sc.ku = (K + BK * KA2 - 1) / (BK * KA2);
-  sc.C = DS ? gridDim.x / 2 : gridDim.x / CL;
+  sc.C = gridDim.x / 2;
   sc.splits = splits;
   sc.streamk = streamk;
   sc.halves = halves;
   sc.ds = DS ? 1 : 0;
-  // item tile -> (m block, n block); MC: pair pr takes the pr-th 256-row half of the unit
+  // item tile -> (m block, n block), M-fastest
   auto tile_mn = [&](int t, int& m_blk, int& n_blk) {
-    m_blk = MC ? 2 * (t % num_mh) + (int)pr : t % num_mh;
-    n_blk = t / num_mh;
+    m_blk = t % num_m;
+    n_blk = t / num_m;
   };
 
   if (warp == 0) {
@@ -1168,22 +1145,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ok = false;
             break;
           }
-          if constexpr (MC) {
-            // own A rows; half of the weight half, multicast to this CTA and its counterpart
-            const uint32_t full_leader = mapa_shared(full0 + 8 * stage, lead);
-            if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, 2 * STAGE2_BYTES);
-            tma_load_2d_pair(sA + stage * A2_STAGE_BYTES, &tma, kb * BK, m_blk * 256 + (int)rank * 128, full_leader);
-            tma_load_2d_pair_mc(sB + stage * B2_STAGE_BYTES + pr * (B2_BLOCK_BYTES / 2), &tmb, kb * BK,
-                                wrow + (int)pr * 64, full_leader, (uint16_t)((1u << crank) | (1u << (crank ^ 2u))));
-          } else {
-            const uint32_t full_leader = mapa_shared(full0 + 8 * stage, lead);
-            if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, stage_tx);
-            for (int a = 0; a < KA2; ++a) {
-              tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, &tma, (kb + a) * BK,
-                               m_blk * 256 + (int)rank * 128, full_leader);
-              tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, tw_map, (kb + a) * BK, wrow,
-                               full_leader);
-            }
+          const uint32_t full_leader = mapa_shared(full0 + 8 * stage, lead);
+          if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, stage_tx);
+          for (int a = 0; a < KA2; ++a) {
+            tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, &tma, (kb + a) * BK,
+                             m_blk * 256 + (int)rank * 128, full_leader);
+            tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, tw_map, (kb + a) * BK, wrow,
+                             full_leader);
           }
           if (++stage == STAGES2) {
             stage = 0;
@@ -1231,7 +1199,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int k = 0; k < BK / 16; ++k)
               umma_bf16_pair(d_tmem, da + 2 * k, db + 2 * k, idesc, (kb > kb0 || a > 0 || k > 0) ? 1u : 0u);
           }
-          umma_commit_pair(empty0 + 8 * stage, MC ? (uint16_t)0xF : pair_mask);
+          umma_commit_pair(empty0 + 8 * stage, pair_mask);
           if (++stage == STAGES2) {
             stage = 0;
             phase ^= 1u;
@@ -1270,16 +1238,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int m_blk, n_blk;
       tile_mn(it.t, m_blk, n_blk);
       const int t = m_blk + num_m * n_blk;  // the tile's id for counters and partials
-      const bool phantom = m_blk >= num_m;  // MC: the second half of a unit past the rows
       const int row = m_blk * 256 + (int)rank * 128 + row_local;
       o.row0 = m_blk * 256 + (int)rank * 128 + q * 32;
       o.live = o.row0 < M;
       Src s;
       s.taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * 256);
       s.row = row_local;
-      if (phantom) {
-        // nothing to store
-      } else if (it.kind == IT_PLAIN) {
+      if (it.kind == IT_PLAIN) {
         epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep, it.piece, it.width);
       } else if (it.kind == IT_DS_RECV) {
         // this pair's MMAs are done (tfull): the operand ring is free for the other K
@@ -1480,10 +1445,10 @@ cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
   return launch_pdl(kern, p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream, p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
 }
 
-template <int EPI, bool MC, bool DS = false>
+template <int EPI, bool DS = false>
 cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   static bool attr_set = false;
-  auto kern = gemm_tc2_kernel<EPI, MC, DS>;
+  auto kern = gemm_tc2_kernel<EPI, DS>;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2);
     if (e != cudaSuccess) return e;
@@ -1496,7 +1461,7 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = (MC || DS) ? 4 : 2;
+  attr[0].val.clusterDim.x = DS ? 4 : 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -1508,10 +1473,10 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
 }
 
 // Clusters of four CTA-pair CTAs that can be resident at once (0 if unknown).
-int mc_max_clusters() {
+int cluster4_max() {
   static int n = -1;
   if (n < 0) {
-    auto kern = gemm_tc2_kernel<EPI_BF16, true, false>;
+    auto kern = gemm_tc2_kernel<EPI_BF16, true>;
     n = 0;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2) == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
@@ -1649,19 +1614,6 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   plan->epi = epi;
   plan->ep = ep;
   if (epi == EPI_LMHEAD) plan->ep.vocab = N;
-  // MC (on request, kTileMulticast): two CTA pairs share every weight tile through
-  // multicast; needs two 256-row blocks, and the four-CTA clusters must all be resident
-  // (grid <= what fits).  Measured inside the LLaDA-8B step it is on par with plain pairs
-  // (the mainloop runs near the tensor peak either way), so the planner does not pick it.
-  int mc = 0, mc_clusters = 0;
-  if (pair_forced && (tile & kTileMulticast)) {
-    mc_clusters = mc_max_clusters();
-    if (cg != 2 || streamk != 0 || KA2 != 1 || M <= 256 || mc_clusters < 1) {
-      *why = "gemm: the multicast pair tile needs M > 256, no stream-K and resident 4-CTA clusters";
-      return cudaErrorInvalidValue;
-    }
-    mc = 1;
-  }
   // Half-width tail (on request, kTileHalves): whole tiles in full rounds, then each
   // tile of a partial last round as two 256 x 128 pieces on two pairs, with no partial
   // sums to combine (each output is still one MMA chain over all of K, so results are
@@ -1671,16 +1623,16 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   // planner does not pick it.
   int halves = 0;
   if (cg == 2 && pair_forced && (tile & kTileHalves)) {
-    if (streamk != 0 || mc != 0 || epi == EPI_LMHEAD || forced_splits > 1) {
-      *why = "gemm: half-width tail tiles exclude stream-K, multicast, K splits and the LM-head epilogue";
+    if (streamk != 0 || epi == EPI_LMHEAD || forced_splits > 1) {
+      *why = "gemm: half-width tail tiles exclude stream-K, K splits and the LM-head epilogue";
       return cudaErrorInvalidValue;
     }
     halves = 1;
     splits = 1;
   }
-  // each CTA loads 128 rows of A; of W a one-CTA tile loads bn rows, a pair CTA 128 (MC: 64)
+  // each CTA loads 128 rows of A; of W a one-CTA tile loads bn rows, a pair CTA 128
   if (!encode_kmajor(&plan->ta, A, M, K, BM) ||
-      !encode_kmajor(&plan->tb, W, N, K, cg == 2 ? (mc ? 64 : 128) : bn) ||
+      !encode_kmajor(&plan->tb, W, N, K, cg == 2 ? 128 : bn) ||
       (cg == 2 && !encode_kmajor(&plan->tbh, W, N, K, 64))) {
     *why = "gemm: cuTensorMapEncodeTiled failed";
     return cudaErrorInvalidValue;
@@ -1721,9 +1673,9 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   int ds = 0, ds_clusters = 0;
   if (cg == 2) {
     const bool ds_forced = pair_forced && (tile & kTileDsmem);
-    const bool ds_ok = streamk == 0 && mc == 0 && halves == 0 && epi != EPI_LMHEAD && units >= 2 &&
+    const bool ds_ok = streamk == 0 && halves == 0 && epi != EPI_LMHEAD && units >= 2 &&
                        (ds_forced ? forced_splits <= 1 : true);
-    const int cl4 = ds_ok ? std::min(num_sms / 4, mc_max_clusters()) : 0;
+    const int cl4 = ds_ok ? std::min(num_sms / 4, cluster4_max()) : 0;
     long full = 0, rest = 0;
     if (cl4 >= 1) {
       full = pair_tiles / (2L * cl4);
@@ -1753,7 +1705,6 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   }
   plan->ds = ds;
   if (ds) plan->splits = 1;
-  plan->mc = mc;
   if (cg == 2) {
     plan->n_tiles = (int)pair_tiles;
     // stream-K: all pairs when there are plain rounds, else only the sharing ones (the
@@ -1762,11 +1713,6 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
                        : halves ? (pair_tiles >= pairs ? pairs : std::min<long>(pairs, 2 * pair_tiles))
                                 : pair_tiles * splits;
     plan->grid = 2 * (int)(items < pairs ? items : pairs);
-    if (mc) {  // units of two 256-row blocks, one per cluster of four
-      const long units = (long)((((M + 255) / 256) + 1) / 2) * ((N + 255) / 256) * splits;
-      const long cl = std::min<long>(num_sms / 4, mc_clusters);
-      plan->grid = 4 * (int)(units < cl ? units : cl);
-    }
     if (ds) plan->grid = 4 * ds_clusters;
     plan->smem = SMEM2;
     if (splits > 1) {
@@ -1863,22 +1809,12 @@ cudaError_t wait_selftest_launch(int which, const int* flag, int* err, cudaStrea
 
 cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
   if ((p.flags_needed && !p.flags) || (p.ws_needed && !p.ws)) return cudaErrorInvalidValue;
-  if (p.cg == 2 && p.mc) {
+  if (p.cg == 2 && p.ds) {
     switch (p.epi) {
       case EPI_BF16: return launch_t2<EPI_BF16, true>(p, err, stream);
       case EPI_RESID_F32: return launch_t2<EPI_RESID_F32, true>(p, err, stream);
       case EPI_QKV_ROPE: return launch_t2<EPI_QKV_ROPE, true>(p, err, stream);
       case EPI_SWIGLU: return launch_t2<EPI_SWIGLU, true>(p, err, stream);
-      case EPI_LMHEAD: return launch_t2<EPI_LMHEAD, true>(p, err, stream);
-    }
-    return cudaErrorInvalidValue;
-  }
-  if (p.cg == 2 && p.ds) {
-    switch (p.epi) {
-      case EPI_BF16: return launch_t2<EPI_BF16, false, true>(p, err, stream);
-      case EPI_RESID_F32: return launch_t2<EPI_RESID_F32, false, true>(p, err, stream);
-      case EPI_QKV_ROPE: return launch_t2<EPI_QKV_ROPE, false, true>(p, err, stream);
-      case EPI_SWIGLU: return launch_t2<EPI_SWIGLU, false, true>(p, err, stream);
     }
     return cudaErrorInvalidValue;
   }

@@ -62,23 +62,19 @@ def test_rmsnorm(ops, rows, d):
 
 
 # ------------------------------------------------------------------ tcgen05 GEMM
-PAIR, SK, MC, HALF, DS = 2, 1 << 16, 1 << 17, 1 << 18, 1 << 19
+PAIR, SK, HALF, DS = 2, 1 << 16, 1 << 18, 1 << 19
 # auto, one-CTA 128 / 256 columns, CTA pair (library's K schedule), CTA pair unsplit,
 # CTA pair with 2 / 3 K splits, CTA pair with stream-K over all pairs / in K halves,
-# clusters of two pairs sharing weight tiles (unsplit / 2 K splits), left-over tiles as
-# two half-width pieces
+# left-over tiles as two half-width pieces, left-over tiles split by K over a cluster's
+# two pairs (DSMEM sum)
 TILES = [0, 128, 256, PAIR, PAIR | (1 << 8), PAIR | (2 << 8), PAIR | (3 << 8), PAIR | SK, PAIR | SK | (2 << 8),
-         PAIR | MC | (1 << 8), PAIR | MC | (2 << 8), PAIR | HALF, PAIR | DS]
+         PAIR | HALF, PAIR | DS]
 
 
 def _splits(tile):
     if (tile & 0xff) != PAIR or tile & SK:
         return 1
     return max(1, (tile >> 8) & 0xff)
-
-
-def _rows_ok(M, tile):
-    return not (tile & MC) or M > 256
 
 
 def _streamk_possible(M, N, K, segments):
@@ -96,7 +92,7 @@ def _unsupported(M, N, K, tile):
         return K // 64 < 2
     if tile & SK:
         return not _streamk_possible(M, N, K, (tile >> 8) & 0xff)
-    return K // 64 < _splits(tile) or not _rows_ok(M, tile)
+    return K // 64 < _splits(tile)
 
 
 @pytest.mark.parametrize("tile", TILES)
@@ -141,7 +137,6 @@ def test_linear_residual(ops, M, N, K, tile):
 
 @pytest.mark.parametrize("tile,mode", [(PAIR | (3 << 8), 1), (PAIR | (2 << 8), 0), (0, 1), (0, 0),
                                        (PAIR | SK, 0), (PAIR | SK, 1), (PAIR | SK | (2 << 8), 1),
-                                       (PAIR | MC | (2 << 8), 1), (PAIR | MC | (3 << 8), 0),
                                        (PAIR | DS, 1), (PAIR | DS, 0)])
 def test_linear_split_k_is_deterministic(ops, tile, mode):
     """Split-K and stream-K partial sums are combined in K order: two runs give the same
@@ -204,7 +199,7 @@ def test_attention_non_causal(ops, B, T, H, G, hd):
 
 
 # ------------------------------------------------------------------ LM head + confidence
-@pytest.mark.parametrize("tile", [0, 256, PAIR, PAIR | SK, PAIR | SK | (2 << 8), PAIR | MC | (1 << 8)])
+@pytest.mark.parametrize("tile", [0, 256, PAIR, PAIR | SK, PAIR | SK | (2 << 8)])
 @pytest.mark.parametrize("R,V,d,sz", [(37, 4096, 256, 12.0), (5, 1000, 128, 6.0), (130, 4096, 64, 20.0),
                                       (300, 4096, 256, 12.0), (64, 126464, 4096, 15.0),
                                       (300, 126464, 4096, 15.0)])
