@@ -213,9 +213,13 @@ dcl_status dcl_accept(dcl_ctx* ctx, const void* logits_dev, int32_t B, int32_t P
  * without any allocation: its scratch (12 bytes per position) is a file-scope device
  * array of DCL_NOALLOC_MAX_POSITIONS positions (384 KB) that every GPU loading this
  * library holds until the process exits.
- *   - B*P above DCL_NOALLOC_MAX_POSITIONS is rejected with DCL_ERR_INVALID_ARG.
+ *   - The size limits are dcl_accept's (1 <= P <= 4096, V >= 2), and B*P at most
+ *     DCL_NOALLOC_MAX_POSITIONS; anything else is rejected with DCL_ERR_INVALID_ARG.
  *   - The first call on a device looks up the array's device address (once per device,
- *     with that device current); make that first call before any stream capture.
+ *     with that device current) and keeps it for the life of the process; make that
+ *     first call before any stream capture.  A cudaDeviceReset unloads the library's
+ *     device code, array included, and leaves the kept address stale: do not call this
+ *     function after one.
  *   - All calls share the one array and it keeps the last call's contents; a call
  *     writes every scratch entry it reads, so nothing needs clearing, but calls whose
  *     work overlaps on the GPU (e.g. on two streams) race on it.

@@ -8,7 +8,9 @@ For each row b of a block of P positions with c_b positions already committed
     probability, or exp(-entropy) with ``confidence = 1``; top-2 probability for reporting),
   * K over the window [p, p + L') with L' = min(L, P - p)          (Eq. compute_k),
   * commit x[p:p+K] and refresh drafts at i >= p + L                (Eq. draft_update),
-using the same readings as ``oracle.decode``.
+using the same readings as ``oracle.decode``; with ``acceptance = 1`` instead every
+uncommitted position of [p, P) with c > tau_commit is committed (Eq. threshold_pd, at least
+``min_commit`` of them by confidence), no drafts, and K is the number committed.
 """
 from __future__ import annotations
 
@@ -39,5 +41,9 @@ def accept(logits: np.ndarray, committed: np.ndarray, x: np.ndarray,
         i_, c1, c2 = model.confidence(z)
         H = model.entropy(z) if cfg.confidence == 1 else None
         ids[b, p:], p1[b, p:], p2[b, p:] = i_, decode.decision_confidence(c1, H, cfg), c2
-        K[b] = decode.commit_and_draft(x_out[b], p, ids[b], p1[b], cfg, window)
+        if cfg.acceptance == 0:
+            K[b] = decode.commit_and_draft(x_out[b], p, ids[b], p1[b], cfg, window)
+        else:  # Eq. threshold_pd over the uncommitted rest of the block, no drafts
+            committed_b = np.arange(P) < p
+            K[b] = len(decode.threshold_commit(x_out[b], committed_b, ids[b], p1[b], p, P, cfg))
     return K, x_out, ids, p1, p2

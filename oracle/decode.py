@@ -31,6 +31,19 @@ Readings where the paper is silent or inconsistent (each one is also a test):
   * every step records Eq. entropy_bound on the set it committed in parallel,
     sum_{i in U} H_i - max_{j in U} H_j with U = [p, p + K) and the step's own marginal
     entropies (0 when K = 1);
+  * ``acceptance = 1`` replaces DCV by the non-contiguous rule DC-Leap is contrasted with
+    (Eq. threshold_pd, Sec. 2.1 and Sec. 3.1): every masked position whose confidence
+    exceeds tau_commit is committed at once, independently of its neighbours.  As the
+    paper runs every method semi-autoregressively with block length 32 (Sec. 4.1), the
+    rule applies to the masked positions of the current block [b0, b0 + Bk),
+    b0 = N + Bk * floor((p - N) / Bk), with p the leftmost uncommitted position; there
+    are no drafts and nothing to re-mask.  Eq. threshold_pd allows an empty set (the
+    same stall as K = 0); when fewer than ``min_commit`` positions pass, the
+    ``min_commit`` most confident masked positions of the block are committed instead
+    (ties to the lower position).  With tau_commit >= 1 nothing passes, which is the
+    low-confidence remasking of the base LLaDA sampler: ``min_commit`` tokens per step,
+    the most confident first.  A committed position stays committed (an explicit flag:
+    the committed token may itself be the MASK id, R8);
   * the approximate cache (``kv_cache = 1``; the paper pairs DC-Leap with a dLLM cache in
     Sec. 4 / Tab. 6 without describing its policy): per row, a step computes all
     positions at the first step and whenever the block-aligned prefix end
@@ -56,6 +69,7 @@ class DecodeConfig:
     contiguous_drafts: bool = False  # App. E variant: drafts only as an unbroken chain
     kv_cache: int = 0
     confidence: int = 0           # 0: top-1 probability (Eq. threshold_pd); 1: exp(-entropy)
+    acceptance: int = 0           # 0: DCV (Eq. compute_k); 1: Eq. threshold_pd in the block
 
     def window(self) -> int:
         return self.max_window if self.max_window > 0 else max(1, self.gen_len // 2)
@@ -93,6 +107,27 @@ def commit_and_draft(x: np.ndarray, p: int, ids: np.ndarray, c: np.ndarray,
         seg = x[lo:T]
         seg[ok] = ids[lo:T][ok]
     return K
+
+
+def threshold_commit(x: np.ndarray, committed: np.ndarray, ids: np.ndarray, c: np.ndarray,
+                     lo: int, hi: int, cfg: DecodeConfig) -> list:
+    """Eq. threshold_pd on the uncommitted positions of [lo, hi) of one row (ids / c / x /
+    committed indexed by absolute position): M_i = 1(c_i > tau_commit) for each one
+    independently, and every position with M_i = 1 is committed in the same step.  When
+    fewer than ``min_commit`` pass, the ``min_commit`` uncommitted positions of highest
+    confidence are committed instead (float32 confidences, ties to the lower position);
+    they include every passing one.  Returns the committed positions, in increasing order."""
+    cand = [i for i in range(lo, hi) if not committed[i]]
+    passing = [i for i in cand if exceeds(c[i], cfg.tau_commit)]
+    if len(passing) >= cfg.min_commit:
+        chosen = passing
+    else:
+        ranked = sorted(cand, key=lambda i: (-float(np.float32(c[i])), i))
+        chosen = sorted(ranked[:cfg.min_commit])
+    for i in chosen:
+        x[i] = ids[i]
+        committed[i] = True
+    return chosen
 
 
 def entropy_confidence(H) -> np.ndarray:
@@ -145,8 +180,14 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
     M = cfg.gen_len
     T = N + M
     L = cfg.window()
+    if cfg.acceptance not in (0, 1):
+        raise ValueError("acceptance must be 0 (DCV) or 1 (Eq. threshold_pd)")
+    if cfg.acceptance == 1 and cfg.block_len < 1:
+        raise ValueError("Eq. threshold_pd decoding needs a block length >= 1")
     x = np.full((B, T), mask_id, dtype=np.int32)
     x[:, :N] = prompt
+    committed = np.zeros((B, T), dtype=bool)  # (Eq. threshold_pd only: commits out of order)
+    committed[:, :N] = True
     p = np.full(B, N, dtype=np.int64)
     steps = np.zeros(B, dtype=np.int64)
     ks, starts, inputs, preds, bounds = [], [], [], [], []
@@ -163,7 +204,8 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             if p[b] >= T:
                 in_step[b] = x[b]
                 continue
-            remask(x[b], int(p[b]), L, mask_id)                  # (i)
+            if cfg.acceptance == 0:
+                remask(x[b], int(p[b]), L, mask_id)              # (i)
             in_step[b] = x[b]
             if cfg.kv_cache:                                     # (ii), approximate cache
                 pe = prefix_end(int(p[b]), N, cfg.block_len)
@@ -180,9 +222,18 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             full_ids[N:] = ids
             full_c[N:] = decision_confidence(p1, H, cfg)
             p0 = int(p[b])
-            k_step[b] = commit_and_draft(x[b], p0, full_ids, full_c, cfg, L)  # (iii)-(iv)
-            jp[b] = np.nan if H is None else jpde_bound(np.asarray(H)[p0 - N:p0 - N + k_step[b]])
-            p[b] += k_step[b]                                    # dynamically advance
+            if cfg.acceptance == 0:
+                k_step[b] = commit_and_draft(x[b], p0, full_ids, full_c, cfg, L)  # (iii)-(iv)
+                jp[b] = np.nan if H is None else jpde_bound(np.asarray(H)[p0 - N:p0 - N + k_step[b]])
+                p[b] += k_step[b]                                # dynamically advance
+            else:                                                # Eq. threshold_pd in the block
+                lo = prefix_end(p0, N, cfg.block_len)
+                chosen = threshold_commit(x[b], committed[b], full_ids, full_c, lo,
+                                          min(lo + cfg.block_len, T), cfg)
+                k_step[b] = len(chosen)
+                jp[b] = np.nan if H is None else jpde_bound(np.asarray(H)[np.asarray(chosen, int) - N])
+                while p[b] < T and committed[b, p[b]]:           # leftmost uncommitted
+                    p[b] += 1
             steps[b] += 1
             pr[0, b], pr[1, b], pr[2, b] = ids, p1, p2
             if H is not None:

@@ -23,7 +23,10 @@ static __device__ __align__(256) unsigned char g_accept_scratch[3 * 4 * kMaxPosi
 std::mutex g_mu;
 void* g_scratch_addr[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device (looked up once per device).
+// Device address of the scratch array on the current device (looked up once per device
+// and kept for the life of the process: a cudaDeviceReset, which unloads this library's
+// device code and frees the array, leaves the kept address stale, so the call is not to be
+// used after one).
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -50,9 +53,9 @@ extern "C" dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int3
     dcl::set_thread_error("dcl_accept_noalloc: NULL argument");
     return DCL_ERR_INVALID_ARG;
   }
-  if (B <= 0 || P <= 0 || V <= 1 || (int64_t)B * P > kMaxPositions) {
-    dcl::set_thread_error(("dcl_accept_noalloc: B*P must be in [1, " + std::to_string(kMaxPositions) +
-                          "] (the size of its static scratch) and V > 1")
+  if (B <= 0 || P <= 0 || V <= 1 || P > 4096 || (int64_t)B * P > kMaxPositions) {
+    dcl::set_thread_error(("dcl_accept_noalloc: need P <= 4096 (as dcl_accept), B*P in [1, " +
+                          std::to_string(kMaxPositions) + "] (the size of its static scratch) and V > 1")
                              .c_str());
     return DCL_ERR_INVALID_ARG;
   }

@@ -20,6 +20,7 @@ import test_oracle_cache as tcache
 import test_oracle_decode as tdec
 import test_oracle_entropy as tent
 import test_oracle_model as tmod
+import test_oracle_threshold as tthr
 
 ROOT_GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
 
@@ -194,8 +195,46 @@ def _commit_drafts_ignore_chain(x, p, ids, c, cfg, window):  # App. E flag ignor
     return _ORIG["commit_and_draft"](x, p, ids, c, replace(cfg, contiguous_drafts=False), window)
 
 
+def _threshold_forced_leftmost(x, committed, ids, c, lo, hi, cfg):
+    """Forced progress commits the leftmost masked positions, not the most confident."""
+    cand = [i for i in range(lo, hi) if not committed[i]]
+    passing = [i for i in cand if decode.exceeds(c[i], cfg.tau_commit)]
+    chosen = passing if len(passing) >= cfg.min_commit else cand[:cfg.min_commit]
+    for i in chosen:
+        x[i] = ids[i]
+        committed[i] = True
+    return chosen
+
+
+def _threshold_ties_high(x, committed, ids, c, lo, hi, cfg):
+    """Equal confidences ranked to the higher position."""
+    cand = [i for i in range(lo, hi) if not committed[i]]
+    passing = [i for i in cand if decode.exceeds(c[i], cfg.tau_commit)]
+    if len(passing) >= cfg.min_commit:
+        chosen = passing
+    else:
+        chosen = sorted(sorted(cand, key=lambda i: (-float(np.float32(c[i])), -i))[:cfg.min_commit])
+    for i in chosen:
+        x[i] = ids[i]
+        committed[i] = True
+    return chosen
+
+
+def _threshold_whole_sequence(x, committed, ids, c, lo, hi, cfg):
+    """The rule applied to every masked position to the sequence end, not the block."""
+    return _ORIG["threshold_commit"](x, committed, ids, c, lo, x.shape[0], cfg)
+
+
+def _threshold_recommits(x, committed, ids, c, lo, hi, cfg):
+    """Committed positions taken as candidates again (their flags ignored when choosing)."""
+    chosen = _ORIG["threshold_commit"](x, np.zeros_like(committed), ids, c, lo, hi, cfg)
+    committed[chosen] = True
+    return chosen
+
+
 _ORIG = {"block": model.block, "confidence": model.confidence, "entropy": model.entropy,
-         "accept": accept.accept, "commit_and_draft": decode.commit_and_draft}
+         "accept": accept.accept, "commit_and_draft": decode.commit_and_draft,
+         "threshold_commit": decode.threshold_commit}
 _TINY_W = syn.model_weights(syn.SHAPES["tiny"], 0, lm_head_scale=40.0, norm_gain_std=0.1)
 
 
@@ -253,6 +292,14 @@ CASES = [
     ("contiguous drafts ignored", decode, "commit_and_draft", _commit_drafts_ignore_chain,
      [lambda: tdec.test_golden_scripted_trajectories(ROOT_GOLDEN),
       lambda: tdec.test_golden_after_states_step_by_step(ROOT_GOLDEN)]),
+    ("threshold rule: forced commit leftmost", decode, "threshold_commit", _threshold_forced_leftmost,
+     [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
+    ("threshold rule: ties to the higher position", decode, "threshold_commit", _threshold_ties_high,
+     [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
+    ("threshold rule: block ignored", decode, "threshold_commit", _threshold_whole_sequence,
+     [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
+    ("threshold rule: committed flags ignored", decode, "threshold_commit", _threshold_recommits,
+     [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
     ("prefix end not block-aligned", decode, "prefix_end", _prefix_end_unaligned,
      [tdec.test_prefix_end_is_the_start_of_the_current_block,
       lambda: tcache.test_refresh_exactly_at_block_changes(_TINY_W)]),
