@@ -252,10 +252,81 @@ def oracle_generation(wl, min_seconds=2.0):
     return (time.perf_counter() - t0) / n, int(out["n_iter"]), n
 
 
+def _step_margin(pr, x_in, p, K, N, L, tau_c, tau_d):
+    """Smallest margin among the decisions of one oracle step of one row: |c - tau_c| over
+    the window up to and including its first failure, |c - tau_d| over the draft region,
+    and the top-1 / top-2 gap of every committed or drafted id."""
+    ids, p1, p2 = pr[0], pr[1], pr[2]
+    T = x_in.shape[0]
+    c = np.zeros(T)
+    gap = np.full(T, np.inf)
+    c[N:], gap[N:] = p1, p1 - p2
+    w = min(L, T - p)
+    m = [np.abs(c[p:p + min(K + 1, w)] - tau_c).min(), gap[p:p + K].min()]
+    if p + L < T:
+        m.append(np.abs(c[p + L:] - tau_d).min())
+        drafted = c[p + L:] > tau_d
+        if drafted.any():
+            m.append(gap[p + L:][drafted].min())
+    return float(min(m))
+
+
+def near_tie_study(ctx, dcl, shape, weights, N, M, L, tau_c, tau_d, seeds, tol=1e-3, drift=5e-2):
+    """Whole generations of `seeds` random prompts on the GPU (step by step) and in the oracle
+    (bf16 operands): per seed, whether the committed sequences are identical, else the
+    oracle's smallest decision margin at the step where the two trajectories split:
+    within `tol` (a near tie), within `drift` (inside the end-to-end confidence drift of the
+    random model), or clear.  Returns the counts and the fraction of diverged seeds."""
+    import synthetic as syn
+    from oracle import decode, model
+    T = N + M
+    cfg = dcl.decode_config(tau_commit=tau_c, tau_draft=tau_d, max_window=L, gen_len=M)
+    ocfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=tau_d, max_window=L, gen_len=M)
+    predict = lambda t: model.predict(shape, weights, t, rows=slice(N, T), bf16_operands=True)  # noqa: E731
+    out = {"seeds": len(seeds), "identical": 0, "split_near_tie": 0, "split_within_drift": 0, "split_clear": 0,
+           "near_tie_margin": tol, "drift_margin": drift, "split_margins": []}
+    for seed in seeds:
+        prompt = syn.prompt_ids(3000 + seed, 1, N, shape.mask_id)
+        ctx.set_prompt(prompt, cfg)
+        states = []
+        for _ in range(2 * M):
+            x, p = ctx.get_state()
+            states.append((x[0].copy(), int(p[0])))
+            if p[0] >= T:
+                break
+            ctx.step()
+        ref = decode.generate(predict, prompt, ocfg, shape.mask_id)
+        p_o, split = N, None
+        for s, xin in enumerate(ref["inputs"]):
+            xg, pg = states[s] if s < len(states) else (None, -1)
+            keep = (np.arange(T) < p_o) | (np.arange(T) >= p_o + L)  # not re-masked at this step
+            if pg != p_o or not (xg == xin[0])[keep].all():
+                split = s
+                break
+            p_o += int(ref["k"][s, 0])
+        if split is None and (states[-1][0][N:] == ref["x"][0, N:]).all():
+            out["identical"] += 1
+            continue
+        s = (split if split is not None else len(ref["inputs"])) - 1
+        p_prev = p_o - int(ref["k"][s, 0]) if split is not None else p_o - int(ref["k"][s, 0])
+        mg = _step_margin(ref["preds"][s][:, 0], ref["inputs"][s][0], p_prev, int(ref["k"][s, 0]), N, L, tau_c,
+                          tau_d)
+        out["split_margins"].append(mg)
+        out["split_near_tie" if mg <= tol else "split_within_drift" if mg <= drift else "split_clear"] += 1
+    out["fraction_diverged"] = 1.0 - out["identical"] / max(1, len(seeds))
+    return out
+
+
 class OracleSample:
     """A bounded sample of one step of the oracle: one transformer block over all T rows,
     and the LM head + confidence over 16 generation rows x 1/16 of the vocabulary; scaled
-    to a step as n_layers x block + (B*M/16) x 16 x LM-head sample."""
+    to a step as n_layers x block + (B*M/16) x 16 x LM-head sample (an estimate of the
+    step's time, not a timed step).  Both oracle legs credit a step one committed token per
+    row, the least a step commits (the oracle cannot afford the 8B-shape trajectory that
+    would give its real rate)."""
+
+    RULE = ("ms_per_step is an estimate (the sample scaled to a step); tokens/s credits one committed token "
+            "per row per step, the least a step commits")
 
     def __init__(self, wl):
         import synthetic as syn
@@ -318,15 +389,15 @@ def run_reference(args):
         secs.append(s)
         cpu += c
     ms = 1e3 * statistics.mean(secs)
-    tps = wl["batch"] * 1.0 / (ms / 1e3)  # one committed token per row per step (see below)
+    tps = wl["batch"] * 1.0 / (ms / 1e3)  # one committed token per row per step (OracleSample.RULE)
     line = {
         "impl": "reference", "metric": METRIC, "value": tps, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": _config(wl, args),
+        "ms_per_step_is_estimate": True,
         "cpu_baseline": {"value": tps, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": samp.describe() + "; tokens/s assumes one committed token per row "
-                         "per step (the oracle cannot afford a full 8B-shape trajectory)",
+                         "sample": samp.describe() + "; " + OracleSample.RULE,
                          "cpu_seconds_timed": cpu},
         "e2e": {"value": tps, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -489,7 +560,7 @@ def run_ours(args):
 
     # per-kernel device times: the same steps with timing events around every kernel
     ctx.set_profiling(True)
-    ms_prof, _ = timed(min(args.steps, max(3, S)))
+    ms_prof, _ = timed(min(args.steps, max(3, S)))  # (n_prof steps)
     kern_ms, kern_kind = ctx.profile_last_step()
     ctx.set_profiling(False)
 
@@ -532,12 +603,14 @@ def run_ours(args):
                                                       statistics.mean(e2e_s), dist, "cuda")
     peaks = _peaks()
     if cached:
-        # the cached step's work varies (refresh or suffix): the trajectory's mean
+        # the cached step's work varies (refresh or suffix): the mean over exactly the steps
+        # timed (the window replays the trajectory from its start, wrapping at its end)
         rl = cached_rows(kper, N, M, wl["block"])
         works = [step_work(shape, B, N, M, r, l, True) for r, l in rl]
+        timed_works = [works[i % S] for i in range(args.steps)]
         per_layer = works[0][0]
-        total_flops = {k: statistics.mean(w[1][k] for w in works) for k in works[0][1]}
-        step_bytes = statistics.mean(w[2] for w in works)
+        total_flops = {k: statistics.mean(w[1][k] for w in timed_works) for k in works[0][1]}
+        step_bytes = statistics.mean(w[2] for w in timed_works)
     else:
         per_layer, total_flops, step_bytes = step_work(shape, B, N, M)
 
@@ -551,19 +624,24 @@ def run_ours(args):
     tot = sum(e["ms"] for e in table.values())
     for e in table.values():
         e["share"] = e["ms"] / tot if tot else 0.0
-    gemms = {k: v for k, v in table.items() if k.startswith("gemm") and k in total_flops}
+    # (the table is the last profiled step: with the cache, that step's own work)
+    n_prof = min(args.steps, max(3, S))
+    kern_flops = works[(n_prof - 1) % S][1] if cached else total_flops
+    gemms = {k: v for k, v in table.items() if k.startswith("gemm") and k in kern_flops}
     dom = max(gemms, key=lambda k: gemms[k]["ms"])
     avg_ms = gemms[dom]["ms"] / gemms[dom]["launches"]
-    flops_launch = total_flops[dom] / gemms[dom]["launches"]
+    flops_launch = kern_flops[dom] / gemms[dom]["launches"]
     achieved = flops_launch / (avg_ms / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
     for k, e in table.items():
-        if k in total_flops:
-            e["tflops"] = total_flops[k] / (e["ms"] / 1e3) / 1e12
+        if k in kern_flops:
+            e["tflops"] = kern_flops[k] / (e["ms"] / 1e3) / 1e12
     step_flops = sum(total_flops.values())
     ms_step = ms_max / args.steps
     t_roof = max(step_flops / (peak * 1e12), step_bytes / (peaks["hbm_gbs"] * 1e9))
     traffic = _traffic_from_profiles(dom)
+    # the launch floor: a graph of as many empty dependent launches as a step has
+    floor_ms = ctx.launch_floor(len(kern_ms), reps=200)
 
     # CPU oracle on a bounded sample (rank 0, one GPU only)
     cpu = None
@@ -574,12 +652,18 @@ def run_ours(args):
                    "sample": f"whole generations end to end ({steps_o} denoise steps, {B * M} tokens each; "
                              f"{n} timed), fp64 numpy", "ms_per_step": 1e3 * s / steps_o,
                    "cpu_seconds_timed": s * n}
+            # the same oracle generations against the GPU's on 32 prompts: how often and at
+            # which decision margins the committed sequences part
+            w_host = syn.model_weights(shape, wl["seed"], 0.02, wl["lm_scale"], 0.0)
+            cpu["near_tie_divergence"] = near_tie_study(ctx, dcl, shape, w_host, N, M, wl["window"], wl["tau_c"],
+                                                        wl["tau_d"], range(32))
         else:
             samp = OracleSample(wl)
             s, c = samp.step_seconds()
-            cpu = {"value": per_step / s, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                   "sample": samp.describe() + "; scaled to one step, tokens per step taken from the "
-                             "GPU run of the same trajectory", "ms_per_step": 1e3 * s, "cpu_seconds_timed": c}
+            cpu = {"value": B * 1.0 / s, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                   "sample": samp.describe() + "; " + OracleSample.RULE, "ms_per_step": 1e3 * s,
+                   "ms_per_step_is_estimate": True, "cpu_seconds_timed": c,
+                   "tokens_per_s_at_gpu_trajectory_rate": per_step / s}
 
     line = {
         "metric": METRIC, "value": tokens_all / (ms_max / 1e3), "unit": "tokens/s", "n_gpus": world,
@@ -603,6 +687,10 @@ def run_ours(args):
         "ms_per_step_at_p": at_p or None,
         "ms_per_step_profiled": ms_prof / min(args.steps, max(3, S)),
         "gpu_launches": args.steps * len(kern_ms),
+        "launch_floor": {"ms_per_graph": floor_ms, "launches_per_step": len(kern_ms),
+                         "step_over_floor": ms_step / floor_ms,
+                         "what": "a CUDA graph of as many empty kernels (dependent launches, as the step's) "
+                                 "as one step launches"},
         "clocks": clocks,
         "e2e": {"value": world * B * M / e2e_mean, "unit": "tokens/s",
                 "h2d_bytes_per_step": 4 * B * T + 12 * B + 4,
@@ -829,13 +917,19 @@ def _traffic_from_profiles(kernel):
 
 
 # Threshold / window grids of the paper's sensitivity ablations (App. F.1: tau_c at
-# tau_d = 0.98, tau_d at tau_c = 0.70, the maximum window L), plus the tau_c grid with
-# the entropy confidence (App. F.3 alternatives).
+# tau_d = 0.98, tau_d at tau_c = 0.70, the maximum window L), the tau_c grid with the
+# entropy confidence (App. F.3 alternatives), and the samplers DC-Leap is contrasted with
+# on the same kernels: the non-contiguous threshold rule (Eq. threshold_pd) in the
+# semi-autoregressive block at the same thresholds, and the base sampler's low-confidence
+# remasking (one token per step, the most confident masked position of the block).
 SWEEPS = (
     [("tau_commit", dict(tau_c=t, tau_d=0.98, window=None, confidence=0)) for t in (0.65, 0.68, 0.70, 0.72, 0.75, 0.80)]
     + [("tau_draft", dict(tau_c=0.70, tau_d=t, window=None, confidence=0)) for t in (0.85, 0.88, 0.90, 0.92, 0.95, 0.98)]
     + [("window", dict(tau_c=0.70, tau_d=0.98, window=w, confidence=0)) for w in (32, 64, 96, 128)]
     + [("tau_commit_entropy", dict(tau_c=t, tau_d=0.98, window=None, confidence=1)) for t in (0.65, 0.70, 0.80)]
+    + [("threshold_pd", dict(tau_c=t, tau_d=0.98, window=None, confidence=0, acceptance=1))
+       for t in (0.65, 0.70, 0.80, 0.90, 0.95)]
+    + [("low_confidence_remasking", dict(tau_c=1.0, tau_d=0.98, window=None, confidence=0, acceptance=1))]
 )
 
 
@@ -862,7 +956,7 @@ def run_sweep(args):
         window = pt["window"] or wl["window"]
         cfg = dcl.decode_config(tau_commit=pt["tau_c"], tau_draft=pt["tau_d"], max_window=window,
                                 block_len=wl["block"], gen_len=M, kv_cache=int(wl.get("cache", 0)),
-                                confidence=pt["confidence"])
+                                confidence=pt["confidence"], acceptance=pt.get("acceptance", 0))
         ctx.set_prompt(prompt, cfg)
         ctx.generate(max_steps=4 * M, out=False)  # warm-up (graph capture for this config)
         secs, st = [], None
@@ -875,6 +969,7 @@ def run_sweep(args):
         sec = min(secs)
         print(json.dumps({"sweep": name, "workload": args.workload, "tau_commit": pt["tau_c"],
                           "tau_draft": pt["tau_d"], "window": window, "confidence": pt["confidence"],
+                          "acceptance": "threshold_pd" if pt.get("acceptance") else "dcv",
                           "steps": int(st.steps), "tokens": int(st.tokens),
                           "steps_per_token": st.steps / max(1, st.tokens / B),
                           "ms_per_step": 1e3 * sec / max(1, st.steps), "tokens_per_s": st.tokens / sec,

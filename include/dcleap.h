@@ -69,6 +69,18 @@ typedef struct {
                                 1: c = exp(-H), H = -sum_v P(v) ln P(v) the marginal entropy of
                                 Eq. entropy_bound (an alternative confidence, cf. App. F.3);
                                 exp(-H) <= p1, so it never accepts more than 0 */
+  int32_t acceptance;        /* 0: DCV, the contiguous rule (Eq. compute_k + Eq. draft_update);
+                                1: the non-contiguous rule DC-Leap is contrasted with
+                                (Eq. threshold_pd, Sec. 2.1): every masked position of the
+                                current semi-autoregressive block (block_len positions from
+                                N + block_len * floor((p - N) / block_len), p the leftmost
+                                uncommitted position) with c > tau_commit is committed at once;
+                                if fewer than min_commit pass, the min_commit most confident
+                                masked positions of the block are (ties to the lower position;
+                                tau_commit >= 1 gives the base sampler's low-confidence
+                                remasking, min_commit tokens per step); no drafts, no
+                                re-masking, tau_draft / max_window / contiguous_drafts unused,
+                                and K is the number committed */
 } dcl_decode_config;
 
 typedef struct {
@@ -138,8 +150,9 @@ dcl_status dcl_init_random_weights(dcl_ctx* ctx, uint64_t seed, float std, float
  * (Eq. 1).  prompt is host int32 [batch][n_prompt]; batch <= max_batch,
  * n_prompt + cfg->gen_len <= max_seq.  Validates ids, uploads the state and builds
  * (or reuses) the CUDA graph of one step for this shape.
- * Errors: INVALID_ARG (also kv_cache or confidence outside {0, 1}), UNSUPPORTED (kv_cache
- * = 1 with N, M or block_len not a multiple of 32), CUDA. */
+ * Errors: INVALID_ARG (also kv_cache, confidence or acceptance outside {0, 1}, or
+ * acceptance = 1 with block_len < 1), UNSUPPORTED (kv_cache = 1 with N, M or block_len not
+ * a multiple of 32), CUDA. */
 dcl_status dcl_set_prompt(dcl_ctx* ctx, int32_t batch, const int32_t* prompt, int32_t n_prompt,
                           const dcl_decode_config* cfg);
 
@@ -163,7 +176,8 @@ dcl_status dcl_restart(dcl_ctx* ctx);
 
 /* Read / write the decoding state (x: host int32 [batch][N+M], p: host int32 [batch]),
  * e.g. to resume a run or to drive teacher-forced parity.  get synchronises.
- * set validates ids and N <= p <= N+M.  Errors: STATE, INVALID_ARG, CUDA. */
+ * set validates ids and N <= p <= N+M; under acceptance = 1 a position counts as committed
+ * when it lies before p or holds a token other than MASK.  Errors: STATE, INVALID_ARG, CUDA. */
 dcl_status dcl_get_state(dcl_ctx* ctx, int32_t* x, int32_t* p);
 dcl_status dcl_set_state(dcl_ctx* ctx, const int32_t* x, const int32_t* p);
 
@@ -180,8 +194,22 @@ dcl_status dcl_forward_debug(dcl_ctx* ctx, void* logits_dev, int32_t* top1_dev, 
 
 /* Parity hook: the residual stream after the embedding (layer = -1) or after
  * transformer block `layer` of the last forward, copied to h_dev (float [batch*(N+M)][d]).
- * Call after dcl_forward_debug.  Errors: STATE, INVALID_ARG, CUDA. */
+ * Call after dcl_forward_debug or dcl_forward_debug_from.  Errors: STATE, INVALID_ARG, CUDA. */
 dcl_status dcl_debug_hidden(dcl_ctx* ctx, int32_t layer, float* h_dev);
+
+/* Parity hook for per-block teacher forcing (Eq. 2's forward, one block at a time): the
+ * forward of step (ii) started at transformer block `layer` (0 <= layer <= n_layers) from
+ * the caller's residual stream h_dev (float [batch*(N+M)][d], row b*(N+M) + t: the stream
+ * entering that block; layer = n_layers runs only the final RMSNorm and the LM head), on
+ * the current state's rows, without re-mask or embedding.  Outputs as dcl_forward_debug
+ * (any may be NULL); dcl_debug_hidden then reads the stream after each later block.  With
+ * commit = 1 the step's acceptance (steps (iii)-(iv) and the advance of p) then runs on
+ * these predictions, as in dcl_step.  Full recompute only, every sequence unfinished.
+ * Synchronises.  Errors: STATE (no prompt, or a finished sequence), INVALID_ARG,
+ * UNSUPPORTED (kv_cache = 1), CUDA. */
+dcl_status dcl_forward_debug_from(dcl_ctx* ctx, int32_t layer, const float* h_dev, int32_t commit,
+                                  void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev,
+                                  float* conf_dev, float* entropy_dev);
 
 /* Acceptance pass of one block from given logits (Eq. 2 confidence + Eq. compute_k +
  * Eq. draft_update), for B independent rows of P positions:
@@ -190,7 +218,9 @@ dcl_status dcl_debug_hidden(dcl_ctx* ctx, int32_t layer, float* h_dev);
  *                 window starts at p = c_b; rows with c_b >= P are left unchanged.
  *   x_dev         int32 [B][P], in/out: receives the committed ids and new drafts.
  *   cfg           thresholds, max_window (0 = P/2), min_commit, contiguous_drafts,
- *                 confidence (0: top-1 probability, 1: exp(-H) of the marginal entropy).
+ *                 confidence (0: top-1 probability, 1: exp(-H) of the marginal entropy),
+ *                 acceptance (0: DCV; 1: Eq. threshold_pd over the uncommitted positions
+ *                 [c_b, P), K = the number committed, no drafts).
  *   k_dev         int32 [B] out: K of every row.
  * Committed c_b and repeated calls: K depends on the logits and c_b only, so a second
  * call on its own output writes the same x.  Async on the context stream; 1 <= B,
@@ -264,9 +294,13 @@ dcl_status dcl_op_linear(dcl_ctx* ctx, const void* a_dev, const void* w_dev, voi
 /* Non-causal attention softmax(q k^T / sqrt(hd)) v over all T positions of each of
  * `batch` sequences (the attention of the bidirectional pass, Eq. 2).  qkv_dev bf16
  * [batch*T][(H+2G)*hd] (q | k | v column blocks, RoPE already applied), out_dev bf16
- * [batch*T][H*hd]; both 16-byte aligned.  hd in {64, 128}.  Synchronises. */
+ * [batch*T][H*hd]; both 16-byte aligned.  hd in {64, 128}.  q_rows > 0 (a multiple of 32,
+ * at most T) takes as queries only the last q_rows positions of each sequence (rows
+ * b*T + T - q_rows onwards), which attend to all T positions, and writes only those
+ * output rows (the suffix rows of a step with the key / value cache); 0 takes all T.
+ * Synchronises. */
 dcl_status dcl_op_attention(dcl_ctx* ctx, const void* qkv_dev, void* out_dev, int32_t batch,
-                            int32_t T, int32_t H, int32_t G, int32_t hd);
+                            int32_t T, int32_t H, int32_t G, int32_t hd, int32_t q_rows);
 
 /* LM head + softmax confidence fused (Eq. 2; top-1 of Eq. threshold_pd; top-2 of
  * Sec. 2.2): for each row r of x_dev (bf16 [R][d]), z = x_r @ w^T (w_dev bf16 [V][d]);
@@ -308,6 +342,14 @@ typedef enum {
  * records the timeout.  Returns DCL_ERR_TIMEOUT (the expected outcome) and leaves the
  * context usable; INVALID_ARG for another `which`.  Synchronises. */
 dcl_status dcl_selftest_wait_timeout(dcl_ctx* ctx, int32_t which);
+
+/* Launch floor of a step: a CUDA graph of n_kernels launches of an empty kernel (each
+ * one does only the dependent-launch handshake the step's kernels do, launched with the
+ * same programmatic-serialisation attribute) is captured on the context stream, launched
+ * 3 times untimed and `reps` times between CUDA events; *ms_per_graph receives the mean
+ * time of one graph.  A step of n_kernels launches cannot run faster.  Synchronises.
+ * Errors: INVALID_ARG (n_kernels outside [1, 100000], reps < 1, NULL output), CUDA. */
+dcl_status dcl_launch_floor(dcl_ctx* ctx, int32_t n_kernels, int32_t reps, float* ms_per_graph);
 
 /* enable = 1 re-captures the step graph with a pair of timing events (CUDA event record
  * nodes on the context stream) around every kernel; 0 restores the plain graph.

@@ -45,7 +45,7 @@ class DecodeConfig(ctypes.Structure):
                 ("max_window", ctypes.c_int32), ("block_len", ctypes.c_int32),
                 ("gen_len", ctypes.c_int32), ("kv_cache", ctypes.c_int32),
                 ("min_commit", ctypes.c_int32), ("contiguous_drafts", ctypes.c_int32),
-                ("confidence", ctypes.c_int32)]
+                ("confidence", ctypes.c_int32), ("acceptance", ctypes.c_int32)]
 
 
 class Stats(ctypes.Structure):
@@ -75,11 +75,13 @@ SIGNATURES = {
     "dcl_set_state": (_I, [_P, _P, _P]),
     "dcl_forward_debug": (_I, [_P, _P, _P, _P, _P, _P, _P]),
     "dcl_debug_hidden": (_I, [_P, _I, _P]),
+    "dcl_forward_debug_from": (_I, [_P, _I, _P, _I, _P, _P, _P, _P, _P, _P]),
+    "dcl_launch_floor": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_float)]),
     "dcl_accept": (_I, [_P, _P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P]),
     "dcl_accept_noalloc": (_I, [_P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P, _P]),
     "dcl_op_rmsnorm": (_I, [_P, _P, _P, _P, _I, _I, _F]),
     "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I]),
-    "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I]),
+    "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I]),
     "dcl_op_lmhead_top2": (_I, [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _I]),
     "dcl_op_generate": (_I, [_P, _P, ctypes.c_uint64, _I, ctypes.c_int64, ctypes.c_int64, _F, _F]),
     "dcl_selftest_wait_timeout": (_I, [_P, _I]),
@@ -144,10 +146,12 @@ def model_config(shape) -> ModelConfig:
 
 
 def decode_config(tau_commit=0.70, tau_draft=0.98, max_window=0, block_len=32, gen_len=0,
-                  kv_cache=0, min_commit=1, contiguous_drafts=0, confidence=0) -> DecodeConfig:
-    """confidence: 0 = top-1 probability, 1 = exp(-entropy)."""
+                  kv_cache=0, min_commit=1, contiguous_drafts=0, confidence=0,
+                  acceptance=0) -> DecodeConfig:
+    """confidence: 0 = top-1 probability, 1 = exp(-entropy); acceptance: 0 = DCV (contiguous),
+    1 = Eq. threshold_pd in the semi-autoregressive block."""
     return DecodeConfig(tau_commit, tau_draft, max_window, block_len, gen_len, kv_cache,
-                        min_commit, int(bool(contiguous_drafts)), confidence)
+                        min_commit, int(bool(contiguous_drafts)), confidence, acceptance)
 
 
 class Context:
@@ -251,6 +255,11 @@ class Context:
     def debug_hidden(self, layer, h):
         self._check(self._L.dcl_debug_hidden(self.ptr, layer, _ptr(h)))
 
+    def forward_debug_from(self, layer, h, commit=False, logits=None, top1=None, p1=None, p2=None, conf=None,
+                           entropy=None):
+        self._check(self._L.dcl_forward_debug_from(self.ptr, layer, _ptr(h), int(bool(commit)), _ptr(logits),
+                                                   _ptr(top1), _ptr(p1), _ptr(p2), _ptr(conf), _ptr(entropy)))
+
     def accept(self, logits, committed, x, cfg: DecodeConfig, k):
         B, P, V = logits.shape
         self._check(self._L.dcl_accept(self.ptr, _ptr(logits), B, P, V, _ptr(committed), _ptr(x),
@@ -265,8 +274,8 @@ class Context:
         N = w.shape[0]
         self._check(self._L.dcl_op_linear(self.ptr, _ptr(a), _ptr(w), _ptr(out), M, N, K, mode, tile))
 
-    def op_attention(self, qkv, out, batch, T, H, G, hd):
-        self._check(self._L.dcl_op_attention(self.ptr, _ptr(qkv), _ptr(out), batch, T, H, G, hd))
+    def op_attention(self, qkv, out, batch, T, H, G, hd, q_rows=0):
+        self._check(self._L.dcl_op_attention(self.ptr, _ptr(qkv), _ptr(out), batch, T, H, G, hd, q_rows))
 
     def op_lmhead_top2(self, x, w, top1, p1, p2, tile=0, entropy=None):
         R, d = x.shape
@@ -280,6 +289,12 @@ class Context:
     def selftest_wait_timeout(self, which):
         """Status of the bounded-wait self-test (DCL_ERR_TIMEOUT is the expected one)."""
         return self._L.dcl_selftest_wait_timeout(self.ptr, which)
+
+    def launch_floor(self, n_kernels, reps=200):
+        """Mean ms of a CUDA graph of n_kernels empty dependent launches."""
+        ms = ctypes.c_float()
+        self._check(self._L.dcl_launch_floor(self.ptr, n_kernels, reps, ctypes.byref(ms)))
+        return ms.value
 
     def set_profiling(self, enable):
         self._check(self._L.dcl_set_profiling(self.ptr, int(bool(enable))))

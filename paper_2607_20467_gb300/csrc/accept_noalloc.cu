@@ -59,7 +59,8 @@ extern "C" dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int3
                              .c_str());
     return DCL_ERR_INVALID_ARG;
   }
-  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1)) {
+  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1) ||
+      (cfg->acceptance != 0 && cfg->acceptance != 1)) {
     dcl::set_thread_error("dcl_accept_noalloc: bad decode config");
     return DCL_ERR_INVALID_ARG;
   }
@@ -78,7 +79,8 @@ extern "C" dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int3
   float* c1 = reinterpret_cast<float*>(ids + n);
   float* c2 = c1 + n;
   const int window = cfg->max_window > 0 ? cfg->max_window : (P / 2 > 0 ? P / 2 : 1);
-  dcl::DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts};
+  dcl::DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts,
+                     cfg->acceptance, P};
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = dcl::accept_stats_launch(static_cast<const __nv_bfloat16*>(logits_dev), committed_dev, B, P, V, ids, c1,
                                c2, cfg->confidence, s);

@@ -5,19 +5,19 @@
 // One CTA = 128 query rows of one (sequence, head); the key axis is walked once, in
 // blocks of 128: S_j = Q K_j^T into TMEM (double-buffered), then per row a running
 // maximum m, P_j = exp2(S_j * log2(e)/sqrt(hd) - m) with the row sum l kept in fp32, P_j
-// written to shared memory as a bf16 pair hi + lo (hi = P with its low 16 bits cleared,
-// lo = bf16(P - hi): about 16 significant bits together), and O += P_hi V_j + P_lo V_j
-// in TMEM.  m moves only when a block's maximum exceeds it by more than 8 (P stays below
-// 2^8); l and O are then scaled by the same factor, so O / l is unchanged.  O / l leaves
-// through TMA.
+// written to shared memory in fp16 (11 significant bits; P <= 2^8), and O += P_j V_j in
+// TMEM with V^T held in fp16 (the bf16 values of v, which fp16 holds exactly).  m moves
+// only when a block's maximum exceeds it by more than 8 (P stays below 2^8); l and O are
+// then scaled by the same factor, so O / l is unchanged.  O / l leaves through TMA.
 //
 // Roles (320 threads): warp 0 lane 0 TMA producer (Q once, then K / V^T blocks through a
-// 2-stage ring in the order the MMAs consume them); warp 1 allocates TMEM and its lane 0
+// 4-stage ring in the order the MMAs consume them); warp 1 allocates TMEM and its lane 0
 // issues the MMAs; warps 2..9 run the softmax and the epilogue, two warps per 32-row
 // band (TMEM lane quarter), each on one 64-column half of every S block: the block
 // maxima and the final sums of the two halves are combined through shared memory.  P is double-buffered so
 // that the softmax of block j + 1 overlaps the P V MMAs of block j.  V enters as V^T (a
-// K-major operand, kv contiguous), written by v_transpose_kernel from the q|k|v buffer.
+// K-major operand, kv contiguous, fp16), written by the QKV GEMM's epilogue or by
+// v_transpose_kernel from the q|k|v buffer.
 // Every wait is bounded (DERR_WAIT_TIMEOUT).
 #include "common.cuh"
 #include "tc_ptx.cuh"
@@ -27,7 +27,7 @@ namespace {
 
 constexpr int AT_THREADS = 320;
 constexpr int AT_SOFTMAX = 8;  // softmax warps (2 .. 9)
-constexpr int AT_STAGES = 2;
+constexpr int AT_STAGES = 4;
 constexpr int AT_BOX = 128 * 128;  // one 128-row x 128-byte swizzle box
 
 template <int HD>
@@ -36,19 +36,21 @@ struct AttnCfg {
   static constexpr int Q_BYTES = 128 * HD * 2;         // Q tile [128][HD]
   static constexpr int STAGE_BYTES = 128 * HD * 2;     // K block [128][HD] or V^T block [HD][128]
   static constexpr int VBOX = HD * 128;                // one V^T box: [HD rows][64 kv]
-  static constexpr int P_BYTES = 2 * 2 * 2 * AT_BOX;   // 2 buffers of P_hi and P_lo, [128][128] each
+  static constexpr int P_BYTES = 2 * 2 * AT_BOX;       // 2 buffers of P (fp16), [128][128] each
   static constexpr int BARS = 256;
   static constexpr int RED = 2 * 128 * 4;              // per-half row maxima / sums [2][128]
   static constexpr size_t SMEM = 1024 + (size_t)Q_BYTES + AT_STAGES * STAGE_BYTES + P_BYTES + BARS + RED;
   static constexpr uint32_t TMEM_COLS = 512;           // S double buffer (2 x 128) + O (HD)
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
-// vt[(b*G + g)*hd + d][t] = v of token t, kv head g, component d (row pitch Tp, zero pad).
-// A block moves a 64-token x 64-channel tile with 16-byte loads and stores.
+// vt[(b*G + g)*hd + d][t] = v of token t, kv head g, component d (row pitch Tp, zero pad),
+// in fp16 (the bf16 values, held exactly).  A block moves a 64-token x 64-channel tile
+// with 16-byte loads and stores.
 __global__ void __launch_bounds__(256) v_transpose_kernel(const __nv_bfloat16* __restrict__ qkv,
-                                                          __nv_bfloat16* __restrict__ vt, int T, int Tp, int cols,
+                                                          __half* __restrict__ vt, int T, int Tp, int cols,
                                                           int v0, int ghd) {
-  __shared__ __nv_bfloat16 tile[64][72];  // [channel][token], rows padded by 16 bytes
+  __shared__ __half tile[64][72];  // [channel][token], rows padded by 16 bytes
   pdl_wait();
   pdl_launch_dependents();
   const int t0 = blockIdx.x * 64, c0 = blockIdx.y * 64, b = blockIdx.z;
@@ -60,7 +62,7 @@ __global__ void __launch_bounds__(256) v_transpose_kernel(const __nv_bfloat16* _
       v = *reinterpret_cast<const uint4*>(qkv + ((size_t)b * T + t) * cols + v0 + c0 + cv);
     const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&v);
 #pragma unroll
-    for (int k = 0; k < 8; ++k) tile[cv + k][r] = e[k];
+    for (int k = 0; k < 8; ++k) tile[cv + k][r] = __float2half_rn(__bfloat162float(e[k]));
   }
   __syncthreads();
   for (int i = threadIdx.x; i < 64 * 8; i += 256) {
@@ -83,7 +85,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   uint8_t* smem = smem_raw + (base - raw);
   const uint32_t sQ = base;
   const uint32_t sKV = sQ + C::Q_BYTES;
-  const uint32_t sP = sKV + AT_STAGES * C::STAGE_BYTES;  // per buffer: P_hi boxes, then P_lo boxes
+  const uint32_t sP = sKV + AT_STAGES * C::STAGE_BYTES;  // per buffer: two 64-key boxes of P
   const uint32_t bars = sP + C::P_BYTES;
   const uint32_t q_full = bars;
   const uint32_t kv_full0 = bars + 8;                   // + 8 s
@@ -100,9 +102,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   float* red = reinterpret_cast<float*>(smem + (bars + C::BARS - base));  // [2][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  // grid (head, sequence, query tile): the query tile is the slowest index, so that the
+  // CTAs with work come first in dispatch order
+  const int h = blockIdx.x, b = blockIdx.y, qt = blockIdx.z;
   const int g = h / (H / G);
   const int nb = (T + 127) / 128;
+
+  pdl_wait();  // the previous kernels of the step (the row plan among them) have completed
+  pdl_launch_dependents();
+  // the query rows of sequence b are rows [off, off + len) of q and of the output; a tile
+  // past them has nothing to do and leaves before any set-up (uniform over the CTA)
+  const int q_off = seq_off ? seq_off[b] : b * T;
+  const int q_len = seq_len ? seq_len[b] : T;
+  if (qt * 128 >= q_len) return;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -132,17 +144,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *holder_ptr;
-  pdl_wait();  // the previous kernel of the step has completed
-  pdl_launch_dependents();
-  // the query rows of sequence b are rows [off, off + len) of q and of the output; a tile
-  // past them has nothing to do
-  const int q_off = seq_off ? seq_off[b] : b * T;
-  const int q_len = seq_len ? seq_len[b] : T;
-  const bool active = qt * 128 < q_len;
 
-  if (!active) {
-    // an empty query tile
-  } else if (warp == 0) {
+  if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------ TMA producer
       bool ok = true;
@@ -203,7 +206,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     if (lane == 0) {
       // ------------------------------------------------ MMA issuer
       constexpr uint32_t idesc_s = make_idesc(128, 128);
-      constexpr uint32_t idesc_o = make_idesc(128, HD);
+      constexpr uint32_t idesc_o = make_idesc_f16(128, HD);  // fp16 P and V
       bool ok = mbar_wait(q_full, 0, abort_flag);
       int stage = 0;
       uint32_t phase = 0;
@@ -236,20 +239,18 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         ++si;
         return true;
       };
-      auto issue_pv = [&](int j) -> bool {  // O += P_hi V_j + P_lo V_j
+      auto issue_pv = [&](int j) -> bool {  // O += P_j V_j (fp16 operands)
         uint32_t vaddr;
         if (!take(vaddr)) return false;
         const int pb = j & 1;
         if (!mbar_wait(p_full0 + 8 * pb, ((uint32_t)j >> 1) & 1u, abort_flag)) return false;
         tc_fence_after();
         const uint32_t d = tmem + 256u;
-        const uint32_t pbase = sP + (uint32_t)pb * 4 * AT_BOX;
+        const uint32_t pbase = sP + (uint32_t)pb * 2 * AT_BOX;
 #pragma unroll
-        for (int part = 0; part < 2; ++part)
-#pragma unroll
-          for (int k = 0; k < 8; ++k)
-            umma_bf16(d, sw128_desc(pbase + part * 2 * AT_BOX + (k >> 2) * AT_BOX) + 2 * (k & 3),
-                      sw128_desc(vaddr + (k >> 2) * C::VBOX) + 2 * (k & 3), idesc_o, (j > 0 || part > 0 || k > 0) ? 1u : 0u);
+        for (int k = 0; k < 8; ++k)
+          umma_bf16(d, sw128_desc(pbase + (k >> 2) * AT_BOX) + 2 * (k & 3), sw128_desc(vaddr + (k >> 2) * C::VBOX) + 2 * (k & 3),
+                    idesc_o, (j > 0 || k > 0) ? 1u : 0u);
         release();
         umma_commit(p_empty0 + 8 * pb);
         return true;
@@ -346,31 +347,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         l *= f;
       }
       if (raise) m = mb;
-      const uint32_t box = sP + (uint32_t)pb * 4 * AT_BOX + (uint32_t)hs * AT_BOX;
+      const uint32_t box = sP + (uint32_t)pb * 2 * AT_BOX + (uint32_t)hs * AT_BOX;
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
-        // P = hi + lo: hi = P with its low 16 bits cleared (a bf16 value), lo = P - hi
-        // (exact) rounded to bf16, so P is carried to about 2^-16 relative
-        uint32_t hb[32];
-        float lo[32];
+        // P in fp16 (round to nearest even: 2^-12 relative, P <= 2^8); l sums the fp32 values
+        float pv[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-          float pv = ex2_approx(fmaf(f32(v[c][e]), scale2, -m));
-          if (32 * c + e >= valid) pv = 0.f;
-          l += pv;
-          hb[e] = __float_as_uint(pv) & 0xFFFF0000u;
-          lo[e] = pv - __uint_as_float(hb[e]);
+          pv[e] = ex2_approx(fmaf(f32(v[c][e]), scale2, -m));
+          if (32 * c + e >= valid) pv[e] = 0.f;
+          l += pv[e];
         }
         const int k0 = c * 4;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          st_shared_v4(box + swz(r, k0 + k), __byte_perm(hb[8 * k], hb[8 * k + 1], 0x7632),
-                       __byte_perm(hb[8 * k + 2], hb[8 * k + 3], 0x7632), __byte_perm(hb[8 * k + 4], hb[8 * k + 5], 0x7632),
-                       __byte_perm(hb[8 * k + 6], hb[8 * k + 7], 0x7632));
-          st_shared_v4(box + 2 * AT_BOX + swz(r, k0 + k), pack_bf16x2(lo[8 * k], lo[8 * k + 1]),
-                       pack_bf16x2(lo[8 * k + 2], lo[8 * k + 3]), pack_bf16x2(lo[8 * k + 4], lo[8 * k + 5]),
-                       pack_bf16x2(lo[8 * k + 6], lo[8 * k + 7]));
-        }
+        for (int k = 0; k < 4; ++k)
+          st_shared_v4(box + swz(r, k0 + k), pack_f16x2(pv[8 * k], pv[8 * k + 1]), pack_f16x2(pv[8 * k + 2], pv[8 * k + 3]),
+                       pack_f16x2(pv[8 * k + 4], pv[8 * k + 5]), pack_f16x2(pv[8 * k + 6], pv[8 * k + 7]));
       }
       tc_fence_before();
       fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
@@ -443,7 +435,7 @@ cudaError_t launch_attn(const AttnPlan& p, int* err, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  dim3 grid((p.T + 127) / 128, p.H, p.batch);
+  dim3 grid(p.H, p.batch, (p.T + 127) / 128);
   return launch_pdl(kern, grid, AT_THREADS, AttnCfg<HD>::SMEM, stream, p.tq, p.tk, p.tv, p.to, p.T, p.H, p.G, p.kcol0,
                     p.seq_off, p.seq_len, err);
 }
@@ -452,7 +444,7 @@ cudaError_t launch_attn(const AttnPlan& p, int* err, cudaStream_t stream) {
 
 int attn_vt_pitch(int T) { return (T + 7) & ~7; }
 
-cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __nv_bfloat16* vt,
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __half* vt,
                            __nv_bfloat16* out, int batch, int T, int H, int G, int hd, int rows_max,
                            const int* seq_off, const int* seq_len) {
   if (batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128) || rows_max <= 0)
@@ -483,7 +475,7 @@ cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfl
     const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
     const uint64_t strides[2] = {Tp * 2, (uint64_t)hd * Tp * 2};
     const uint32_t box[3] = {64, (uint32_t)hd, 1};
-    if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
+    if (!encode_tmap(&p->tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_128B))
       return cudaErrorInvalidValue;
   }
   if (seq_off) {  // output rows of the step: [rows_max][H*hd] (32-row bands of one sequence)

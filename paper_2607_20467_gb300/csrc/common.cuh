@@ -4,6 +4,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -52,6 +53,11 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // ---------------------------------------------------------------- small helpers
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
@@ -155,17 +161,18 @@ bool encode_tmap(CUtensorMap* tm, CUtensorMapDataType dt, int rank, void* ptr, c
 // T; with tables every seq_len and seq_off is a multiple of 32), its keys and values are
 // all T positions: keys from kbuf [batch][T][G*hd] (NULL: the
 // k columns of qkv, rows b*T + t), values from vt [batch*G][hd][attn_vt_pitch(T)]
-// (v transposed: the attention_transpose_launch output, or what the QKV epilogue wrote).
+// (v transposed, in fp16 holding the bf16 values exactly: the attention_transpose_launch
+// output, or what the QKV epilogue wrote).
 struct AttnPlan {
   CUtensorMap tq, tk, tv, to;
   const __nv_bfloat16* qkv = nullptr;
-  __nv_bfloat16* vt = nullptr;
+  __half* vt = nullptr;
   const int* seq_off = nullptr;
   const int* seq_len = nullptr;
   int batch = 0, T = 0, H = 0, G = 0, hd = 0, kcol0 = 0;
 };
 int attn_vt_pitch(int T);
-cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __nv_bfloat16* vt,
+cudaError_t attention_plan(AttnPlan* p, const __nv_bfloat16* qkv, const __nv_bfloat16* kbuf, __half* vt,
                            __nv_bfloat16* out, int batch, int T, int H, int G, int hd, int rows_max,
                            const int* seq_off, const int* seq_len);
 cudaError_t attention_launch(const AttnPlan& p, int* err, cudaStream_t stream);  // both kernels
@@ -214,12 +221,16 @@ cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int ro
 struct DcvParams {
   float tau_commit, tau_draft;
   int window, min_commit, contiguous_drafts;
+  int acceptance = 0;  // 0: DCV (Eq. compute_k + Eq. draft_update); 1: Eq. threshold_pd
+  int block_len = 0;   // acceptance 1: the semi-autoregressive block the rule applies to
 };
 // One step's acceptance on the generation rows: ids/c (and ent) are [batch][M] (position
 // N + i).  With ent, jpde[b] accumulates Eq. entropy_bound of the set row b commits.
+// cmt: committed flags [batch][N + M] (read and written with acceptance 1 only).
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
                               const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
-                              int N, int M, const DcvParams& prm, int32_t* done_count, cudaStream_t stream);
+                              int N, int M, const DcvParams& prm, int32_t* done_count, uint8_t* cmt,
+                              cudaStream_t stream);
 // Block acceptance from bf16 logits (dcl_accept): c1 = p1 (mode 0) or exp(-H) (mode 1).
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B,
                                 int P, int V, int32_t* ids, float* c1, float* c2, int mode,
@@ -227,6 +238,8 @@ cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* comm
 cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, const float* c1,
                                  int32_t* x, int32_t* k, int B, int P, const DcvParams& prm,
                                  cudaStream_t stream);
+// One launch of a kernel that does only the dependent-launch handshake (launch floor).
+cudaError_t empty_launch(cudaStream_t stream);
 // Counter-based weight generator (SplitMix64 + Irwin-Hall(4)), with an optional
 // row remap: element e of a [rows][cols] tensor goes to
 // dst[(e/cols) / blk * blk_stride + blk_off + (e/cols) % blk) * cols + e % cols]

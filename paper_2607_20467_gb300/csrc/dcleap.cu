@@ -1,6 +1,7 @@
 // C ABI of libdcleap.so (include/dcleap.h): the context, weight layout, the captured
 // CUDA graph of one denoise step (Sec. 3.3 steps (i)-(iv), Algorithm 1), the host
 // loop of Algorithm 1, and single-kernel entry points for parity tests.
+#include <algorithm>
 #include <chrono>
 #include <cstdarg>
 #include <cstdio>
@@ -51,7 +52,7 @@ struct dcl_ctx {
   // activations, sized for max_batch * max_seq rows
   float* h = nullptr;
   __nv_bfloat16 *xn = nullptr, *qkv = nullptr, *attn = nullptr, *act = nullptr, *xg = nullptr;
-  __nv_bfloat16* vt = nullptr;    // v transposed for the attention kernel (full recompute)
+  __half* vt = nullptr;           // v transposed (fp16) for the attention kernel (full recompute)
   __nv_bfloat16* kbuf = nullptr;  // keys after RoPE [B][T][G*hd] (full recompute)
   __nv_bfloat16* kvstore = nullptr;  // approximate cache: per layer keys [B][T][G*hd], v^T
   size_t kvstore_bytes = 0;
@@ -66,6 +67,7 @@ struct dcl_ctx {
   float* jpde = nullptr;  // per row: Eq. entropy_bound summed over the committed sets
   int32_t *x = nullptr, *p = nullptr, *k = nullptr, *steps = nullptr, *done_count = nullptr;
   int32_t *x_init = nullptr, *p_init = nullptr;  // state at the last dcl_set_prompt
+  uint8_t *cmt = nullptr, *cmt_init = nullptr;    // committed flags [B][T] (Eq. threshold_pd decoding)
   int* derr = nullptr;
   float *rope_cos = nullptr, *rope_sin = nullptr;
   float* snap = nullptr;  // residual stream after the embedding and after each layer (debug)
@@ -208,8 +210,11 @@ struct Enq {
   }
 };
 
-// Enqueue the forward (and, if with_dcv, the acceptance) on the context stream.
-cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, const char** what) {
+// Enqueue the forward (and, if with_dcv, the acceptance) on the context stream.  With
+// h_in the forward starts at block first_layer from that residual stream (row b*T + t;
+// no re-mask, no embedding; full recompute only).
+cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, const char** what,
+                         int first_layer = 0, const float* h_in = nullptr) {
   const dcl_model_config& m = c->cfg;
   const int R = c->B * c->T;
   const int d = m.d_model;
@@ -219,13 +224,21 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
   q.end(row_plan_launch(c->rp, c->p, c->B, c->N, c->T, c->dcfg.block_len, c->dcfg.kv_cache, with_dcv ? 1 : 0,
                         c->stream),
         "row_plan");
-  q.begin(DCL_K_EMBED);
-  q.end(embed_remask_launch(c->x, c->p, c->B, c->T, c->window, m.mask_id, m.vocab, c->embed, d, c->h,
-                            c->derr, c->rp, c->stream),
-        "embed");
+  if (h_in) {
+    if (q.err == cudaSuccess)
+      q.err = cudaMemcpyAsync(c->h, h_in, sizeof(float) * R * d, cudaMemcpyDeviceToDevice, c->stream);
+  } else {
+    first_layer = 0;
+    q.begin(DCL_K_EMBED);
+    // (the threshold rule keeps no drafts: nothing to re-mask)
+    q.end(embed_remask_launch(c->x, c->p, c->B, c->T, c->dcfg.acceptance ? 0 : c->window, m.mask_id, m.vocab,
+                              c->embed, d, c->h, c->derr, c->rp, c->stream),
+          "embed");
+  }
   if (snapshots && q.err == cudaSuccess)
-    q.err = cudaMemcpyAsync(c->snap, c->h, sizeof(float) * R * d, cudaMemcpyDeviceToDevice, c->stream);
-  for (int l = 0; l < m.n_layers && q.err == cudaSuccess; ++l) {
+    q.err = cudaMemcpyAsync(c->snap + (size_t)first_layer * R * d, c->h, sizeof(float) * R * d,
+                            cudaMemcpyDeviceToDevice, c->stream);
+  for (int l = first_layer; l < m.n_layers && q.err == cudaSuccess; ++l) {
     const Layer& L = c->layers[l];
     const GemmPlan* P = &c->plans[4 * l];
     q.begin(DCL_K_RMSNORM);
@@ -270,10 +283,10 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
         "combine");
   if (with_dcv) {
     DcvParams prm{c->dcfg.tau_commit, c->dcfg.tau_draft, c->window, c->dcfg.min_commit,
-                  c->dcfg.contiguous_drafts};
+                  c->dcfg.contiguous_drafts, c->dcfg.acceptance, c->dcfg.block_len};
     q.begin(DCL_K_DCV);
     q.end(dcv_commit_launch(c->x, c->p, c->k, c->steps, c->top1, co.conf, c->ent, c->jpde, c->B, c->N, c->M, prm,
-                            c->done_count, c->stream),
+                            c->done_count, c->cmt, c->stream),
           "dcv_commit");
   }
   if (what) *what = q.what;
@@ -354,7 +367,9 @@ dcl_status build_plans(dcl_ctx* c) {
     }
   }
   auto kbuf_of = [&](int l) { return cached ? c->kvstore + (size_t)l * (k_elems + v_elems) : c->kbuf; };
-  auto vbuf_of = [&](int l) { return cached ? c->kvstore + (size_t)l * (k_elems + v_elems) + k_elems : c->vt; };
+  auto vbuf_of = [&](int l) {  // (the store's v^T part holds fp16, 2 bytes per element like the keys)
+    return cached ? reinterpret_cast<__half*>(c->kvstore + (size_t)l * (k_elems + v_elems) + k_elems) : c->vt;
+  };
   for (int l = 0; l < m.n_layers; ++l) {
     const Layer& L = c->layers[l];
     EpiParams e0;
@@ -401,12 +416,13 @@ dcl_status build_plans(dcl_ctx* c) {
     }
   }
   c->attn_plans.assign(m.n_layers, AttnPlan{});
-  for (int l = 0; l < m.n_layers; ++l)
+  for (int l = 0; l < m.n_layers; ++l) {
     // (without the fused key store the rows are the identity layout b*T + t: no tables)
     if (attention_plan(&c->attn_plans[l], c->qkv, c->kv_fused ? kbuf_of(l) : nullptr, vbuf_of(l), c->attn, c->B, c->T,
                        H, G, hd, R, c->kv_fused ? c->rp.seq_off : nullptr, c->kv_fused ? c->rp.seq_len : nullptr) !=
         cudaSuccess)
       return fail(c, DCL_ERR_UNSUPPORTED, "attention plan failed");
+  }
   EpiParams el;
   el.out = c->part;
   el.ent_part = c->ent_part;
@@ -631,7 +647,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->xn = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->qkv = (__nv_bfloat16*)dev_alloc(c, 2 * R * (H + 2 * G) * hd);
     c->attn = (__nv_bfloat16*)dev_alloc(c, 2 * R * H * hd);
-    c->vt = (__nv_bfloat16*)dev_alloc(c, 2 * (size_t)max_batch * G * hd * attn_vt_pitch(max_seq));
+    c->vt = (__half*)dev_alloc(c, 2 * (size_t)max_batch * G * hd * attn_vt_pitch(max_seq));
     c->kbuf = (__nv_bfloat16*)dev_alloc(c, 2 * R * G * hd);
     c->rp_buf = (int*)dev_alloc(c, sizeof(int) * (2 + 4 * R + 3 * (size_t)max_batch));
     c->act = (__nv_bfloat16*)dev_alloc(c, 2 * R * F);
@@ -651,11 +667,13 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->done_count = (int32_t*)dev_alloc(c, 16);
     c->x_init = (int32_t*)dev_alloc(c, 4 * R);
     c->p_init = (int32_t*)dev_alloc(c, 4 * max_batch);
+    c->cmt = (uint8_t*)dev_alloc(c, R);
+    c->cmt_init = (uint8_t*)dev_alloc(c, R);
     c->rope_cos = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
     c->rope_sin = (float*)dev_alloc(c, 4 * (size_t)max_seq * hd / 2);
     if (!c->wbuf || !c->h || !c->xn || !c->qkv || !c->attn || !c->vt || !c->kbuf || !c->rp_buf || !c->act || !c->xg || !c->part || !c->ent_part ||
         !c->ent || !c->conf || !c->jpde || !c->top1 ||
-        !c->p1 || !c->p2 || !c->x || !c->p || !c->k || !c->steps || !c->done_count || !c->x_init || !c->p_init || !c->rope_cos ||
+        !c->p1 || !c->p2 || !c->x || !c->p || !c->k || !c->steps || !c->done_count || !c->x_init || !c->p_init || !c->cmt || !c->cmt_init || !c->rope_cos ||
         !c->rope_sin) {
       dev_free_all(c);
       release_stream(c);
@@ -767,6 +785,9 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
     return fail(c, DCL_ERR_INVALID_ARG, "N + M = %d + %d exceeds max_seq %d", n_prompt, cfg->gen_len, c->max_seq);
   if (cfg->kv_cache != 0 && cfg->kv_cache != 1) return fail(c, DCL_ERR_INVALID_ARG, "kv_cache must be 0 or 1");
   if (cfg->confidence != 0 && cfg->confidence != 1) return fail(c, DCL_ERR_INVALID_ARG, "confidence must be 0 or 1");
+  if (cfg->acceptance != 0 && cfg->acceptance != 1) return fail(c, DCL_ERR_INVALID_ARG, "acceptance must be 0 or 1");
+  if (cfg->acceptance == 1 && cfg->block_len <= 0)
+    return fail(c, DCL_ERR_INVALID_ARG, "the threshold rule (acceptance = 1) needs block_len >= 1");
   if (cfg->kv_cache && (cfg->block_len <= 0 || cfg->block_len % 32 || n_prompt % 32 || cfg->gen_len % 32))
     return fail(c, DCL_ERR_UNSUPPORTED, "the key / value cache needs N, M and the block length multiples of 32");
   if (cfg->max_window < 0 || cfg->min_commit < 0 || !(cfg->tau_commit == cfg->tau_commit) ||
@@ -785,14 +806,19 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   c->window = window;
   c->dcfg = *cfg;
   std::vector<int32_t> xh((size_t)batch * c->T, c->cfg.mask_id), ph(batch, n_prompt), zero(batch, 0);
-  for (int b = 0; b < batch; ++b)
+  std::vector<uint8_t> ch((size_t)batch * c->T, 0);
+  for (int b = 0; b < batch; ++b) {
     memcpy(&xh[(size_t)b * c->T], prompt + (size_t)b * n_prompt, sizeof(int32_t) * n_prompt);
+    memset(&ch[(size_t)b * c->T], 1, n_prompt);
+  }
   CUDA_TRY(c, cudaMemcpyAsync(c->x, xh.data(), 4 * xh.size(), cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p, ph.data(), 4 * batch, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->steps, zero.data(), 4 * batch, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->k, zero.data(), 4 * batch, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->x_init, c->x, 4 * xh.size(), cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p_init, c->p, 4 * batch, cudaMemcpyDeviceToDevice, c->stream));
+  CUDA_TRY(c, cudaMemcpyAsync(c->cmt, ch.data(), ch.size(), cudaMemcpyHostToDevice, c->stream));
+  CUDA_TRY(c, cudaMemcpyAsync(c->cmt_init, c->cmt, ch.size(), cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)batch, c->stream));  // no stored keys / values
   CUDA_TRY(c, cudaMemsetAsync(c->jpde, 0, 4 * (size_t)batch, c->stream));
   s = reset_done_count(c, ph.data());
@@ -884,6 +910,7 @@ dcl_status dcl_restart(dcl_ctx* c) {
   const size_t B = c->B;
   CUDA_TRY(c, cudaMemcpyAsync(c->x, c->x_init, 4 * B * c->T, cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p, c->p_init, 4 * B, cudaMemcpyDeviceToDevice, c->stream));
+  CUDA_TRY(c, cudaMemcpyAsync(c->cmt, c->cmt_init, B * c->T, cudaMemcpyDeviceToDevice, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->steps, 0, 4 * B, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->k, 0, 4 * B, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->done_count, 0, 4, c->stream));
@@ -909,6 +936,13 @@ dcl_status dcl_set_state(dcl_ctx* c, const int32_t* x, const int32_t* p) {
   if (s != DCL_OK) return s;
   for (int b = 0; b < c->B; ++b)
     if (p[b] < c->N || p[b] > c->T) return fail(c, DCL_ERR_INVALID_ARG, "p[%d] = %d outside [N, N+M]", b, p[b]);
+  // committed flags (read by the threshold rule only): every position before p, and every
+  // later position that holds a token other than MASK
+  std::vector<uint8_t> ch((size_t)c->B * c->T);
+  for (int b = 0; b < c->B; ++b)
+    for (int i = 0; i < c->T; ++i)
+      ch[(size_t)b * c->T + i] = (i < p[b] || x[(size_t)b * c->T + i] != c->cfg.mask_id) ? 1 : 0;
+  CUDA_TRY(c, cudaMemcpyAsync(c->cmt, ch.data(), ch.size(), cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->x, x, 4 * (size_t)c->B * c->T, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemcpyAsync(c->p, p, 4 * (size_t)c->B, cudaMemcpyHostToDevice, c->stream));
   CUDA_TRY(c, cudaMemsetAsync(c->rp.pe_cache, 0xff, 4 * (size_t)c->B, c->stream));  // the next step refreshes
@@ -916,10 +950,11 @@ dcl_status dcl_set_state(dcl_ctx* c, const int32_t* x, const int32_t* p) {
   return reset_done_count(c, p);
 }
 
-dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev,
-                             float* conf_dev, float* entropy_dev) {
-  if (!c) return DCL_ERR_INVALID_ARG;
-  if (!c->prompt_set) return fail(c, DCL_ERR_STATE, "no prompt set");
+namespace {
+// The parity hooks' common body: the forward (from the embedding, or from block `layer` on
+// h_in), optionally the acceptance, then copies of the predictions.
+dcl_status forward_debug_impl(dcl_ctx* c, int layer, const float* h_in, bool commit, void* logits_dev,
+                              int32_t* top1_dev, float* p1_dev, float* p2_dev, float* conf_dev, float* entropy_dev) {
   const size_t R = (size_t)c->B * c->T;
   if (!c->snap || c->snap_rows < R) {
     c->snap = (float*)dev_alloc(c, sizeof(float) * (c->cfg.n_layers + 1) * R * c->cfg.d_model);
@@ -927,7 +962,7 @@ dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, fl
     c->snap_rows = R;
   }
   const char* what = nullptr;
-  cudaError_t e = enqueue_step(c, false, false, true, &what);
+  cudaError_t e = enqueue_step(c, commit, false, true, &what, layer, h_in);
   if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "forward failed at %s: %s", what ? what : "?", cudaGetErrorString(e));
   const size_t G = (size_t)c->B * c->M;
   if (top1_dev) CUDA_TRY(c, cudaMemcpyAsync(top1_dev, c->top1, 4 * G, cudaMemcpyDeviceToDevice, c->stream));
@@ -953,6 +988,33 @@ dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, fl
   }
   return check_device(c);
 }
+}  // namespace
+
+dcl_status dcl_forward_debug(dcl_ctx* c, void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev,
+                             float* conf_dev, float* entropy_dev) {
+  if (!c) return DCL_ERR_INVALID_ARG;
+  if (!c->prompt_set) return fail(c, DCL_ERR_STATE, "no prompt set");
+  return forward_debug_impl(c, 0, nullptr, false, logits_dev, top1_dev, p1_dev, p2_dev, conf_dev, entropy_dev);
+}
+
+dcl_status dcl_forward_debug_from(dcl_ctx* c, int32_t layer, const float* h_dev, int32_t commit, void* logits_dev,
+                                  int32_t* top1_dev, float* p1_dev, float* p2_dev, float* conf_dev,
+                                  float* entropy_dev) {
+  if (!c) return DCL_ERR_INVALID_ARG;
+  if (!c->prompt_set) return fail(c, DCL_ERR_STATE, "no prompt set");
+  if (!h_dev || layer < 0 || layer > c->cfg.n_layers || (commit != 0 && commit != 1))
+    return fail(c, DCL_ERR_INVALID_ARG, "bad layer / h / commit");
+  if (c->dcfg.kv_cache) return fail(c, DCL_ERR_UNSUPPORTED, "a forward from a given stream needs full recompute");
+  // the stream's rows are every (sequence, position): no sequence may have finished (a
+  // finished sequence contributes no rows to the step)
+  std::vector<int32_t> ph(c->B);
+  CUDA_TRY(c, cudaMemcpyAsync(ph.data(), c->p, 4 * (size_t)c->B, cudaMemcpyDeviceToHost, c->stream));
+  CUDA_TRY(c, cudaStreamSynchronize(c->stream));
+  for (int b = 0; b < c->B; ++b)
+    if (ph[b] >= c->T) return fail(c, DCL_ERR_STATE, "sequence %d has finished", b);
+  return forward_debug_impl(c, layer, h_dev, commit != 0, logits_dev, top1_dev, p1_dev, p2_dev, conf_dev,
+                            entropy_dev);
+}
 
 dcl_status dcl_debug_hidden(dcl_ctx* c, int32_t layer, float* h_dev) {
   if (!c) return DCL_ERR_INVALID_ARG;
@@ -971,7 +1033,8 @@ dcl_status dcl_accept(dcl_ctx* c, const void* logits_dev, int32_t B, int32_t P, 
   if (!logits_dev || !committed_dev || !x_dev || !cfg || !k_dev) return fail(c, DCL_ERR_INVALID_ARG, "NULL argument");
   if (B <= 0 || P <= 0 || V <= 1 || P > 4096 || (int64_t)B * P > (1 << 20))
     return fail(c, DCL_ERR_INVALID_ARG, "bad B/P/V (P <= 4096, B*P <= 2^20)");
-  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1))
+  if (cfg->max_window < 0 || cfg->min_commit < 0 || (cfg->confidence != 0 && cfg->confidence != 1) ||
+      (cfg->acceptance != 0 && cfg->acceptance != 1))
     return fail(c, DCL_ERR_INVALID_ARG, "bad decode config");
   const size_t n = (size_t)B * P;
   if (c->acc_cap < n) {
@@ -982,7 +1045,8 @@ dcl_status dcl_accept(dcl_ctx* c, const void* logits_dev, int32_t B, int32_t P, 
     c->acc_cap = n;
   }
   const int window = cfg->max_window > 0 ? cfg->max_window : (P / 2 > 0 ? P / 2 : 1);
-  DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts};
+  DcvParams prm{cfg->tau_commit, cfg->tau_draft, window, cfg->min_commit, cfg->contiguous_drafts,
+                cfg->acceptance, P};
   CUDA_TRY(c, accept_stats_launch(static_cast<const __nv_bfloat16*>(logits_dev), committed_dev, B, P, V, c->acc_ids,
                                   c->acc_c1, c->acc_c2, cfg->confidence, c->stream));
   CUDA_TRY(c, accept_commit_launch(committed_dev, c->acc_ids, c->acc_c1, x_dev, k_dev, B, P, prm, c->stream));
@@ -1020,26 +1084,44 @@ dcl_status dcl_op_linear(dcl_ctx* c, const void* a_dev, const void* w_dev, void*
 }
 
 dcl_status dcl_op_attention(dcl_ctx* c, const void* qkv_dev, void* out_dev, int32_t batch, int32_t T, int32_t H,
-                            int32_t G, int32_t hd) {
+                            int32_t G, int32_t hd, int32_t q_rows) {
   if (!c) return DCL_ERR_INVALID_ARG;
-  if (!qkv_dev || !out_dev || batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128))
+  if (!qkv_dev || !out_dev || batch <= 0 || T <= 0 || H <= 0 || G <= 0 || H % G || (hd != 64 && hd != 128) ||
+      q_rows < 0 || q_rows > T || q_rows % 32)
     return fail(c, DCL_ERR_INVALID_ARG, "bad attention args");
-  __nv_bfloat16* vt = static_cast<__nv_bfloat16*>(dev_alloc(c, 2 * (size_t)batch * G * hd * attn_vt_pitch(T)));
-  if (!vt) return fail(c, DCL_ERR_OOM, "attention scratch allocation failed");
+  __half* vt = static_cast<__half*>(dev_alloc(c, 2 * (size_t)batch * G * hd * attn_vt_pitch(T)));
+  int* tab = q_rows > 0 ? static_cast<int*>(dev_alloc(c, sizeof(int) * 2 * (size_t)batch)) : nullptr;
+  auto release = [&]() {
+    cudaStreamSynchronize(c->stream);
+    dev_free_one(c, vt);
+    dev_free_one(c, tab);
+  };
+  if (!vt || (q_rows > 0 && !tab)) {
+    release();
+    return fail(c, DCL_ERR_OOM, "attention scratch allocation failed");
+  }
+  if (tab) {  // sequence b's queries: positions [T - q_rows, T), rows b*T + T - q_rows onwards
+    std::vector<int> th(2 * (size_t)batch);
+    for (int b = 0; b < batch; ++b) {
+      th[b] = b * T + T - q_rows;
+      th[batch + b] = q_rows;
+    }
+    CUDA_TRY(c, cudaMemcpyAsync(tab, th.data(), sizeof(int) * th.size(), cudaMemcpyHostToDevice, c->stream));
+    CUDA_TRY(c, cudaStreamSynchronize(c->stream));
+  }
   AttnPlan pl;
   if (attention_plan(&pl, static_cast<const __nv_bfloat16*>(qkv_dev), nullptr, vt, static_cast<__nv_bfloat16*>(out_dev),
-                     batch, T, H, G, hd, batch * T, nullptr, nullptr) != cudaSuccess) {
-    dev_free_one(c, vt);
+                     batch, T, H, G, hd, batch * T, tab, tab ? tab + batch : nullptr) != cudaSuccess) {
+    release();
     return fail(c, DCL_ERR_INVALID_ARG, "attention: operands must be 16-byte aligned");
   }
   const cudaError_t e = attention_launch(pl, c->derr, c->stream);
   if (e != cudaSuccess) {
-    cudaStreamSynchronize(c->stream);
-    dev_free_one(c, vt);
+    release();
     return fail(c, DCL_ERR_CUDA, "attention launch: %s", cudaGetErrorString(e));
   }
   const dcl_status s = check_device(c);
-  dev_free_one(c, vt);
+  release();
   return s;
 }
 
@@ -1109,6 +1191,36 @@ dcl_status dcl_selftest_wait_timeout(dcl_ctx* c, int32_t which) {
   const dcl_status s = check_device(c);
   dev_free_one(c, flag);
   return s;
+}
+
+dcl_status dcl_launch_floor(dcl_ctx* c, int32_t n_kernels, int32_t reps, float* ms_per_graph) {
+  if (!c) return DCL_ERR_INVALID_ARG;
+  if (n_kernels < 1 || n_kernels > 100000 || reps < 1 || !ms_per_graph)
+    return fail(c, DCL_ERR_INVALID_ARG, "need 1 <= n_kernels <= 100000, reps >= 1 and an output");
+  cudaGraph_t g = nullptr;
+  cudaGraphExec_t ge = nullptr;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  cudaError_t e = cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal);
+  for (int i = 0; i < n_kernels && e == cudaSuccess; ++i) e = empty_launch(c->stream);
+  cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
+  if (e == cudaSuccess) e = e2;
+  if (e == cudaSuccess) e = cudaGraphInstantiate(&ge, g, 0);
+  if (e == cudaSuccess) e = cudaEventCreate(&e0);
+  if (e == cudaSuccess) e = cudaEventCreate(&e1);
+  for (int i = 0; i < 3 && e == cudaSuccess; ++i) e = cudaGraphLaunch(ge, c->stream);  // warm-up
+  if (e == cudaSuccess) e = cudaEventRecord(e0, c->stream);
+  for (int i = 0; i < reps && e == cudaSuccess; ++i) e = cudaGraphLaunch(ge, c->stream);
+  if (e == cudaSuccess) e = cudaEventRecord(e1, c->stream);
+  if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+  float ms = 0.f;
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  if (ge) cudaGraphExecDestroy(ge);
+  if (g) cudaGraphDestroy(g);
+  if (e != cudaSuccess) return fail(c, DCL_ERR_CUDA, "launch floor: %s", cudaGetErrorString(e));
+  *ms_per_graph = ms / reps;
+  return DCL_OK;
 }
 
 dcl_status dcl_set_profiling(dcl_ctx* c, int32_t enable) {

@@ -713,7 +713,8 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
       }
     } else if (ep.vt_heads > 0) {
       // v columns leave transposed, as the attention's K-major operand: boxes of 64
-      // channels x 32 tokens of vt [batch * G][hd][T]
+      // channels x 32 tokens of vt [batch * G][hd][T], in fp16 (the attention multiplies P in
+      // fp16 by them; the bf16-rounded v is held exactly)
 #pragma unroll 1
       for (int c = 0; c < W && n0 + c < N; c += 64) {
         const int cv = n0 + c - ep.rope_cols, g = cv / ep.head_dim, d0 = cv - g * ep.head_dim;
@@ -723,7 +724,9 @@ __device__ __forceinline__ void epilogue_pair(const Src& s, Stage& o, const CUte
           float v[32];
           src_cols(s, c + 32 * h, v);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) st_shared_u16(b + (uint32_t)((32 * h + e) * 64 + 2 * o.lane), bf16_bits(v[e]));
+          for (int e = 0; e < 32; ++e)
+            st_shared_u16(b + (uint32_t)((32 * h + e) * 64 + 2 * o.lane),
+                          __half_as_ushort(__float2half_rn(__bfloat162float(__float2bfloat16_rn(v[e])))));
         }
         o.issue3(tmv, b, t0, d0, bz * ep.vt_heads + g);
       }
@@ -1751,7 +1754,7 @@ bool gemm_fuse_kv(GemmPlan* p, void* kbuf, void* vt, int batch, int T, int H, in
     const uint64_t dims[3] = {(uint64_t)T, (uint64_t)hd, (uint64_t)batch * G};
     const uint64_t strides[2] = {(uint64_t)Tp * 2, (uint64_t)hd * Tp * 2};
     const uint32_t box[3] = {32, 64, 1};
-    if (!encode_tmap(&tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE))
+    if (!encode_tmap(&tv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, vt, dims, strides, box, CU_TENSOR_MAP_SWIZZLE_NONE))
       return false;
   }
   {

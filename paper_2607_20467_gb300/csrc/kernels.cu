@@ -323,11 +323,92 @@ __device__ int dcv_row(int32_t* xrow, const int32_t* ids, const float* c, int pb
   return K;
 }
 
+// ------------------------------------------------------------------ Eq. threshold_pd
+// The non-contiguous rule on one row, one full warp: every uncommitted position of
+// [lo, hi) with c > tau_commit is committed in the same step (Eq. threshold_pd, applied
+// independently per position); when fewer than min_commit pass, the min_commit
+// uncommitted positions of highest confidence are committed instead (ties to the lower
+// position: round r takes the best position ranked strictly after round r-1's, so nothing
+// needs marking).  cmt (committed flags by absolute position) may be NULL: then every
+// position of [lo, hi) is uncommitted.  Returns the number committed; *hsum / *hmax get the
+// sum and maximum of ent over the committed set (warp-uniform; ent may be NULL).
+__device__ int threshold_row(int32_t* xrow, uint8_t* cmt, const int32_t* ids, const float* c, const float* ent,
+                             int lo, int hi, const DcvParams& prm, float* hsum, float* hmax) {
+  const int lane = threadIdx.x & 31;
+  int npass = 0;
+  for (int base = lo; base < hi; base += 32) {
+    const int i = base + lane;
+    const bool ok = i < hi && !(cmt && cmt[i]) && c[i] > prm.tau_commit;
+    npass += __popc(__ballot_sync(kFull, ok));
+  }
+  float hs = 0.f, hm = 0.f;
+  int K = 0;
+  if (npass >= prm.min_commit) {
+    for (int i = lo + lane; i < hi; i += 32) {
+      if (!(cmt && cmt[i]) && c[i] > prm.tau_commit) {
+        xrow[i] = ids[i];
+        if (cmt) cmt[i] = 1;
+        if (ent) {
+          hs += ent[i];
+          hm = fmaxf(hm, ent[i]);
+        }
+      }
+    }
+    K = npass;
+  } else {
+    float pc = INFINITY;  // the previous pick's key (confidence, position)
+    int pi = -1;
+    for (int r = 0; r < prm.min_commit; ++r) {
+      float bc = -INFINITY;
+      int bi = 0x7fffffff;
+      for (int i = lo + lane; i < hi; i += 32) {
+        if (cmt && cmt[i]) continue;
+        const float ci = c[i];
+        const bool after = ci < pc || (ci == pc && i > pi);  // ranked after the previous pick
+        if (after && (ci > bc || (ci == bc && i < bi))) {
+          bc = ci;
+          bi = i;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float oc = __shfl_xor_sync(kFull, bc, o);
+        const int oi = __shfl_xor_sync(kFull, bi, o);
+        if (oc > bc || (oc == bc && oi < bi)) {
+          bc = oc;
+          bi = oi;
+        }
+      }
+      if (bi == 0x7fffffff) break;  // no uncommitted position left in the block
+      if (lane == 0) {
+        xrow[bi] = ids[bi];
+        if (cmt) cmt[bi] = 1;
+        if (ent) {
+          hs += ent[bi];
+          hm = fmaxf(hm, ent[bi]);
+        }
+      }
+      pc = bc;
+      pi = bi;
+      ++K;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    hs += __shfl_xor_sync(kFull, hs, o);
+    hm = fmaxf(hm, __shfl_xor_sync(kFull, hm, o));
+  }
+  *hsum = hs;
+  *hmax = hm;
+  __syncwarp();  // this warp's commits (x and flags) are visible to all its lanes
+  return K;
+}
+
 __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__ p,
                                   int32_t* __restrict__ k_out, int32_t* __restrict__ steps,
                                   const int32_t* __restrict__ ids, const float* __restrict__ c,
                                   const float* __restrict__ ent, float* __restrict__ jpde, int N, int M,
-                                  DcvParams prm, int32_t* done_count) {
+                                  DcvParams prm, int32_t* done_count, uint8_t* __restrict__ cmt) {
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.x;
@@ -335,6 +416,32 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
   const int pb = p[b];
   if (pb >= T) {
     if (threadIdx.x == 0) k_out[b] = 0;
+    return;
+  }
+  if (prm.acceptance == 1) {
+    // Eq. threshold_pd in the semi-autoregressive block holding p, then p moves to the
+    // leftmost uncommitted position
+    const int lo = N + prm.block_len * ((pb - N) / prm.block_len), hi = min(lo + prm.block_len, T);
+    uint8_t* crow = cmt + (size_t)b * T;
+    float hs, hm;
+    const int K = threshold_row(x + (size_t)b * T, crow, ids + (size_t)b * M - N, c + (size_t)b * M - N,
+                                ent ? ent + (size_t)b * M - N : nullptr, lo, hi, prm, &hs, &hm);
+    int np = T;
+    for (int base = pb; base < T; base += 32) {
+      const int i = base + (threadIdx.x & 31);
+      const unsigned bal = __ballot_sync(kFull, i < T && !crow[i]);
+      if (bal) {
+        np = base + __ffs(bal) - 1;
+        break;
+      }
+    }
+    if (threadIdx.x == 0) {
+      if (ent) jpde[b] += K > 1 ? hs - hm : 0.f;
+      k_out[b] = K;
+      p[b] = np;
+      steps[b] += 1;
+      if (np >= T) atomicAdd(done_count, 1);
+    }
     return;
   }
   // shift the [M]-sized generation arrays so they are indexed by absolute position
@@ -427,19 +534,60 @@ __device__ __forceinline__ void take8(Part& a, const uint4& q, int col) {
   }
 }
 
-// One CTA of THREADS per position: thread t takes the 16-byte vectors t, t + THREADS, ...
-// of the row, ACC_AHEAD of them loaded before any is used (several loads in flight per
-// thread: with one, the latency of each load paced the thread).  256 threads and at
-// most 32 registers keep eight CTAs, so that ~1200 rows, resident on the 152 SMs at once.
+// One CTA of THREADS per uncommitted position: thread t takes the 16-byte vectors t, t +
+// THREADS, ... of the row, ACC_AHEAD of them loaded before any is used (several loads in
+// flight per thread: with one, the latency of each load paced the thread).  256 threads
+// and at most 32 registers keep eight CTAs, so that ~1200 rows, resident on the 152 SMs at
+// once.  CTA a takes the a-th uncommitted position (row by row), so that the CTAs with
+// work are the first of the grid and spread evenly over the SMs; the committed positions'
+// CTAs, which read nothing, come last (with one CTA per position in place, the live rows
+// landed unevenly: 3 on some SMs, 10 on others).
 constexpr int ACC_THREADS = 256;
 constexpr int ACC_AHEAD = 4;
+constexpr int ACC_COMPACT_MAX_B = 256;  // (each CTA scans the rows; larger batches keep one CTA per position in place)
+// The a-th uncommitted position of the block (row-major over B rows of P positions, c_b
+// committed in row b): its index b * P + i, or -1 if there are fewer (warp-wide call).
+__device__ __forceinline__ int nth_uncommitted(const int32_t* committed, int B, int P, int a) {
+  const int lane = threadIdx.x & 31;
+  for (int b0 = 0; b0 < B; b0 += 32) {
+    const int b = b0 + lane;
+    const int n = b < B ? P - min(max(committed[b], 0), P) : 0;  // uncommitted positions of row b
+    int incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += t;
+    }
+    const int total = __shfl_sync(kFull, incl, 31);
+    if (a < total) {
+      const unsigned hit = __ballot_sync(kFull, a < incl);
+      const int l = __ffs(hit) - 1;  // the first row whose running count passes a
+      const int before = __shfl_sync(kFull, incl - n, l);
+      const int nl = __shfl_sync(kFull, n, l);
+      return (b0 + l) * P + (P - nl) + (a - before);
+    }
+    a -= total;
+  }
+  return -1;
+}
+
 template <int THREADS, bool ENT>
 __global__ void __launch_bounds__(THREADS, 2048 / THREADS) accept_stats_kernel(
-    const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int P, int V,
+    const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int B, int P, int V,
     int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2, int mode) {
-  const int pos = blockIdx.x;  // b * P + i
-  const int b = pos / P, i = pos % P;
-  if (i < committed[b]) return;  // committed positions are never read
+  int pos = blockIdx.x;  // b * P + i
+  if (B <= ACC_COMPACT_MAX_B) {
+    __shared__ int pos_s;
+    if (threadIdx.x < 32) {
+      const int q = nth_uncommitted(committed, B, P, (int)blockIdx.x);
+      if (threadIdx.x == 0) pos_s = q;
+    }
+    __syncthreads();
+    pos = pos_s;
+    if (pos < 0) return;  // (uniform over the CTA)
+  } else if (pos % P < committed[pos / P]) {
+    return;  // committed positions are never read
+  }
   const __nv_bfloat16* row = logits + (size_t)pos * V;
   Part a{-INFINITY, 0.f, -INFINITY, 0x7fffffff};
   const bool vec = ((reinterpret_cast<uintptr_t>(row) & 15) == 0);
@@ -492,8 +640,23 @@ __global__ void accept_commit_kernel(const int32_t* __restrict__ committed,
     if (threadIdx.x == 0) k[b] = 0;
     return;
   }
-  const int K = dcv_row(x + (size_t)b * P, ids + (size_t)b * P, c1 + (size_t)b * P, pb, P, prm);
+  int K;
+  if (prm.acceptance == 1) {  // Eq. threshold_pd over the uncommitted rest [c_b, P), no drafts
+    float hs, hm;
+    K = threshold_row(x + (size_t)b * P, nullptr, ids + (size_t)b * P, c1 + (size_t)b * P, nullptr, pb, P, prm, &hs,
+                      &hm);
+  } else {
+    K = dcv_row(x + (size_t)b * P, ids + (size_t)b * P, c1 + (size_t)b * P, pb, P, prm);
+  }
   if (threadIdx.x == 0) k[b] = K;
+}
+
+// ------------------------------------------------------------------ launch floor
+// A kernel that does nothing but the step kernels' dependent-launch handshake: a graph of
+// n of them measures the launch cost a step of n launches cannot go below.
+__global__ void empty_step_kernel() {
+  pdl_wait();
+  pdl_launch_dependents();
 }
 
 // ------------------------------------------------------------------ weight generator
@@ -566,18 +729,20 @@ cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int ro
 
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
                               const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
-                              int N, int M, const DcvParams& prm, int32_t* done_count, cudaStream_t stream) {
+                              int N, int M, const DcvParams& prm, int32_t* done_count, uint8_t* cmt,
+                              cudaStream_t stream) {
+  if (prm.acceptance == 1 && (prm.block_len < 1 || !cmt)) return cudaErrorInvalidValue;
   return launch_pdl(dcv_commit_kernel, batch, 32, 0, stream, x, p, k_out, steps, ids, c, ent, jpde, N, M, prm,
-                    done_count);
+                    done_count, cmt);
 }
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
                                 int V, int32_t* ids, float* c1, float* c2, int mode, cudaStream_t stream) {
   if (mode)
-    accept_stats_kernel<ACC_THREADS, true><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, P, V, ids, c1, c2,
+    accept_stats_kernel<ACC_THREADS, true><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, B, P, V, ids, c1, c2,
                                                                              mode);
   else
-    accept_stats_kernel<ACC_THREADS, false><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, P, V, ids, c1, c2,
+    accept_stats_kernel<ACC_THREADS, false><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, B, P, V, ids, c1, c2,
                                                                               mode);
   return cudaGetLastError();
 }
@@ -588,6 +753,8 @@ cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, c
   accept_commit_kernel<<<B, 32, 0, stream>>>(committed, ids, c1, x, k, P, prm);
   return cudaGetLastError();
 }
+
+cudaError_t empty_launch(cudaStream_t stream) { return launch_pdl(empty_step_kernel, 1, 32, 0, stream); }
 
 cudaError_t generate_launch(__nv_bfloat16* dst, uint64_t seed, int tid, int64_t start, int64_t count,
                             float std, float mean, int64_t cols, int blk, int blk_stride, int blk_off,

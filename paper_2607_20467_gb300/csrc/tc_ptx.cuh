@@ -137,6 +137,10 @@ __host__ __device__ constexpr uint32_t make_idesc(int m, int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
          ((uint32_t)(m >> 4) << 24);
 }
+// The same with fp16 A and B (both operands of one instruction share their type).
+__host__ __device__ constexpr uint32_t make_idesc_f16(int m, int n) {
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
 
 __device__ __forceinline__ float f32(uint32_t v) { return __uint_as_float(v); }
 // 2^x on the special-function unit (ex2.approx.ftz: about 2 ulp; inputs below -126 give 0)

@@ -189,12 +189,13 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 
 def model_weights(shape: ModelShape, seed: int, std: float = 0.02,
                   lm_head_scale: float = 1.0, norm_gain_std: float = 0.0,
-                  layers=None, global_tensors: bool = True) -> dict:
+                  layers=None, global_tensors: bool = True, embed: bool = True) -> dict:
     """Weights of ``shape`` from the counter-based generator, as bf16-exact float32.
 
     Matrices are [out][in] (the nn.Linear layout).  Norm gains are 1 + N(0, norm_gain_std).
     ``layers`` restricts the per-layer tensors generated (all by default);
-    ``global_tensors=False`` leaves out the embedding, final norm and LM head (None).
+    ``global_tensors=False`` leaves out the embedding, final norm and LM head (None);
+    ``embed=False`` leaves out only the embedding table (see embed_rows).
     """
     d, hd, H, G, F, V = (shape.d_model, shape.head_dim, shape.n_heads,
                          shape.n_kv_heads, shape.ffn_dim, shape.vocab)
@@ -220,7 +221,7 @@ def model_weights(shape: ModelShape, seed: int, std: float = 0.02,
              TensorKind.WV: "wv", TensorKind.WO: "wo", TensorKind.MLP_NORM: "mlp_norm",
              TensorKind.W_GATE: "w_gate", TensorKind.W_UP: "w_up", TensorKind.W_DOWN: "w_down"}
     if global_tensors:
-        out = {"embed": gen(TensorKind.EMBED, 0), "final_norm": gen(TensorKind.FINAL_NORM, 0),
+        out = {"embed": gen(TensorKind.EMBED, 0) if embed else None, "final_norm": gen(TensorKind.FINAL_NORM, 0),
                "lm_head": gen(TensorKind.LM_HEAD, 0), "layers": []}
     else:
         out = {"embed": None, "final_norm": None, "lm_head": None, "layers": []}
@@ -250,6 +251,27 @@ def prompt_ids(seed: int, batch: int, n_prompt: int, mask_id: int) -> np.ndarray
     """Uniform random prompt ids in [0, mask_id) (never the mask id), int32 [batch][N]."""
     rng = np.random.Generator(np.random.PCG64(seed))
     return rng.integers(0, mask_id, size=(batch, n_prompt), dtype=np.int64).astype(np.int32)
+
+
+def decode_state(seed: int, prompt: np.ndarray, gen_len: int, p_offset: int, window: int, mask_id: int,
+                 draft_frac: float = 0.4):
+    """A decoding state of Algorithm 1's shape for every row of ``prompt`` (int32 [B][N]):
+    x = prompt ++ committed ids on [N, p) ++ MASK on the window [p, p + window) ++ draft
+    ids on about ``draft_frac`` of the future positions (MASK elsewhere), p = N + p_offset.
+    Ids are uniform in [0, mask_id).  Returns (x int32 [B][N + M], p int32 [B])."""
+    rng = np.random.Generator(np.random.PCG64([seed, p_offset]))
+    prompt = np.atleast_2d(np.asarray(prompt, dtype=np.int32))
+    B, N = prompt.shape
+    T = N + gen_len
+    p = N + p_offset
+    x = np.full((B, T), mask_id, np.int32)
+    x[:, :N] = prompt
+    x[:, N:p] = rng.integers(0, mask_id, size=(B, p - N))
+    lo = min(p + window, T)
+    drafts = rng.random((B, T - lo)) < draft_frac
+    ids = rng.integers(0, mask_id, size=(B, T - lo))
+    x[:, lo:] = np.where(drafts, ids, mask_id)
+    return x, np.full(B, p, np.int32)
 
 
 def _beta_mixture(rng, n):

@@ -1,0 +1,74 @@
+"""Where the full-size block tolerance comes from (no GPU).
+
+The GPU accumulates every matrix product in fp32; the oracle in fp64.  Both round the same
+operands to bf16 (the RMSNorm outputs, q / k after RoPE, v, the attention output and the
+SwiGLU output).  At the LLaDA-8B and Dream-7B shapes, fp32 accumulation over K = 4096 ..
+18944 products moves enough values across bf16 rounding boundaries that even an exact
+IEEE-fp32 evaluation differs visibly from the fp64 oracle.  This test makes that
+evaluation, in PyTorch on the CPU from the same seeded weights and tokens, and checks that
+it lies within the bound the GPU parity tests use for one block (relative rms error per
+row: 3.5e-3 mean, 6e-3 max) but clearly away from zero: the bound is what a correct fp32
+implementation reaches, not slack.
+"""
+import numpy as np
+import pytest
+import torch
+
+import synthetic as syn
+from oracle import model
+
+TOL_BLOCK = (3.5e-3, 6e-3)
+
+
+def _bf(t):
+    return t.to(torch.bfloat16).to(torch.float32)
+
+
+def _block_fp32(shape, lw, h, angles):
+    """One block in IEEE fp32 (torch, CPU) with the oracle's bf16 rounding points."""
+    T = h.shape[0]
+    H, G, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    f = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))  # noqa: E731
+
+    def rms(x, g):
+        return x * torch.rsqrt((x * x).mean(dim=-1, keepdim=True) + shape.rms_eps) * f(g)
+
+    def rope(x):
+        c, s = torch.cos(angles)[:, None, :], torch.sin(angles)[:, None, :]
+        x1, x2 = x[..., :hd // 2], x[..., hd // 2:]
+        return torch.cat([x1 * c - x2 * s, x2 * c + x1 * s], dim=-1)
+
+    xn = _bf(rms(h, lw["attn_norm"]))
+    q = _bf(rope((xn @ f(lw["wq"]).T).reshape(T, H, hd)))
+    k = _bf(rope((xn @ f(lw["wk"]).T).reshape(T, G, hd)))
+    v = _bf((xn @ f(lw["wv"]).T).reshape(T, G, hd))
+    rep = H // G
+    k = k.repeat_interleave(rep, dim=1)
+    v = v.repeat_interleave(rep, dim=1)
+    s = torch.einsum("thd,shd->hts", q, k) / np.float32(np.sqrt(hd))
+    a = torch.einsum("hts,shd->thd", torch.softmax(s, dim=-1), v).reshape(T, H * hd)
+    h = h + _bf(a) @ f(lw["wo"]).T
+    xn = _bf(rms(h, lw["mlp_norm"]))
+    g = xn @ f(lw["w_gate"]).T
+    act = _bf(g * torch.sigmoid(g) * (xn @ f(lw["w_up"]).T))
+    return h + act @ f(lw["w_down"]).T
+
+
+@pytest.mark.parametrize("name,seed,N,M", [("llada8b", 1, 256, 256), ("dream7b", 2, 384, 512)])
+def test_fp32_block_zero_lies_within_the_gpu_bound(name, seed, N, M):
+    sh = syn.SHAPES[name]
+    T = N + M
+    torch.set_num_threads(max(1, torch.get_num_threads()))
+    prompt = syn.prompt_ids(1000, 1, N, sh.mask_id)[0]
+    x = np.concatenate([prompt, np.full(M, sh.mask_id, np.int32)])
+    uniq, inv = np.unique(x, return_inverse=True)
+    h0 = syn.embed_rows(sh, seed, uniq, 0.02)[inv]
+    lw = syn.model_weights(sh, seed, 0.02, 12.0, 0.0, layers=(0,), global_tensors=False)["layers"][0]
+    angles = model.rope_angles(T, sh.head_dim, sh.rope_theta)
+    ref = model.block(sh, lw, h0.astype(np.float64), angles, bf16_operands=True)
+    with torch.no_grad():
+        got = _block_fp32(sh, lw, torch.from_numpy(h0), torch.from_numpy(angles.astype(np.float32))).numpy()
+    err = np.sqrt(((got - ref) ** 2).mean(axis=1)) / np.sqrt((ref ** 2).mean(axis=1))
+    print(f"{name} block 0, IEEE fp32 vs fp64 oracle: relative rms per row mean {err.mean():.2e} max {err.max():.2e}")
+    assert err.mean() <= TOL_BLOCK[0] and err.max() <= TOL_BLOCK[1]
+    assert err.mean() >= 0.1 * TOL_BLOCK[0]  # the rounding-boundary effect is real, not slack

@@ -87,3 +87,42 @@ def test_accept_rejects_bad_arguments(ops):
     bad = dcl.decode_config(gen_len=32, confidence=2)
     st = dcl.lib().dcl_accept(ops.ptr, t.data_ptr(), 1, 32, 100, t.data_ptr(), t.data_ptr(), bad, t.data_ptr())
     assert st == dcl.DCL_ERR_INVALID_ARG
+
+
+def test_accept_raw_inputs_guard_band_report(ops):
+    """The acceptance pass on the seeded config-2 inputs as generated (no position moved out
+    of the guard band): K and x must equal the oracle's on every row whose decisions have
+    no confidence within 1e-4 of a threshold; on the other rows they must be one of the
+    outcomes the band allows.  The counts are printed (the design doc keeps them)."""
+    import paper_2607_20467_gb300 as dcl
+    B, P, V, L, tc, td = 64, 32, 126464, 16, 0.7, 0.98
+    d = syn.accept_inputs(7, B, P, V, V - 1)
+    z = syn.bf16_to_f32(d["logits_bf16"]).astype(np.float64)
+    logits = torch.from_numpy(d["logits_bf16"].view(np.int16)).cuda().view(torch.bfloat16)
+    committed = torch.from_numpy(d["committed"]).cuda()
+    x = torch.from_numpy(d["x"].copy()).cuda()
+    k = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    cfg = dcl.decode_config(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P)
+    ops.accept(logits, committed, x, cfg, k)
+    torch.cuda.synchronize()
+    ocfg = decode.DecodeConfig(tau_commit=tc, tau_draft=td, max_window=L, gen_len=P)
+    K, x_out, _, c1, _ = accept.accept(z, d["committed"], d["x"], ocfg, L)
+    kg, xg = k.cpu().numpy(), x.cpu().numpy()
+    band = 1e-4
+    in_band = rows_in_band = rows_differ = differ_outside = 0
+    for b in range(B):
+        p = int(d["committed"][b])
+        if p >= P:
+            continue
+        c = c1[b]
+        near = (np.abs(c[p:] - tc) < band) | (np.abs(c[p:] - td) < band)
+        in_band += int(near.sum())
+        rows_in_band += int(near.any())
+        same = kg[b] == K[b] and (xg[b] == x_out[b]).all()
+        if not same:
+            rows_differ += 1
+            if not near.any():
+                differ_outside += 1
+    print(f"raw config-2 inputs: {in_band} positions within {band} of a threshold, in {rows_in_band} of {B} rows; "
+          f"{rows_differ} rows decided differently, {differ_outside} of them without a position in the band")
+    assert differ_outside == 0

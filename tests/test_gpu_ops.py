@@ -176,23 +176,30 @@ def test_linear_half_pieces_equal_whole_tiles(ops, M, N, K, mode):
 
 
 # ------------------------------------------------------------------ attention
-@pytest.mark.parametrize("B,T,H,G,hd", [(1, 96, 4, 4, 64), (2, 65, 4, 2, 128), (1, 1, 2, 1, 64),
-                                        (1, 512, 32, 32, 128), (2, 200, 28, 4, 128), (1, 1536, 4, 4, 128)])
-def test_attention_non_causal(ops, B, T, H, G, hd):
-    rng = np.random.default_rng(B * T * H + hd)
+@pytest.mark.parametrize("B,T,H,G,hd,qr", [(1, 96, 4, 4, 64, 0), (2, 65, 4, 2, 128, 0), (1, 1, 2, 1, 64, 0),
+                                           (1, 512, 32, 32, 128, 0), (2, 200, 28, 4, 128, 0), (1, 1536, 4, 4, 128, 0),
+                                           # queries = the last qr positions (the suffix of a cached step),
+                                           # keys = all T positions; a ragged last key block; GQA; hd 64
+                                           (1, 1536, 32, 32, 128, 32), (2, 300, 4, 2, 128, 160),
+                                           (1, 1000, 28, 4, 128, 192), (1, 640, 2, 2, 64, 64)])
+def test_attention_non_causal(ops, B, T, H, G, hd, qr):
+    rng = np.random.default_rng(B * T * H + hd + qr)
     cols = (H + 2 * G) * hd
     qkv = syn.round_bf16(rng.normal(0, 1, (B * T, cols)).astype(np.float32))
     out = torch.full((B * T, H * hd), float("nan"), dtype=torch.bfloat16, device="cuda")
-    ops.op_attention(_bf16(qkv), out, B, T, H, G, hd)
+    ops.op_attention(_bf16(qkv), out, B, T, H, G, hd, qr)
     torch.cuda.synchronize()
     got = _f64(out)
+    q0 = T - qr if qr else 0
     for b in range(B):
         blk = qkv[b * T:(b + 1) * T].astype(np.float64)
-        q = blk[:, :H * hd].reshape(T, H, hd)
+        q = blk[q0:, :H * hd].reshape(T - q0, H, hd)
         k = blk[:, H * hd:(H + G) * hd].reshape(T, G, hd)
         v = blk[:, (H + G) * hd:].reshape(T, G, hd)
         ref = model.attention(q, k, v)
-        g = got[b * T:(b + 1) * T]
+        g = got[b * T + q0:(b + 1) * T]
+        if q0:
+            assert np.isnan(got[b * T:b * T + q0]).all()  # rows outside the query set untouched
         assert np.isfinite(g).all()
         assert np.abs(g - ref).max() <= 1.5e-2 * np.abs(ref).max() + 1e-3
         assert np.abs(g - ref).mean() <= 3e-3 * np.sqrt((ref ** 2).mean())
