@@ -555,7 +555,11 @@ def run_ours(args):
 
     sampler = ClockSampler(_gpu_uuid(torch, local))
     sampler.start()
+    if args.profiler_range:
+        torch.cuda.cudart().cudaProfilerStart()
     ms, tokens = timed(args.steps)
+    if args.profiler_range:
+        torch.cuda.cudart().cudaProfilerStop()
     clocks = sampler.stop()
 
     # per-kernel device times: the same steps with timing events around every kernel
@@ -626,7 +630,8 @@ def run_ours(args):
         e["share"] = e["ms"] / tot if tot else 0.0
     # (the table is the last profiled step: with the cache, that step's own work)
     n_prof = min(args.steps, max(3, S))
-    kern_flops = works[(n_prof - 1) % S][1] if cached else total_flops
+    kern_flops = dict(works[(n_prof - 1) % S][1] if cached else total_flops)
+    kern_flops["gemm_mlp"] = kern_flops["gemm_gateup"] + kern_flops["gemm_down"]  # (the fused MLP launch)
     gemms = {k: v for k, v in table.items() if k.startswith("gemm") and k in kern_flops}
     dom = max(gemms, key=lambda k: gemms[k]["ms"])
     avg_ms = gemms[dom]["ms"] / gemms[dom]["launches"]
@@ -987,6 +992,9 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="llada8b")
     ap.add_argument("--e2e-iters", type=int, default=2)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profiler-range", action="store_true",
+                    help="bracket the timed steps with cudaProfilerStart / Stop (for a profiler started "
+                         "with profiling off, e.g. ncu --profile-from-start off)")
     ap.add_argument("--sweep", action="store_true",
                     help="steps / throughput over the tau_c, tau_d, L (and entropy) grids, one JSON line each")
     args = ap.parse_args()

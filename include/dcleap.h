@@ -332,7 +332,9 @@ typedef enum {
   DCL_K_COMBINE = 8,     /* merge of the LM-head partials */
   DCL_K_DCV = 9,         /* commit / draft / advance */
   DCL_K_VTRANSPOSE = 10, /* v written transposed for the attention kernel */
-  DCL_K_ROWPLAN = 11     /* the rows the step computes (full recompute or cache suffix) */
+  DCL_K_ROWPLAN = 11,    /* the rows the step computes (full recompute or cache suffix) */
+  DCL_K_GEMM_MLP = 12    /* gate/up + SwiGLU and down + residual as one launch (the step's
+                            default; the two launches above when the fusion is off) */
 } dcl_kernel_kind;
 
 /* Fault-handling self-test (the device waits of the GEMM and attention pipelines are

@@ -29,7 +29,7 @@ STATUS_NAMES = ["OK", "INVALID_ARG", "STATE", "OOM", "CUDA", "TIMEOUT", "UNSUPPO
  DCL_W_UP, DCL_W_DOWN, DCL_W_FINAL_NORM, DCL_W_LM_HEAD) = range(12)
 
 KERNEL_KINDS = ["embed", "rmsnorm", "gemm_qkv", "attention", "gemm_o", "gemm_gateup",
-                "gemm_down", "gemm_lmhead", "combine", "dcv", "v_transpose", "row_plan"]
+                "gemm_down", "gemm_lmhead", "combine", "dcv", "v_transpose", "row_plan", "gemm_mlp"]
 
 
 class ModelConfig(ctypes.Structure):

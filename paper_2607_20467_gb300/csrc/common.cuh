@@ -122,6 +122,14 @@ struct GemmPlan {
   size_t ws_needed = 0;    // floats of workspace for split-K partials
   int* flags = nullptr;    // set through gemm_bind_scratch when flags_needed > 0
   float* ws = nullptr;     // set through gemm_bind_scratch when ws_needed > 0
+  // fused MLP (gemm_plan_mlp): one persistent launch runs the gate/up tiles (this plan, SwiGLU
+  // into ep.out = act) and then the down projection's K-split tiles (act @ Wdown^T added to
+  // the residual stream ep2.out), each down item waiting only for the gate/up tiles that
+  // produce its K range of act
+  int fuse = 0;
+  CUtensorMap ta2, tb2, tc2;  // down: act [M][F] (A), Wdown [d][F] (W), residual [M][d] fp32 (out)
+  int N2 = 0, K2 = 0, splits2 = 1;
+  EpiParams ep2;
 };
 
 // Encode the tensor maps and choose the tile / grid.  A is [M][K] bf16 (row pitch K),
@@ -136,6 +144,12 @@ constexpr int kTileHalves = 1 << 18;     // with kTilePair: left-over tiles as t
 constexpr int kTileDsmem = 1 << 19;      // with kTilePair: left-over tiles split by K over a cluster's pairs
 cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W, int N,
                       int epi, const EpiParams& ep, int num_sms, int tile, const char** why);
+// The fused MLP of one layer: act = SwiGLU(xn @ Wgu^T) (Wgu [2F][d], gate / up rows
+// interleaved per 128; ep_act.out = act [M][F]) and then h += act @ Wdown^T (Wdown [d][F];
+// ep_res.out = h, fp32 [M][d]) in one launch of CTA-pair tiles; F a multiple of 128.
+cudaError_t gemm_plan_mlp(GemmPlan* plan, const void* xn, int M, int d, const void* Wgu, int F,
+                          const EpiParams& ep_act, const void* Wdown, const EpiParams& ep_res, int num_sms,
+                          const char** why);
 // Attach the zero-initialised counters (>= flags_needed ints) and the workspace
 // (>= ws_needed floats, 16-byte aligned) a plan needs; they may be shared by plans that
 // run one after another on one stream.

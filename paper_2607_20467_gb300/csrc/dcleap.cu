@@ -255,10 +255,15 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
     q.end(gemm_launch(P[1], c->derr, c->stream), "gemm_o");
     q.begin(DCL_K_RMSNORM);
     q.end(rmsnorm_launch(c->h, L.mlp_norm, c->xn, R, d, m.rms_eps, c->rp.counts, nullptr, c->stream), "rmsnorm");
-    q.begin(DCL_K_GEMM_GATEUP);
-    q.end(gemm_launch(P[2], c->derr, c->stream), "gemm_gateup");
-    q.begin(DCL_K_GEMM_DOWN);
-    q.end(gemm_launch(P[3], c->derr, c->stream), "gemm_down");
+    if (P[2].fuse) {  // gate/up + SwiGLU and down + residual in one launch
+      q.begin(DCL_K_GEMM_MLP);
+      q.end(gemm_launch(P[2], c->derr, c->stream), "gemm_mlp");
+    } else {
+      q.begin(DCL_K_GEMM_GATEUP);
+      q.end(gemm_launch(P[2], c->derr, c->stream), "gemm_gateup");
+      q.begin(DCL_K_GEMM_DOWN);
+      q.end(gemm_launch(P[3], c->derr, c->stream), "gemm_down");
+    }
     if (snapshots && q.err == cudaSuccess)
       q.err = cudaMemcpyAsync(c->snap + (size_t)(l + 1) * R * d, c->h, sizeof(float) * R * d,
                               cudaMemcpyDeviceToDevice, c->stream);
@@ -396,11 +401,19 @@ dcl_status build_plans(dcl_ctx* c) {
     e2.out = c->act;
     e2.ldo = m.ffn_dim;
     e2.m_dev = c->rp.counts;
-    if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms, t_gu, &why))
-      return fail(c, DCL_ERR_UNSUPPORTED, "gate/up plan: %s", why ? why : "?");
-    if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms, t_down,
-                  &why))
-      return fail(c, DCL_ERR_UNSUPPORTED, "down plan: %s", why ? why : "?");
+    // the MLP as one launch (gate/up tiles, then the down projection's K-split items, each
+    // waiting only for the act columns it reads), unless a tile override or DCL_MLP_FUSED=0
+    // asks for the two GEMMs on their own
+    const char* fenv = getenv("DCL_MLP_FUSED");
+    const bool fuse_mlp = !(fenv && fenv[0] == '0') && t_gu == kTilePair && t_down == kTilePair;
+    if (!fuse_mlp || gemm_plan_mlp(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, m.ffn_dim, e2, L.wdown, e1,
+                                   c->num_sms, &why) != cudaSuccess) {
+      if (gemm_plan(&c->plans[4 * l + 2], c->xn, R, d, L.wgu, 2 * m.ffn_dim, EPI_SWIGLU, e2, c->num_sms, t_gu, &why))
+        return fail(c, DCL_ERR_UNSUPPORTED, "gate/up plan: %s", why ? why : "?");
+      if (gemm_plan(&c->plans[4 * l + 3], c->act, R, m.ffn_dim, L.wdown, d, EPI_RESID_F32, e1, c->num_sms, t_down,
+                    &why))
+        return fail(c, DCL_ERR_UNSUPPORTED, "down plan: %s", why ? why : "?");
+    }
     for (int i = 0; i < 4; ++i)
       if (c->plans[4 * l + i].streamk)
         return fail(c, DCL_ERR_UNSUPPORTED, "stream-K needs a fixed row count; the step's GEMMs cannot use it");

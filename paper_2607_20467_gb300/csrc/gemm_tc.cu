@@ -915,6 +915,8 @@ __device__ __noinline__ bool fixup_to_tmem(const CUtensorMap* tmw, int y0, int s
 enum ItemKind : int { IT_PLAIN = 0, IT_SPLIT = 1, IT_PART = 2, IT_LAST = 3, IT_DS_RECV = 4, IT_DS_SEND = 5 };
 struct Sched {
   int tiles, ku, C, splits;
+  int fuse;     // 1: after the tiles, the second GEMM's tiles2 x splits2 K-split items (fused MLP)
+  int tiles2, ku2, splits2;
   int streamk;  // 0: off; else the number of pairs (<= C) that share the left-over tiles
   int halves;   // 1: the tiles of a partial last round run as two 256 x 128 pieces each
   int ds;       // 1: the tiles of a partial last round are split by K over the two pairs
@@ -922,6 +924,7 @@ struct Sched {
 };
 struct Item {
   int t, ku0, ku1, kind;
+  int g = 0;                   // fused MLP: 0 the first GEMM (gate/up), 1 the second (down)
   int piece = 0, width = 256;  // columns [piece * width, + width) of tile t
   int sp;     // IT_SPLIT: split index
   int rel;    // IT_PART / IT_LAST: stream-K tile index (0..R-1)
@@ -931,6 +934,30 @@ struct Item {
 __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& it) {
   it.piece = 0;
   it.width = 256;
+  it.g = 0;
+  if (s.fuse) {
+    // round robin over one sequence: the first GEMM's tiles (M-fastest), then the second's
+    // K-split items, split-major (split s of every tile, M-fastest, before split s + 1):
+    // split s reads the act columns that the first GEMM's tiles of column range s wrote,
+    // which come early in the first sequence, so the items rarely wait
+    const long w = (long)c + (long)idx * s.C;
+    if (w < s.tiles) {
+      it.t = (int)w;
+      it.ku0 = 0;
+      it.ku1 = s.ku;
+      it.kind = IT_PLAIN;
+      return true;
+    }
+    const long w2 = w - s.tiles;
+    if (w2 >= (long)s.tiles2 * s.splits2) return false;
+    it.g = 1;
+    it.sp = (int)(w2 / s.tiles2);
+    it.t = (int)(w2 % s.tiles2);
+    it.ku0 = (int)((long)it.sp * s.ku2 / s.splits2);
+    it.ku1 = (int)((long)(it.sp + 1) * s.ku2 / s.splits2);
+    it.kind = IT_SPLIT;
+    return true;
+  }
   if (s.ds) {
     // c = pair index (pairs 2k and 2k + 1 form cluster k): full rounds of whole tiles,
     // then left-over tile `first + k` on cluster k, K lower half on its first pair (which
@@ -1044,13 +1071,25 @@ __device__ __forceinline__ bool next_item(int idx, const Sched& s, int c, Item& 
 // + r holds row r of CTA `rank`'s half of the tile (S slots per tile).  Items that are
 // waited on never wait themselves before they publish, and every CTA is resident (grid <=
 // SMs, one CTA per SM), so every wait ends.
-template <int EPI, bool DS>
+//
+// FUSE (the fused MLP, gemm_plan_mlp): the item sequence continues past the first GEMM's
+// tiles with the second GEMM's K-split items (A = ta2, W = tb2, out = tc2 / ep2, N2 x K2,
+// splits2 splits added to the residual in split order).  flags then holds, from the plan's
+// row-block count num_m_max = ceil(M / 256): [num_m_max * num_n2 * 2] ordered-add counters,
+// [num_m_max * splits2] readiness counters (each first-GEMM tile, when its act stores have
+// completed, adds 1 per CTA to every split its 128 act columns fall in) and [num_m_max *
+// splits2] pass counters (the last CTA to pass a readiness wait zeroes both for the next
+// launch).  Every CTA is resident and a second-GEMM item waits only on first-GEMM tiles
+// earlier in the sequence, which resident pairs have taken, so every wait ends.
+template <int EPI, bool DS, bool FUSE = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
                     const __grid_constant__ CUtensorMap tmbh, const __grid_constant__ CUtensorMap tmc,
                     const __grid_constant__ CUtensorMap tmw, const __grid_constant__ CUtensorMap tmv,
                     const __grid_constant__ CUtensorMap tmk, int M, int N, int K, EpiParams ep, int splits,
-                    int streamk, int halves, int ws_slots, int* flags, float* ws, int* err) {
+                    int streamk, int halves, int ws_slots, int* flags, float* ws, int* err,
+                    const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb2,
+                    const __grid_constant__ CUtensorMap tc2, int N2, int K2, int splits2, EpiParams ep2) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -1097,6 +1136,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     prefetch_tmap(&tma);
     prefetch_tmap(&tmb);
     prefetch_tmap(&tmbh);
+    if (FUSE) {
+      prefetch_tmap(&ta2);
+      prefetch_tmap(&tb2);
+    }
   }
   if (warp == 1) tmem_alloc_pair(holder, TMEM2_COLS);
   tc_fence_before();
@@ -1106,6 +1149,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem_base = *holder_ptr;
   pdl_wait();  // the previous kernel of the step has completed
   pdl_launch_dependents();
+  static_assert(!FUSE || KA2 == 1, "the fused MLP counts its second GEMM's K in 64-column blocks");
+  const int num_m_max = (M + 255) / 256;  // (the plan's rows: the layout of the fused counters)
   if (ep.m_dev) M = min(M, *ep.m_dev);  // the step's row count (written by an earlier kernel)
   const int num_m = (M + 255) / 256;
   const int num_n = (N + 255) / 256;
@@ -1117,6 +1162,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   sc.streamk = streamk;
   sc.halves = halves;
   sc.ds = DS ? 1 : 0;
+  sc.fuse = FUSE ? 1 : 0;
+  const int num_n2 = FUSE ? (N2 + 255) / 256 : 0;
+  sc.tiles2 = num_m * num_n2;
+  sc.ku2 = FUSE ? K2 / BK : 0;
+  sc.splits2 = FUSE ? splits2 : 1;
+  // fused-MLP counters (see above)
+  int* const f_ord = flags;
+  int* const f_dep = FUSE ? flags + (size_t)num_m_max * num_n2 * 2 : nullptr;
+  int* const f_pass = FUSE ? f_dep + (size_t)num_m_max * splits2 : nullptr;
   // item tile -> (m block, n block), M-fastest
   auto tile_mn = [&](int t, int& m_blk, int& n_blk) {
     m_blk = t % num_m;
@@ -1142,6 +1196,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                          (!hw ? (int)rank * 128
                               : (EPI == EPI_SWIGLU ? (int)rank * 128 + it.piece * 64 : it.piece * 128 + (int)rank * 64));
         const CUtensorMap* tw_map = hw ? &tmbh : &tmb;
+        const CUtensorMap* ta_map = &tma;
+        if (FUSE && it.g == 1) {
+          // the second GEMM reads act columns [ku0 * 64, ku1 * 64) of rows m_blk: wait until
+          // the first GEMM's tiles writing them (act columns 128 n .. 128 n + 127 from tile n,
+          // both CTAs of its pair) have stored them
+          ta_map = &ta2;
+          tw_map = &tb2;
+          const int need = 2 * ((it.ku1 + 1) / 2 - it.ku0 / 2);
+          int* dep = f_dep + m_blk * splits2 + it.sp;
+          if (!wait_flag_geq(dep, need, abort_flag)) {
+            ok = false;
+            break;
+          }
+          fence_proxy_async_global();  // the act stores (acquired) before this CTA's TMA loads
+          // the last of the pair CTAs that wait on this counter resets it for the next launch
+          if (atomicAdd(f_pass + m_blk * splits2 + it.sp, 1) == 2 * num_n2 - 1) {
+            atomicExch(dep, 0);
+            atomicExch(f_pass + m_blk * splits2 + it.sp, 0);
+          }
+        }
         const uint32_t stage_tx = 2u * (uint32_t)(hw ? A2_STAGE_BYTES + B2_STAGE_BYTES / 2 : STAGE2_BYTES);
         for (int kb = kb0; kb < kb1; kb += KA2) {
           if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) {
@@ -1151,7 +1225,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t full_leader = mapa_shared(full0 + 8 * stage, lead);
           if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, stage_tx);
           for (int a = 0; a < KA2; ++a) {
-            tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, &tma, (kb + a) * BK,
+            tma_load_2d_pair(sA + stage * A2_STAGE_BYTES + a * A_STAGE_BYTES, ta_map, (kb + a) * BK,
                              m_blk * 256 + (int)rank * 128, full_leader);
             tma_load_2d_pair(sB + stage * B2_STAGE_BYTES + a * B2_BLOCK_BYTES, tw_map, (kb + a) * BK, wrow,
                              full_leader);
@@ -1249,6 +1323,36 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       s.row = row_local;
       if (it.kind == IT_PLAIN) {
         epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep, it.piece, it.width);
+        if (FUSE) {
+          // publish the tile's act columns to the second GEMM's items that read them: once
+          // this CTA's stores have completed, one arrival per split range they fall in
+          o.drain();
+          epilogue_bar();
+          if (et == 0) {
+            __threadfence();
+            const int kb_lo = 2 * n_blk, kb_hi = 2 * n_blk + 1;  // its act columns in 64-column K blocks
+            const int s_lo = ((kb_lo + 1) * splits2 - 1) / sc.ku2, s_hi = ((kb_hi + 1) * splits2 - 1) / sc.ku2;
+            atomicAdd(f_dep + m_blk * splits2 + s_lo, 1);
+            if (s_hi != s_lo) atomicAdd(f_dep + m_blk * splits2 + s_hi, 1);
+          }
+        }
+      } else if (FUSE && it.g == 1) {
+        // the second GEMM's split it.sp of tile (m_blk, n_blk), added to the residual stream
+        // after split it.sp - 1 (a per-tile counter, reset by the last split)
+        const int sp = it.sp;
+        int* flag = f_ord + (m_blk + num_m * n_blk) * 2 + rank;
+        if (et == 0 && !wait_flag_geq(flag, sp, abort_flag)) {
+          *abort_flag = 1;
+          report_error(err, DERR_WAIT_TIMEOUT);
+        }
+        epilogue_bar();
+        if (!*abort_flag) epilogue_pair<EPI_RESID_F32>(s, o, &tc2, &tmv, &tmk, row, n_blk, M, N2, ep2);
+        o.drain();
+        epilogue_bar();
+        if (et == 0) {
+          __threadfence();
+          atomicExch(flag, sp + 1 == splits2 ? 0 : sp + 1);
+        }
       } else if (it.kind == IT_DS_RECV) {
         // this pair's MMAs are done (tfull): the operand ring is free for the other K
         // half's sum, which the other pair of the cluster writes into it; then the
@@ -1448,10 +1552,10 @@ cudaError_t launch_t(const GemmPlan& p, int* err, cudaStream_t stream) {
   return launch_pdl(kern, p.grid, NUM_THREADS, Cfg<BN>::SMEM, stream, p.ta, p.tb, p.M, p.N, p.K, p.ep, err);
 }
 
-template <int EPI, bool DS = false>
+template <int EPI, bool DS = false, bool FUSE = false>
 cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   static bool attr_set = false;
-  auto kern = gemm_tc2_kernel<EPI, DS>;
+  auto kern = gemm_tc2_kernel<EPI, DS, FUSE>;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM2);
     if (e != cudaSuccess) return e;
@@ -1472,7 +1576,8 @@ cudaError_t launch_t2(const GemmPlan& p, int* err, cudaStream_t stream) {
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, p.ta, p.tb, p.tbh, p.tc, p.tw, p.tv, p.tk, p.M, p.N, p.K, p.ep, p.splits,
-                            p.streamk, p.halves, p.ws_slots, p.flags, p.ws, err);
+                            p.streamk, p.halves, p.ws_slots, p.flags, p.ws, err, p.ta2, p.tb2, p.tc2, p.N2, p.K2,
+                            p.splits2, p.ep2);
 }
 
 // Clusters of four CTA-pair CTAs that can be resident at once (0 if unknown).
@@ -1612,6 +1717,12 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   plan->M = M;
   plan->N = N;
   plan->K = K;
+  plan->fuse = 0;
+  plan->N2 = plan->K2 = 0;
+  plan->splits2 = 1;
+  memset(&plan->ta2, 0, sizeof(plan->ta2));
+  memset(&plan->tb2, 0, sizeof(plan->tb2));
+  memset(&plan->tc2, 0, sizeof(plan->tc2));
   plan->bn = bn;
   plan->cg = cg;
   plan->epi = epi;
@@ -1745,6 +1856,49 @@ cudaError_t gemm_plan(GemmPlan* plan, const void* A, int M, int K, const void* W
   return cudaSuccess;
 }
 
+cudaError_t gemm_plan_mlp(GemmPlan* plan, const void* xn, int M, int d, const void* Wgu, int F,
+                          const EpiParams& ep_act, const void* Wdown, const EpiParams& ep_res, int num_sms,
+                          const char** why) {
+  *why = nullptr;
+  if (F % 128 != 0 || d % 256 != 0 || M <= 0) {
+    *why = "fused MLP: needs F a multiple of 128 and d a multiple of 256";
+    return cudaErrorInvalidValue;
+  }
+  // the gate/up part: CTA-pair tiles, unsplit, in plain rounds
+  cudaError_t e = gemm_plan(plan, xn, M, d, Wgu, 2 * F, EPI_SWIGLU, ep_act, num_sms, kTilePair | (1 << 8), why);
+  if (e != cudaSuccess) return e;
+  if (plan->cg != 2 || plan->ds || plan->splits != 1 || plan->streamk || plan->halves) {
+    *why = "fused MLP: the gate/up plan is not a plain CTA-pair plan";
+    return cudaErrorInvalidValue;
+  }
+  if ((reinterpret_cast<uintptr_t>(ep_res.out) & 15) || (reinterpret_cast<uintptr_t>(Wdown) & 15) ||
+      ep_res.ldo < d || (ep_res.ldo * 4) % 16) {
+    *why = "fused MLP: the residual stream and the down weights must be 16-byte aligned";
+    return cudaErrorInvalidValue;
+  }
+  if (!encode_kmajor(&plan->ta2, ep_act.out, M, F, BM) || !encode_kmajor(&plan->tb2, Wdown, d, F, 128) ||
+      !encode_rows(&plan->tc2, ep_res.out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, M, d, ep_res.ldo)) {
+    *why = "fused MLP: cuTensorMapEncodeTiled failed";
+    return cudaErrorInvalidValue;
+  }
+  plan->fuse = 1;
+  plan->N2 = d;
+  plan->K2 = F;
+  plan->ep2 = ep_res;
+  // the down projection split along K into items as long as a gate/up tile (its K)
+  const int ku1 = d / BK, ku2 = F / BK;
+  int s2 = (ku2 + ku1 / 2) / ku1;
+  s2 = s2 < 1 ? 1 : (s2 > ku2 ? ku2 : s2);
+  plan->splits2 = s2;
+  const long num_m = (M + 255) / 256, num_n2 = d / 256;
+  plan->flags_needed = (size_t)(num_m * num_n2 * 2 + 2 * num_m * s2);
+  plan->ws_needed = 0;
+  const int pairs = num_sms / 2;
+  const long items = num_m * (2L * F / 256) + num_m * num_n2 * s2;
+  plan->grid = 2 * (int)(items < pairs ? items : pairs);
+  return cudaSuccess;
+}
+
 bool gemm_fuse_kv(GemmPlan* p, void* kbuf, void* vt, int batch, int T, int H, int G, int hd, int Tp) {
   if (p->cg != 2 || p->epi != EPI_QKV_ROPE || T % 32 != 0 || p->ep.rope_cols % 256 != 0 || (H * hd) % 256 != 0 ||
       (reinterpret_cast<uintptr_t>(vt) & 15) || (reinterpret_cast<uintptr_t>(kbuf) & 15) || Tp % 8 != 0)
@@ -1812,6 +1966,8 @@ cudaError_t wait_selftest_launch(int which, const int* flag, int* err, cudaStrea
 
 cudaError_t gemm_launch(const GemmPlan& p, int* err, cudaStream_t stream) {
   if ((p.flags_needed && !p.flags) || (p.ws_needed && !p.ws)) return cudaErrorInvalidValue;
+  if (p.fuse) return p.cg == 2 && p.epi == EPI_SWIGLU ? launch_t2<EPI_SWIGLU, false, true>(p, err, stream)
+                                                      : cudaErrorInvalidValue;
   if (p.cg == 2 && p.ds) {
     switch (p.epi) {
       case EPI_BF16: return launch_t2<EPI_BF16, true>(p, err, stream);
