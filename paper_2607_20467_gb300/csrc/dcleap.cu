@@ -1051,6 +1051,11 @@ dcl_status dcl_accept(dcl_ctx* c, const void* logits_dev, int32_t B, int32_t P, 
     return fail(c, DCL_ERR_INVALID_ARG, "bad decode config");
   const size_t n = (size_t)B * P;
   if (c->acc_cap < n) {
+    CUDA_TRY(c, cudaStreamSynchronize(c->stream));  // no launch may still use the old buffers
+    dev_free_one(c, c->acc_ids);
+    dev_free_one(c, c->acc_c1);
+    dev_free_one(c, c->acc_c2);
+    c->acc_cap = 0;
     c->acc_ids = (int32_t*)dev_alloc(c, 4 * n);
     c->acc_c1 = (float*)dev_alloc(c, 4 * n);
     c->acc_c2 = (float*)dev_alloc(c, 4 * n);

@@ -161,13 +161,17 @@ __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)in_row * d);
   const int n4 = d / 4;
   float4 v[VPT];
+  uint2 gv[VPT];  // (the gain, loaded with the row: a load next to each store waited for it)
+  const uint2* g2 = reinterpret_cast<const uint2*>(gain);
   float ss = 0.f;
 #pragma unroll
   for (int i = 0; i < VPT; ++i) {
     const int j = t + 128 * i;
     v[i] = (live && j < n4) ? xr[j] : make_float4(0.f, 0.f, 0.f, 0.f);
-    ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+    gv[i] = (live && j < n4) ? __ldg(g2 + j) : make_uint2(0u, 0u);
   }
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(kFull, ss, o);
   __shared__ float red[ROWS][4];
@@ -176,13 +180,12 @@ __global__ void __launch_bounds__(128 * ROWS) rmsnorm_reg_kernel(
   const float tot = red[sub][0] + red[sub][1] + red[sub][2] + red[sub][3];
   const float inv = rsqrtf(tot / (float)d + eps);
   if (!live) return;
-  const uint2* g2 = reinterpret_cast<const uint2*>(gain);
   uint2* y2 = reinterpret_cast<uint2*>(y + (size_t)r * d);
 #pragma unroll
   for (int i = 0; i < VPT; ++i) {
     const int j = t + 128 * i;
     if (j < n4) {
-      const uint2 g = __ldg(g2 + j);
+      const uint2 g = gv[i];
       y2[j] = make_uint2(pack_bf16x2(v[i].x * inv * bf16_lo(g.x), v[i].y * inv * bf16_hi(g.x)),
                          pack_bf16x2(v[i].z * inv * bf16_lo(g.y), v[i].w * inv * bf16_hi(g.y)));
     }
@@ -497,11 +500,37 @@ __device__ __forceinline__ void take1(Part& a, float v, int col) {
 // on the special-function unit.  The argmax's own term is exp2 of the rounding residual
 // of the fused multiply-add, within an ulp of 1 (write_conf clamps p1 and p2).  A vector
 // holding an infinity takes the exact column-by-column path.
+// Packed pairs of fp32 (sm_100+ f32x2 arithmetic: one instruction for two lanes, each
+// rounded as its scalar form) and the three-input maximum.
+__device__ __forceinline__ unsigned long long pk2(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk2(unsigned long long r, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b, unsigned long long c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 template <bool ENT>
 __device__ __forceinline__ void take8(Part& a, const uint4& q, int col) {
   const float v[8] = {bf16_lo(q.x), bf16_hi(q.x), bf16_lo(q.y), bf16_hi(q.y),
                       bf16_lo(q.z), bf16_hi(q.z), bf16_lo(q.w), bf16_hi(q.w)};
-  const float cm = fmaxf(fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3])), fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7])));
+  const float cm = fmaxf(max3f(max3f(v[0], v[1], v[2]), max3f(v[3], v[4], v[5]), v[6]), v[7]);
   if (!(fabsf(cm) < INFINITY)) {
 #pragma unroll
     for (int k = 0; k < 8; ++k) take1<ENT>(a, v[k], col + k);
@@ -524,14 +553,22 @@ __device__ __forceinline__ void take8(Part& a, const uint4& q, int col) {
   } else {
     a.t2 = fmaxf(a.t2, cm);
   }
+  // y = z log2(e) - m log2(e) and its exp2 for the eight columns, two lanes per
+  // instruction; the eight terms are summed as a tree of pairs
   const float ml = a.m * kLog2e;
+  const unsigned long long l2 = pk2(kLog2e, kLog2e), nm = pk2(-ml, -ml);
+  unsigned long long e2[4];
 #pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const float y = fmaf(v[k], kLog2e, -ml);
-    const float e = ex2_approx(y);
-    a.s += e;
-    if (ENT) a.u = fmaf(e, fmaxf(y, -200.f), a.u);
+  for (int k = 0; k < 4; ++k) {
+    float y0, y1;
+    upk2(ffma2(pk2(v[2 * k], v[2 * k + 1]), l2, nm), y0, y1);
+    const float x0 = ex2_approx(y0), x1 = ex2_approx(y1);
+    e2[k] = pk2(x0, x1);
+    if (ENT) a.u = fmaf(x1, fmaxf(y1, -200.f), fmaf(x0, fmaxf(y0, -200.f), a.u));
   }
+  float s0, s1;
+  upk2(fadd2(fadd2(e2[0], e2[1]), fadd2(e2[2], e2[3])), s0, s1);
+  a.s += s0 + s1;
 }
 
 // One CTA of THREADS per uncommitted position: thread t takes the 16-byte vectors t, t +

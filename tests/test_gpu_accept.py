@@ -50,10 +50,13 @@ def _guarded(seed, B, P, V, taus, confidence=0):
 @pytest.mark.parametrize("B,P,V,L,contig,conf", [(8, 32, 4096, 16, 0, 0), (16, 32, 1000, 32, 0, 0),
                                                  (6, 40, 3001, 7, 1, 0), (64, 32, 126464, 16, 0, 0),
                                                  (64, 32, 126464, 32, 1, 0), (16, 32, 4096, 16, 0, 1),
-                                                 (32, 32, 126464, 16, 0, 1), (3, 4096, 1000, 2048, 0, 0)])
+                                                 (32, 32, 126464, 16, 0, 1), (3, 4096, 1000, 2048, 0, 0),
+                                                 (300, 8, 1000, 8, 0, 0), (4, 16, 9, 8, 0, 0), (5, 8, 2, 4, 1, 0)])
 def test_accept_bit_exact(ops, B, P, V, L, contig, conf):
     """conf = 1: the thresholds see exp(-H) (marginal entropy); the guard band then keeps
-    exp(-H) 1e-4 away from them (H is summed in fp32 on the GPU, fp64 in the oracle)."""
+    exp(-H) 1e-4 away from them (H is summed in fp32 on the GPU, fp64 in the oracle).
+    B = 300 takes the positions in place (beyond the compaction's batch limit); V = 9 and
+    V = 2 leave rows that are not 16-byte aligned or shorter than one vector."""
     import paper_2607_20467_gb300 as dcl
     tc, td = (0.7, 0.9) if not conf else (0.5, 0.8)
     d, z = _guarded(B * 131 + P + L, B, P, V, (tc, td), conf)
@@ -126,3 +129,28 @@ def test_accept_raw_inputs_guard_band_report(ops):
     print(f"raw config-2 inputs: {in_band} positions within {band} of a threshold, in {rows_in_band} of {B} rows; "
           f"{rows_differ} rows decided differently, {differ_outside} of them without a position in the band")
     assert differ_outside == 0
+
+
+def test_accept_calls_of_changing_size(ops):
+    """One context, calls that shrink and grow (without outgrowing the first scratch):
+    each result equals the oracle's."""
+    import paper_2607_20467_gb300 as dcl
+    ctx = dcl.Context(None, 1, 1)
+    try:
+        for B, P, V, conf in ((64, 32, 4096, 0), (16, 32, 4096, 1), (8, 32, 1000, 0), (3, 40, 3001, 1),
+                              (64, 32, 4096, 1)):
+            tc, td = (0.7, 0.9) if not conf else (0.5, 0.8)
+            d, z = _guarded(B * 17 + P + V, B, P, V, (tc, td), conf)
+            logits = torch.from_numpy(d["logits_bf16"].view(np.int16)).cuda().view(torch.bfloat16)
+            committed = torch.from_numpy(d["committed"]).cuda()
+            x = torch.from_numpy(d["x"].copy()).cuda()
+            k = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+            cfg = dcl.decode_config(tau_commit=tc, tau_draft=td, max_window=16, gen_len=P, confidence=conf)
+            ctx.accept(logits, committed, x, cfg, k)
+            torch.cuda.synchronize()
+            ocfg = decode.DecodeConfig(tau_commit=tc, tau_draft=td, max_window=16, gen_len=P, confidence=conf)
+            K, x_out, _, _, _ = accept.accept(z, d["committed"], d["x"], ocfg, 16)
+            assert (k.cpu().numpy() == K).all(), (B, P, V, conf)
+            assert (x.cpu().numpy() == x_out).all(), (B, P, V, conf)
+    finally:
+        ctx.close()

@@ -135,11 +135,16 @@ def test_teacher_forced_blocks_head_and_decisions(dcl, name):
                 h.append(syn.embed_rows(sh, seed, uniq, STD)[inv].astype(np.float64))
         angles = model.rope_angles(T, sh.head_dim, sh.rope_theta)
         worst = [0.0, 0.0]
+        # block 1 from the GPU's own block-0 output (its attn_norm is the RMSNorm that the
+        # previous block's MLP launch runs at its end), and the input of the last block
+        second, last_in = {}, {}
         for layer in range(sh.n_layers):
             lw = (w_all if w_all is not None else
                   syn.model_weights(sh, seed, STD, lm_scale, gstd, layers=(layer,), global_tensors=False))["layers"][layer]
             for s in range(len(states)):
                 h_in = h[s].astype(np.float32)
+                if layer == sh.n_layers - 1:
+                    last_in[s] = h_in
                 ref = model.block(sh, lw, h_in.astype(np.float64), angles, bf16_operands=True)
                 load_state(s)
                 run_from(layer, h_in)
@@ -150,6 +155,14 @@ def test_teacher_forced_blocks_head_and_decisions(dcl, name):
                 err = _rel_rms(g[:T].astype(np.float64), ref)
                 worst = [max(worst[0], float(err.mean())), max(worst[1], float(err.max()))]
                 assert err.mean() <= TOL_BLOCK[0] and err.max() <= TOL_BLOCK[1], (layer, s, err.mean(), err.max())
+                if layer == 0 and sh.n_layers > 1:
+                    with torch.cuda.stream(stream):
+                        ctx.debug_hidden(1, got)
+                    second[s] = (g[:T].astype(np.float64), got.cpu().numpy()[:T].astype(np.float64))
+                if layer == 1:
+                    ref2 = model.block(sh, lw, second[s][0], angles, bf16_operands=True)
+                    err2 = _rel_rms(second[s][1], ref2)
+                    assert err2.mean() <= TOL_BLOCK[0] and err2.max() <= TOL_BLOCK[1], (s, err2.mean(), err2.max())
                 h[s] = ref
         print(f"{name}: every block teacher-forced, relative rms per row: worst mean {worst[0]:.2e}, "
               f"worst max {worst[1]:.2e}")
@@ -211,6 +224,21 @@ def test_teacher_forced_blocks_head_and_decisions(dcl, name):
             near_total += near
             exact_total += int((~unsure).sum()) + int(K_o is not None)
         print(f"{name}: decisions exact {exact_total}, near ties (margin <= {TOL_PATH}) {near_total}")
+
+        # the final RMSNorm as the last MLP launch runs it, on the GPU's own last block
+        # output: p1 against the oracle's final norm + LM head of that output
+        for s in range(len(states)):
+            load_state(s)
+            run_from(sh.n_layers - 1, last_in[s], top1=top1, p1=q1, p2=q2)
+            with torch.cuda.stream(stream):
+                ctx.debug_hidden(sh.n_layers - 1, got)
+            g = got.cpu().numpy()[:T].astype(np.float64)
+            hn = model.rms_norm(g[N:], gw["final_norm"], sh.rms_eps)
+            ids_o, p1_o, p2_o = model.confidence(model.logits(gw, model.to_bf16(hn)))
+            g1, gi = q1.cpu().numpy()[:M], top1.cpu().numpy()[:M]
+            assert np.abs(g1 - p1_o).max() <= TOL_PATH, float(np.abs(g1 - p1_o).max())
+            clear = p1_o - p2_o > TOL_PATH
+            assert (gi[clear] == ids_o[clear]).all()
         ops.close()
 
         # for the record: the accumulated forward from the tokens (no teacher forcing)

@@ -65,11 +65,13 @@ def test_noalloc_matches_dcl_accept_on_two_calls(dcl, confidence):
     ctx.close()
 
 
-def test_noalloc_at_the_scratch_limit_on_a_side_stream(dcl):
+@pytest.mark.parametrize("P", [32, 128])
+def test_noalloc_at_the_scratch_limit_on_a_side_stream(dcl, P):
     """B*P exactly DCL_NOALLOC_MAX_POSITIONS (the three scratch arrays reach the end of
-    the static array), issued on a non-default stream, twice."""
+    the static array), issued on a non-default stream, twice: with B = 1024 the
+    statistics pass takes its positions in place, with B = 256 compacted."""
     ctx = dcl.Context(None, 1, 1)
-    B, P, V = MAX_POSITIONS // 32, 32, 64
+    B, V = MAX_POSITIONS // P, 64
     d, logits, committed = _inputs(21, B, P, V)
     cfg = dcl.decode_config(tau_commit=0.5, tau_draft=0.9, max_window=8, gen_len=P)
     side = torch.cuda.Stream()
