@@ -108,14 +108,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   const int g = h / (H / G);
   const int nb = (T + 127) / 128;
 
-  pdl_wait();  // the previous kernels of the step (the row plan among them) have completed
-  pdl_launch_dependents();
-  // the query rows of sequence b are rows [off, off + len) of q and of the output; a tile
-  // past them has nothing to do and leaves before any set-up (uniform over the CTA)
-  const int q_off = seq_off ? seq_off[b] : b * T;
-  const int q_len = seq_len ? seq_len[b] : T;
-  if (qt * 128 >= q_len) return;
-
+  // set-up first (it reads nothing that earlier kernels write), so that under programmatic
+  // dependent launch it overlaps the tail of the kernel before
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < AT_STAGES; ++s) {
@@ -144,6 +138,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *holder_ptr;
+
+  pdl_wait();  // the previous kernels of the step (the row plan among them) have completed
+  pdl_launch_dependents();
+  // the query rows of sequence b are rows [off, off + len) of q and of the output; a tile
+  // past them has nothing to do and leaves at once (uniform over the CTA)
+  const int q_off = seq_off ? seq_off[b] : b * T;
+  const int q_len = seq_len ? seq_len[b] : T;
+  if (qt * 128 >= q_len) {
+    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
+    return;
+  }
 
   if (warp == 0) {
     if (lane == 0) {
@@ -307,10 +312,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(s_empty0 + 8 * sb);  // the S buffer is free for S_{j+2}
         if (valid >= 64) {
+          // four independent three-input maximum chains over the 64 columns
+          float a4[4];
 #pragma unroll
-          for (int c = 0; c < 2; ++c)
+          for (int t = 0; t < 4; ++t) {
+            const uint32_t* w = &v[t >> 1][(t & 1) * 16];
+            float acc = f32(w[0]);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) mm = fmaxf(mm, f32(v[c][e]));
+            for (int e = 1; e < 15; e += 2) acc = max3f(acc, f32(w[e]), f32(w[e + 1]));
+            a4[t] = fmaxf(acc, f32(w[15]));
+          }
+          mm = max3f(a4[0], a4[1], fmaxf(a4[2], a4[3]));
         } else {
 #pragma unroll
           for (int c = 0; c < 2; ++c)
@@ -348,21 +360,45 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       if (raise) m = mb;
       const uint32_t box = sP + (uint32_t)pb * 2 * AT_BOX + (uint32_t)hs * AT_BOX;
+      const bool full = valid >= 64;
+      // the block's sum of this half, in two packed partial sums (fixed order)
+      unsigned long long la = 0ull, lb = 0ull;
+      const unsigned long long sc2 = pk2(scale2, scale2), nm2 = pk2(-m, -m);
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         // P in fp16 (round to nearest even: 2^-12 relative, P <= 2^8); l sums the fp32 values
         float pv[32];
+        if (full) {  // the exponent arguments two lanes per instruction, no column mask
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          pv[e] = ex2_approx(fmaf(f32(v[c][e]), scale2, -m));
-          if (32 * c + e >= valid) pv[e] = 0.f;
-          l += pv[e];
+          for (int e = 0; e < 32; e += 2) {
+            float y0, y1;
+            upk2(ffma2(pk2(f32(v[c][e]), f32(v[c][e + 1])), sc2, nm2), y0, y1);
+            pv[e] = ex2_approx(y0);
+            pv[e + 1] = ex2_approx(y1);
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            pv[e] = ex2_approx(fmaf(f32(v[c][e]), scale2, -m));
+            if (32 * c + e >= valid) pv[e] = 0.f;
+          }
+        }
+#pragma unroll
+        for (int e = 0; e < 32; e += 4) {
+          la = fadd2(la, pk2(pv[e], pv[e + 1]));
+          lb = fadd2(lb, pk2(pv[e + 2], pv[e + 3]));
         }
         const int k0 = c * 4;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           st_shared_v4(box + swz(r, k0 + k), pack_f16x2(pv[8 * k], pv[8 * k + 1]), pack_f16x2(pv[8 * k + 2], pv[8 * k + 3]),
                        pack_f16x2(pv[8 * k + 4], pv[8 * k + 5]), pack_f16x2(pv[8 * k + 6], pv[8 * k + 7]));
+      }
+      {
+        float a0, a1, b0, b1;
+        upk2(la, a0, a1);
+        upk2(lb, b0, b1);
+        l += (a0 + b0) + (a1 + b1);
       }
       tc_fence_before();
       fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
@@ -408,7 +444,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       if (lane == 0) {
         bulk_commit();
-        bulk_wait_all();
+        bulk_wait_read<0>();  // the staging boxes were read (the writes complete with the grid)
       }
       __syncwarp();
     }

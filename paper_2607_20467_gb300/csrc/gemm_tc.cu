@@ -1486,7 +1486,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(mapa_shared(tempty0 + 8 * ab, lead));
     }
-    if (lane == 0) bulk_wait_all();  // the staging boxes outlive every store reading them
+    if (lane == 0) bulk_wait_read<0>();  // the staging boxes outlive every store reading them
     __syncwarp();
   }
 
