@@ -1353,34 +1353,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           __threadfence();
           atomicExch(flag, sp + 1 == splits2 ? 0 : sp + 1);
         }
-      } else if (it.kind == IT_DS_RECV) {
-        // this pair's MMAs are done (tfull): the operand ring is free for the other K
-        // half's sum, which the other pair of the cluster writes into it; then the
-        // epilogue adds it to this accumulator (lower half + upper half, a fixed order)
-        // The sum arrives in four 64-column chunks per band; the epilogue waits for each
-        // chunk when it first reads it, so it overlaps the rest of the transfer.
+      } else if (it.kind == IT_DS_RECV || it.kind == IT_DS_SEND) {
+        // The two K halves of a left-over tile meet half way: the lower-K pair finalises
+        // columns [0, 128) of the tile, the upper-K pair columns [128, 256).  Each pair's
+        // MMAs are done (tfull), so its operand ring is free: it writes the other pair's
+        // 128 columns of its own accumulator there and, once the other pair's ring is free,
+        // one bulk copy per (band, 64-column chunk) moves them into the same place of the
+        // other pair's ring; then its epilogue adds the received half to its own (lower +
+        // upper: one addition, the same value either way round) over its 128 columns,
+        // waiting for each received chunk when it first reads it.
+        const int mine = it.kind == IT_DS_SEND ? 1 : 0;  // the 128-column piece finalised here
         const uint32_t partner = crank ^ 2u;
         if (lane == 0) {
-          for (int c = 0; c < 4; ++c) mbar_arrive_expect_tx(ds_data0 + 8 * (4 * q + c), DS_BLOCK_BYTES);
+          for (int c = 0; c < 2; ++c) mbar_arrive_expect_tx(ds_data0 + 8 * (4 * q + 2 * mine + c), DS_BLOCK_BYTES);
           mbar_arrive_cluster(mapa_shared(ds_go, partner));
         }
         __syncwarp();
-        s.dpart = sA;
-        s.dbar = ds_data0 + 8 * (4 * q);
-        s.dready = 0;
-        s.dabort = abort_flag;
-        s.derr = err;
-        if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep);
-        // every chunk has landed before this CTA may leave (one the epilogue skipped too)
-        for (int c = 0; c < 4; ++c) ds_chunk_ready(s, c);
-      } else if (it.kind == IT_DS_SEND) {
-        // the K upper half: each lane writes its accumulator row into this CTA's own ring
-        // (free: this pair's MMAs are done), then, once the receiving pair's ring is free,
-        // one bulk copy per warp moves the band's 32 rows into the same place there
-        const uint32_t partner = crank ^ 2u;
         bool go = false;
 #pragma unroll 1
-        for (int chunk = 0; chunk < 4; ++chunk) {
+        for (int c = 0; c < 2; ++c) {
+          const int chunk = 2 * (1 - mine) + c;  // a chunk of the other pair's piece
           const uint32_t blk = sA + (uint32_t)((4 * q + chunk) * DS_BLOCK_BYTES);
           const uint32_t own = blk + (uint32_t)(lane * DS_ROW_BYTES);
 #pragma unroll 1
@@ -1408,7 +1400,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             bulk_commit();
           }
         }
-        if (lane == 0) bulk_wait_read<0>();  // this CTA's rows were read (the ring is not touched again)
+        // this pair's piece: TMEM columns and received chunks from 128 * mine on
+        s.taddr += (uint32_t)(128 * mine);
+        s.dpart = sA + (uint32_t)(2 * mine * 32 * DS_ROW_BYTES);
+        s.dbar = ds_data0 + 8 * (4 * q + 2 * mine);
+        s.dready = 0;
+        s.dabort = abort_flag;
+        s.derr = err;
+        if (!*abort_flag) epilogue_pair<EPI>(s, o, &tmc, &tmv, &tmk, row, n_blk, M, N, ep, mine, 128);
+        // every chunk has landed before this CTA may leave (one the epilogue skipped too),
+        // and the other pair has read this CTA's rows (the ring is not touched again)
+        for (int c = 0; c < 2; ++c) ds_chunk_ready(s, c);
+        if (lane == 0) bulk_wait_read<0>();
         __syncwarp();
       } else if (it.kind == IT_SPLIT) {
         const int sp = it.sp;
