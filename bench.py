@@ -18,7 +18,9 @@ generations through the public API (prompt from pinned host memory, result read 
 
 Under full recompute the line also carries `ms_per_step_at_p`: one step timed from the
 trajectory's states at p - N = 0, M/4, M/2, 3M/4 (set back each time), so that the step
-cost is read at fixed positions as well as over the trajectory.
+cost is read at fixed positions as well as over the trajectory.  With the key / value
+cache it carries `ms_per_step_by_rows`: the trajectory's steps (each between CUDA events)
+grouped by the rows they compute, median time and roofline fraction per row count.
 
 --workload accept times the acceptance pass alone (dcl_accept on seeded bf16 logits
 [64][32][126464], window 16) against the HBM roofline of the uncommitted logit rows it
@@ -149,6 +151,28 @@ def cached_rows(kper, N, M, block):
             lm += T - max(start, N)
             p[b] += int(k[b])
         out.append((rows, lm))
+    return out
+
+
+def steps_by_rows(rl, works, traj_ms, peaks):
+    """Cached trajectories: the step time by the number of rows the step computes (all T
+    positions at a refresh, the block-aligned suffix otherwise), median over the
+    trajectory's steps with that row count, against the roofline of that step's own work
+    (measured sustained bf16 peak, measured HBM copy rate)."""
+    groups = {}
+    for (rows, _), w, ms in zip(rl, works, traj_ms):
+        g = groups.setdefault(rows, {"ms": [], "work": w})
+        g["ms"].append(ms)
+    out = []
+    for rows in sorted(groups, reverse=True):
+        g = groups[rows]
+        flops = sum(g["work"][1].values())
+        t_tensor = flops / (peaks["bf16_tflops_sustained"] * 1e12)
+        t_hbm = g["work"][2] / (peaks["hbm_gbs"] * 1e9)
+        ms = statistics.median(g["ms"])
+        out.append({"rows": int(rows), "steps": len(g["ms"]), "ms": ms, "t_roof_ms": 1e3 * max(t_tensor, t_hbm),
+                    "bound": "hbm" if t_hbm >= t_tensor else "tensor",
+                    "frac": 1e3 * max(t_tensor, t_hbm) / ms if ms > 0 else None})
     return out
 
 
@@ -513,14 +537,20 @@ def run_ours(args):
     # first state at or past each mark) are kept for the fixed-state step timings.
     marks = [] if cached else [0, M // 4, M // 2, 3 * M // 4]
     snaps = []
-    ks, kper = [], []
+    ks, kper, traj_ms = [], [], []
     p_host = np.full(B, N, np.int64)
     while sum(ks) < B * M and len(ks) < 4 * M:
         if marks and int(p_host.min()) - N >= marks[0]:
             snaps.append(ctx.get_state())
             while marks and int(p_host.min()) - N >= marks[0]:
                 marks.pop(0)
-        kr = ctx.step(return_k=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ctx.step()
+        e1.record(stream)
+        _, p_new = ctx.get_state()  # (synchronises) K = the advance of p (contiguous commits)
+        kr = (p_new.astype(np.int64) - p_host).astype(np.int32)
+        traj_ms.append(e0.elapsed_time(e1))
         kper.append(kr.copy())
         ks.append(int(kr.sum()))
         p_host += kr
@@ -615,7 +645,9 @@ def run_ours(args):
         per_layer = works[0][0]
         total_flops = {k: statistics.mean(w[1][k] for w in timed_works) for k in works[0][1]}
         step_bytes = statistics.mean(w[2] for w in timed_works)
+        by_rows = steps_by_rows(rl, works, traj_ms, peaks)
     else:
+        by_rows = None
         per_layer, total_flops, step_bytes = step_work(shape, B, N, M)
 
     # per-kernel table and the dominant kernel's roofline
@@ -690,6 +722,7 @@ def run_ours(args):
                      "avg_launch_ms": avg_ms, "flops_per_launch": flops_launch},
         "kernels": table,
         "ms_per_step_at_p": at_p or None,
+        "ms_per_step_by_rows": by_rows,
         "ms_per_step_profiled": ms_prof / min(args.steps, max(3, S)),
         "gpu_launches": args.steps * len(kern_ms),
         "launch_floor": {"ms_per_graph": floor_ms, "launches_per_step": len(kern_ms),

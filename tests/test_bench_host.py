@@ -108,3 +108,28 @@ def test_step_work_of_a_cached_suffix_step():
     assert total["gemm_lmhead"] == 2.0 * 32 * 4096 * 126464
     assert b_cached - b_plain == pytest.approx(0.524e6 * 1536, rel=1e-3)
     assert b_cached - b_plain == pytest.approx(805e6, rel=1e-3)
+
+
+def test_steps_by_rows_groups_and_grades_each_row_count():
+    """Cached trajectories are graded per computed-row count: a refresh (all rows) and the
+    suffix steps are separate groups, each with the median of its steps and the roofline
+    of its own work (the larger of its tensor and HBM times)."""
+    shape = syn.SHAPES["llada8b"]
+    N, M = 512, 1024
+    rl = [(1536, 1024), (1024, 1024), (1024, 1024), (1536, 1024), (1024, 1024)]
+    works = [bench.step_work(shape, 1, N, M, r, l, True) for r, l in rl]
+    ms = [20.0, 12.0, 13.0, 19.0, 14.0]
+    peaks = {"bf16_tflops_sustained": 1699.7, "hbm_gbs": 6793.8}
+    out = bench.steps_by_rows(rl, works, ms, peaks)
+    assert [g["rows"] for g in out] == [1536, 1024]
+    assert [g["steps"] for g in out] == [2, 3]
+    assert out[0]["ms"] == pytest.approx(19.5) and out[1]["ms"] == pytest.approx(13.0)
+    for g, w in zip(out, (works[0], works[1])):
+        t_t = sum(w[1].values()) / 1699.7e12
+        t_h = w[2] / 6793.8e9
+        assert g["t_roof_ms"] == pytest.approx(1e3 * max(t_t, t_h))
+        assert g["bound"] == ("hbm" if t_h >= t_t else "tensor")
+        assert g["frac"] == pytest.approx(g["t_roof_ms"] / g["ms"])
+    # 32 suffix rows at batch 1 stream 15 GB of weights for far fewer flops: HBM-bound
+    small = bench.steps_by_rows([(32, 32)], [bench.step_work(shape, 1, N, M, 32, 32, True)], [6.0], peaks)
+    assert small[0]["bound"] == "hbm"
