@@ -49,7 +49,14 @@ Readings where the paper is silent or inconsistent (each one is also a test):
     positions at the first step and whenever the block-aligned prefix end
     N + Bk * floor((p - N) / Bk) changes, else only the positions from that prefix end on,
     attending to the keys and values the prefix had at its last refresh
-    (``model.forward_rows``).
+    (``model.forward_rows``);
+  * the dual cache (``kv_cache = 2``; a serving refinement, not in the paper): refreshes
+    as above, and between refreshes only the positions of the current block
+    [b0, min(b0 + Bk, T)) are computed, b0 that prefix end, their queries attending to the
+    stored keys and values of every position (the block's fresh, the rest from the last
+    refresh); the generation positions outside the block keep the predictions of the step
+    that last computed them, K is capped at the block end (commits use fresh predictions
+    only) and the drafts past p + L read the kept predictions.
 """
 from __future__ import annotations
 
@@ -67,7 +74,7 @@ class DecodeConfig:
     gen_len: int = 0              # M
     min_commit: int = 1
     contiguous_drafts: bool = False  # App. E variant: drafts only as an unbroken chain
-    kv_cache: int = 0
+    kv_cache: int = 0             # 0: none; 1: prefix cache; 2: dual (prefix + suffix) cache
     confidence: int = 0           # 0: top-1 probability (Eq. threshold_pd); 1: exp(-entropy)
     acceptance: int = 0           # 0: DCV (Eq. compute_k); 1: Eq. threshold_pd in the block
 
@@ -92,12 +99,15 @@ def remask(x: np.ndarray, p: int, window: int, mask_id: int) -> None:
 
 
 def commit_and_draft(x: np.ndarray, p: int, ids: np.ndarray, c: np.ndarray,
-                     cfg: DecodeConfig, window: int) -> int:
-    """Steps (iii)-(iv) on one row; ids/c are indexed by absolute position.  Returns K."""
+                     cfg: DecodeConfig, window: int, k_max: int | None = None) -> int:
+    """Steps (iii)-(iv) on one row; ids/c are indexed by absolute position.  Returns K.
+    ``k_max`` (the dual cache between refreshes) caps K: commits stop at the block end."""
     T = x.shape[0]
     w_eff = min(window, T - p)
     K = window_length(c[p:p + w_eff], cfg.tau_commit)
     K = min(max(K, cfg.min_commit), w_eff)
+    if k_max is not None:
+        K = min(K, k_max)
     x[p:p + K] = ids[p:p + K]                                   # commit verified tokens
     lo = p + window                                             # future region i >= p + L
     if lo < T:
@@ -161,19 +171,33 @@ def prefix_end(p: int, n_prompt: int, block_len: int) -> int:
     return n_prompt + block_len * ((p - n_prompt) // block_len)
 
 
+def computed_range(p: int, n_prompt: int, T: int, cfg: DecodeConfig, refresh: bool) -> tuple:
+    """Positions [start, end) a cached step computes (R18 / dual cache): everything at a
+    refresh; else from the prefix end to T (prefix cache) or to the current block's end
+    (dual cache)."""
+    if refresh:
+        return 0, T
+    pe = prefix_end(p, n_prompt, cfg.block_len)
+    return pe, (T if cfg.kv_cache == 1 else min(pe + cfg.block_len, T))
+
+
 def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
              max_steps: int = 1 << 30, record: bool = True) -> dict:
     """Algorithm 1 for a batch of independent rows.
 
     predict_fn(tokens[T]) -> (ids[M], p1[M], p2[M]) or (ids, p1, p2, H[M]) for the
     generation positions (H, the marginal entropies, is needed by ``confidence = 1``).  With
-    ``cfg.kv_cache`` it is called as predict_fn(tokens[T], start, state): only positions
+    ``cfg.kv_cache = 1`` it is called as predict_fn(tokens[T], start, state): only positions
     >= start need be computed and ``state`` is the row's cache; start is 0 at the first
-    step and whenever prefix_end(p) changes (a refresh), else prefix_end(p).
-    Returns the final x [B][T], per-row steps, the K of every step, the start of every
-    step (-1 for finished rows), Eq. entropy_bound of every step's committed set (NaN
-    without entropies), and (if ``record``) the forward input of every step and the
-    predictions it produced (ids, p1, p2, H).
+    step and whenever prefix_end(p) changes (a refresh), else prefix_end(p).  With
+    ``cfg.kv_cache = 2`` it is called as predict_fn(tokens[T], start, state, end): only
+    positions in [start, end) need be computed (end = T at a refresh, else the block end);
+    the predictions of the other generation positions are kept from the step that last
+    computed them.
+    Returns the final x [B][T], per-row steps, the K of every step, the start and end of
+    every step's computed positions (-1 for finished rows), Eq. entropy_bound of every
+    step's committed set (NaN without entropies), and (if ``record``) the forward input of
+    every step and the predictions it used (ids, p1, p2, H).
     """
     prompt = np.atleast_2d(np.asarray(prompt, dtype=np.int32))
     B, N = prompt.shape
@@ -184,18 +208,23 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
         raise ValueError("acceptance must be 0 (DCV) or 1 (Eq. threshold_pd)")
     if cfg.acceptance == 1 and cfg.block_len < 1:
         raise ValueError("Eq. threshold_pd decoding needs a block length >= 1")
+    if cfg.kv_cache not in (0, 1, 2):
+        raise ValueError("kv_cache must be 0 (none), 1 (prefix) or 2 (dual)")
+    if cfg.kv_cache == 2 and cfg.acceptance != 0:
+        raise ValueError("the dual cache is defined for the DCV acceptance")
     x = np.full((B, T), mask_id, dtype=np.int32)
     x[:, :N] = prompt
     committed = np.zeros((B, T), dtype=bool)  # (Eq. threshold_pd only: commits out of order)
     committed[:, :N] = True
     p = np.full(B, N, dtype=np.int64)
     steps = np.zeros(B, dtype=np.int64)
-    ks, starts, inputs, preds, bounds = [], [], [], [], []
+    ks, starts, ends, inputs, preds, bounds = [], [], [], [], [], []
     caches = [{"pe": None} for _ in range(B)]
     n_iter = 0
     while (p < T).any() and n_iter < max_steps:
         k_step = np.zeros(B, dtype=np.int64)
         s_step = np.full(B, -1, dtype=np.int64)
+        e_step = np.full(B, -1, dtype=np.int64)
         in_step = np.empty((B, T), dtype=np.int32)
         pr = np.zeros((4, B, M))
         pr[3] = np.nan
@@ -207,13 +236,29 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             if cfg.acceptance == 0:
                 remask(x[b], int(p[b]), L, mask_id)              # (i)
             in_step[b] = x[b]
+            k_max = None
             if cfg.kv_cache:                                     # (ii), approximate cache
                 pe = prefix_end(int(p[b]), N, cfg.block_len)
-                s_step[b] = 0 if caches[b]["pe"] != pe else pe
-                out = predict_fn(x[b].copy(), int(s_step[b]), caches[b])
+                refresh = caches[b]["pe"] != pe
+                s_step[b], e_step[b] = computed_range(int(p[b]), N, T, cfg, refresh)
+                if cfg.kv_cache == 1:
+                    out = predict_fn(x[b].copy(), int(s_step[b]), caches[b])
+                else:                                            # dual: the block between refreshes
+                    fresh = predict_fn(x[b].copy(), int(s_step[b]), caches[b], int(e_step[b]))
+                    kept = caches[b].get("pred")
+                    out = []
+                    for f_arr, k_arr in zip(fresh, kept if kept is not None else fresh):
+                        merged = np.array(k_arr, copy=True)
+                        lo_g, hi_g = max(int(s_step[b]), N) - N, int(e_step[b]) - N
+                        merged[lo_g:hi_g] = np.asarray(f_arr)[lo_g:hi_g]
+                        out.append(merged)
+                    caches[b]["pred"] = [a.copy() for a in out]
+                    if not refresh:
+                        k_max = int(e_step[b]) - int(p[b])
                 caches[b]["pe"] = pe
             else:                                                # (ii)
                 s_step[b] = 0
+                e_step[b] = T
                 out = predict_fn(x[b].copy())
             ids, p1, p2 = out[:3]
             H = out[3] if len(out) > 3 else None
@@ -223,7 +268,7 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
             full_c[N:] = decision_confidence(p1, H, cfg)
             p0 = int(p[b])
             if cfg.acceptance == 0:
-                k_step[b] = commit_and_draft(x[b], p0, full_ids, full_c, cfg, L)  # (iii)-(iv)
+                k_step[b] = commit_and_draft(x[b], p0, full_ids, full_c, cfg, L, k_max)  # (iii)-(iv)
                 jp[b] = np.nan if H is None else jpde_bound(np.asarray(H)[p0 - N:p0 - N + k_step[b]])
                 p[b] += k_step[b]                                # dynamically advance
             else:                                                # Eq. threshold_pd in the block
@@ -240,12 +285,13 @@ def generate(predict_fn, prompt: np.ndarray, cfg: DecodeConfig, mask_id: int,
                 pr[3, b] = H
         ks.append(k_step)
         starts.append(s_step)
+        ends.append(e_step)
         bounds.append(jp)
         if record:
             inputs.append(in_step)
             preds.append(pr)
         n_iter += 1
-    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "start": np.array(starts),
+    return {"x": x, "p": p, "steps": steps, "k": np.array(ks), "start": np.array(starts), "end": np.array(ends),
             "jpde": np.array(bounds), "inputs": inputs,
             "preds": preds, "n_iter": n_iter, "done": bool((p >= T).all())}
 

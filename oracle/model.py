@@ -179,15 +179,16 @@ def new_kv_store(shape, T: int) -> list:
 
 
 def predict_from(shape, weights: dict, tokens: np.ndarray, start: int, state: dict, n_prompt: int,
-                 bf16_operands: bool = False, with_entropy: bool = False):
+                 bf16_operands: bool = False, with_entropy: bool = False, end: int | None = None):
     """(ids, p1, p2) over the generation positions [n_prompt, T) computing only positions
-    >= start (the others are returned as -1 / NaN); ``state["kv"]`` is the sequence's
-    key / value store, created on first use.  With ``with_entropy`` the marginal entropy
-    H of every computed position follows (NaN elsewhere)."""
+    in [start, end) (end = T by default; the others are returned as -1 / NaN);
+    ``state["kv"]`` is the sequence's key / value store, created on first use.  With
+    ``with_entropy`` the marginal entropy H of every computed position follows (NaN
+    elsewhere)."""
     T = len(tokens)
     if state.get("kv") is None:
         state["kv"] = new_kv_store(shape, T)
-    pos = np.arange(start, T)
+    pos = np.arange(start, T if end is None else end)
     hid = forward_rows(shape, weights, tokens, pos, state["kv"], bf16_operands)
     M = T - n_prompt
     ids = np.full(M, -1, np.int32)

@@ -104,3 +104,87 @@ def test_refresh_exactly_at_block_changes(weights):
         assert p == T
     # the committed region is a contiguous run and nothing is MASK at the end
     assert (out["x"][:, N:] != TINY.mask_id).all()
+
+
+# ---------------------------------------------------------------- the dual cache (kv_cache = 2)
+def _predict(weights, with_entropy=False):
+    def fn(tokens, start, state, end=None):
+        return model.predict_from(TINY, weights, tokens, start, state, N, with_entropy=with_entropy, end=end)
+    return fn
+
+
+def _run(weights, seed, kv_cache, block_len, tau_c=0.5, tau_d=0.9, L=16):
+    prompt = np.random.default_rng(seed).integers(0, TINY.vocab - 1, (1, N)).astype(np.int32)
+    cfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=tau_d, max_window=L, block_len=block_len, gen_len=M,
+                              kv_cache=kv_cache)
+    if kv_cache:
+        return decode.generate(_predict(weights), prompt, cfg, TINY.mask_id)
+    fn = _predict(weights)
+    return decode.generate(lambda toks: fn(toks, 0, {}), prompt, cfg, TINY.mask_id)
+
+
+@pytest.mark.parametrize("seed,tau_c", [(5, 0.5), (6, 0.3)])
+def test_dual_with_one_block_equals_the_prefix_cache(weights, seed, tau_c):
+    """A block as long as the generation: every step after the first computes [N, T) with
+    fresh predictions at every generation position and the block end is T, so the dual
+    cache is the prefix cache, token for token and step for step."""
+    a = _run(weights, seed, 2, M, tau_c)
+    b = _run(weights, seed, 1, M, tau_c)
+    assert np.array_equal(a["x"], b["x"]) and np.array_equal(a["k"], b["k"])
+    assert np.array_equal(a["start"], b["start"]) and (a["end"] == T).all()
+
+
+def test_dual_with_block_one_equals_the_uncached_loop(weights):
+    """Block length 1: the prefix end is p itself and moves at every step (K >= 1), so
+    every step refreshes (a full forward over fresh keys / values): the uncached
+    Algorithm 1."""
+    a = _run(weights, 7, 2, 1)
+    b = _run(weights, 7, 0, 1)
+    assert np.array_equal(a["x"], b["x"]) and np.array_equal(a["k"], b["k"])
+    assert (a["start"] == 0).all() and (a["end"] == T).all()
+
+
+@pytest.mark.parametrize("seed,tau_c,bk", [(10, 0.5, 8), (10, 0.7, 16), (8, 0.9, 32), (16, 0.7, 8)])
+def test_dual_steps_between_refreshes_stay_in_the_block(weights, seed, tau_c, bk):
+    """Between refreshes a dual step computes exactly the current block [b0, b0 + Bk)
+    (clipped to T), commits only inside it, and the predictions it uses outside the block
+    are those of the last step that computed them (the refresh); every generation ends
+    with the whole sequence committed."""
+    r = _run(weights, seed, 2, bk, tau_c)
+    assert r["done"]
+    p = N
+    last = None
+    n_between = 0
+    for s, (k, st, en, pr) in enumerate(zip(r["k"][:, 0], r["start"][:, 0], r["end"][:, 0], r["preds"])):
+        b0 = N + bk * ((p - N) // bk)
+        if st == 0:
+            assert en == T
+            last = pr[:, 0].copy()
+        else:
+            n_between += 1
+            assert st == b0 and en == min(b0 + bk, T)
+            assert 1 <= k <= en - p
+            out = np.r_[0:st - N, en - N:M]
+            assert np.array_equal(pr[:3, 0][:, out], last[:3][:, out])
+            last[:, st - N:en - N] = pr[:, 0][:, st - N:en - N]
+        p += int(k)
+    assert p == T and n_between > 0
+
+
+def test_dual_cap_binds_where_the_window_runs_past_the_block(weights):
+    """The cap is what keeps commits inside the block: on the same trajectory, some step
+    between refreshes would have committed past the block end had K not been capped (its
+    confident run, by Eq. compute_k over the whole window, reaches beyond the block)."""
+    r = _run(weights, 16, 2, 8, 0.7)
+    p, capped = N, 0
+    for k, st, en, pr in zip(r["k"][:, 0], r["start"][:, 0], r["end"][:, 0], r["preds"]):
+        if st > 0:
+            c = np.zeros(T)
+            c[N:] = pr[1, 0]
+            w_eff = min(16, T - p)
+            k_free = max(decode.window_length(c[p:p + w_eff], 0.7), 1)
+            if k_free > en - p:
+                capped += 1
+                assert k == en - p
+        p += int(k)
+    assert capped > 0

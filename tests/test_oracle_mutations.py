@@ -122,7 +122,7 @@ def _exceeds_ge(c, tau):  # c >= tau instead of c > tau
     return np.asarray(c, dtype=np.float32) >= np.float32(tau)
 
 
-def _commit_drafts_from_p_plus_k(x, p, ids, c, cfg, window):  # future region from p + K
+def _commit_drafts_from_p_plus_k(x, p, ids, c, cfg, window, k_max=None):  # future region from p + K
     T = x.shape[0]
     w_eff = min(window, T - p)
     K = min(max(decode.window_length(c[p:p + w_eff], cfg.tau_commit), cfg.min_commit), w_eff)
@@ -191,8 +191,19 @@ def _entropy_confidence_wrong_sign(H):  # exp(+H)
     return np.exp(np.asarray(H, dtype=np.float64))
 
 
-def _commit_drafts_ignore_chain(x, p, ids, c, cfg, window):  # App. E flag ignored
-    return _ORIG["commit_and_draft"](x, p, ids, c, replace(cfg, contiguous_drafts=False), window)
+def _commit_drafts_ignore_chain(x, p, ids, c, cfg, window, k_max=None):  # App. E flag ignored
+    return _ORIG["commit_and_draft"](x, p, ids, c, replace(cfg, contiguous_drafts=False), window, k_max)
+
+
+def _dual_range_to_the_end(p, n_prompt, T, cfg, refresh):
+    """The dual cache computing the whole suffix between refreshes (the prefix cache's range)."""
+    if refresh:
+        return 0, T
+    return decode.prefix_end(p, n_prompt, cfg.block_len), T
+
+
+def _commit_uncapped(x, p, ids, c, cfg, window, k_max=None):  # the dual cache's block cap ignored
+    return _ORIG["commit_and_draft"](x, p, ids, c, cfg, window)
 
 
 def _threshold_forced_leftmost(x, committed, ids, c, lo, hi, cfg):
@@ -300,6 +311,11 @@ CASES = [
      [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
     ("threshold rule: committed flags ignored", decode, "threshold_commit", _threshold_recommits,
      [lambda: tthr.test_golden_threshold_trajectories(ROOT_GOLDEN)]),
+    ("dual cache: suffix computed to the end", decode, "computed_range", _dual_range_to_the_end,
+     [lambda: tcache.test_dual_steps_between_refreshes_stay_in_the_block(_TINY_W, 10, 0.7, 16)]),
+    ("dual cache: K not capped at the block end", decode, "commit_and_draft", _commit_uncapped,
+     [lambda: tcache.test_dual_cap_binds_where_the_window_runs_past_the_block(_TINY_W),
+      lambda: tcache.test_dual_steps_between_refreshes_stay_in_the_block(_TINY_W, 16, 0.7, 8)]),
     ("prefix end not block-aligned", decode, "prefix_end", _prefix_end_unaligned,
      [tdec.test_prefix_end_is_the_start_of_the_current_block,
       lambda: tcache.test_refresh_exactly_at_block_changes(_TINY_W)]),
