@@ -66,6 +66,11 @@ WORKLOADS = {
                                seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=1),
     "llada8b-long-b8-cache": dict(shape="llada8b", batch=8, n_prompt=512, gen=1024, block=32, window=512,
                                   seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=1),
+    # the dual (prefix + suffix) cache: between refreshes only the current 32-position block
+    "llada8b-long-dualcache": dict(shape="llada8b", batch=1, n_prompt=512, gen=1024, block=32, window=512,
+                                   seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=2),
+    "llada8b-long-b8-dualcache": dict(shape="llada8b", batch=8, n_prompt=512, gen=1024, block=32, window=512,
+                                      seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=2),
     "dream7b-cache": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
                           seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98, cache=1),
     # the LLaDA-8B shape cut to 2 layers (~3 GB on the device): the same GEMM, attention and
@@ -131,9 +136,10 @@ def step_work(shape, B, N, M, rows=None, lm_rows=None, cached=False):
     return per_layer, total, bytes_
 
 
-def cached_rows(kper, N, M, block):
+def cached_rows(kper, N, M, block, dual=False):
     """Per step of a trajectory (per-row K values), the rows the cached step computes and
-    its LM rows (the refresh rule of the key / value cache)."""
+    its LM rows (the refresh rule of the key / value cache; with ``dual``, between
+    refreshes only the current block)."""
     B = len(kper[0])
     T = N + M
     p = [N] * B
@@ -146,9 +152,10 @@ def cached_rows(kper, N, M, block):
                 continue
             pe = N + block * ((p[b] - N) // block)
             start = 0 if pe != pe_prev[b] else pe
+            end = min(pe + block, T) if (dual and start) else T
             pe_prev[b] = pe
-            rows += T - start
-            lm += T - max(start, N)
+            rows += end - start
+            lm += end - max(start, N)
             p[b] += int(k[b])
         out.append((rows, lm))
     return out
@@ -457,7 +464,8 @@ def _config(wl, args):
     return {"workload": f"{wl['shape']}-shape batch {wl['batch']}, prompt {wl['n_prompt']}, gen {wl['gen']}, "
                         f"block {wl['block']}, window {wl['window']}, tau_commit {wl['tau_c']}, "
                         f"tau_draft {wl['tau_d']}, "
-                        + ("approximate prefix key/value cache" if wl.get("cache") else "full recompute"),
+                        + {0: "full recompute", 1: "approximate prefix key/value cache",
+                           2: "dual (prefix + suffix) key/value cache"}[int(wl.get("cache", 0))],
             "global_batch": wl["batch"] * max(1, args.gpus), "seq_len": wl["n_prompt"] + wl["gen"],
             "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single",
             "l2": _l2_note(wl)}
@@ -639,7 +647,7 @@ def run_ours(args):
     if cached:
         # the cached step's work varies (refresh or suffix): the mean over exactly the steps
         # timed (the window replays the trajectory from its start, wrapping at its end)
-        rl = cached_rows(kper, N, M, wl["block"])
+        rl = cached_rows(kper, N, M, wl["block"], dual=cached == 2)
         works = [step_work(shape, B, N, M, r, l, True) for r, l in rl]
         timed_works = [works[i % S] for i in range(args.steps)]
         per_layer = works[0][0]

@@ -61,7 +61,16 @@ typedef struct {
   int32_t block_len;         /* 32: semi-autoregressive block length */
   int32_t gen_len;           /* M, the number of generated positions */
   int32_t kv_cache;          /* 0: full recompute every step; 1: approximate prefix key /
-                                value cache refreshed at block boundaries (see dcl_set_prompt) */
+                                value cache refreshed at block boundaries: between refreshes a
+                                step computes the positions from the block-aligned prefix end
+                                N + block_len * floor((p - N) / block_len) to the end, against
+                                the stored keys / values of the rest; 2: dual (prefix + suffix)
+                                cache, a serving refinement outside the paper: refreshes as 1,
+                                between refreshes only the current block (block_len positions
+                                from the prefix end) is computed, the other generation positions
+                                keep the predictions of the last refresh, and K is capped at
+                                the block end (commits use fresh predictions only); acceptance
+                                0 only */
   int32_t min_commit;        /* 1: K = max(K, min_commit) so every step makes progress;
                                 0 keeps the literal rule (may stall; bounded by max_steps) */
   int32_t contiguous_drafts; /* 0; 1 = App. E variant (drafts only as an unbroken chain) */
@@ -150,9 +159,9 @@ dcl_status dcl_init_random_weights(dcl_ctx* ctx, uint64_t seed, float std, float
  * (Eq. 1).  prompt is host int32 [batch][n_prompt]; batch <= max_batch,
  * n_prompt + cfg->gen_len <= max_seq.  Validates ids, uploads the state and builds
  * (or reuses) the CUDA graph of one step for this shape.
- * Errors: INVALID_ARG (also kv_cache, confidence or acceptance outside {0, 1}, or
- * acceptance = 1 with block_len < 1), UNSUPPORTED (kv_cache = 1 with N, M or block_len not
- * a multiple of 32), CUDA. */
+ * Errors: INVALID_ARG (also kv_cache outside {0, 1, 2}, confidence or acceptance outside
+ * {0, 1}, or acceptance = 1 with block_len < 1), UNSUPPORTED (kv_cache = 1 or 2 with N, M or
+ * block_len not a multiple of 32; kv_cache = 2 with acceptance = 1), CUDA. */
 dcl_status dcl_set_prompt(dcl_ctx* ctx, int32_t batch, const int32_t* prompt, int32_t n_prompt,
                           const dcl_decode_config* cfg);
 
@@ -206,7 +215,7 @@ dcl_status dcl_debug_hidden(dcl_ctx* ctx, int32_t layer, float* h_dev);
  * commit = 1 the step's acceptance (steps (iii)-(iv) and the advance of p) then runs on
  * these predictions, as in dcl_step.  Full recompute only, every sequence unfinished.
  * Synchronises.  Errors: STATE (no prompt, or a finished sequence), INVALID_ARG,
- * UNSUPPORTED (kv_cache = 1), CUDA. */
+ * UNSUPPORTED (kv_cache != 0), CUDA. */
 dcl_status dcl_forward_debug_from(dcl_ctx* ctx, int32_t layer, const float* h_dev, int32_t commit,
                                   void* logits_dev, int32_t* top1_dev, float* p1_dev, float* p2_dev,
                                   float* conf_dev, float* entropy_dev);

@@ -208,11 +208,16 @@ struct RowPlan {
   int* lm_src = nullptr;    // [B*M] computed row of LM row j
   int* lm_slot = nullptr;   // [B*M] b*M + position - N of LM row j
   int* pe_cache = nullptr;  // [B] prefix end the stored keys / values belong to (-1: none)
+  int* kcap = nullptr;      // [B] cap on the step's K: the block end - p between refreshes of the
+                            // dual cache, T otherwise
 };
-// update = 0 plans the rows without recording the prefix end (a forward that commits
-// nothing, e.g. a debug pass, leaves the next step's refresh decision unchanged).
+// cached: 0 every position; 1 the prefix cache (all positions at a refresh, else from the
+// block-aligned prefix end to T); 2 the dual cache (as 1, but between refreshes only the
+// current block).  update = 0 plans the rows without recording the prefix end (a forward
+// that commits nothing, e.g. a debug pass, leaves the next step's refresh decision
+// unchanged).
 cudaError_t row_plan_launch(const RowPlan& rp, const int32_t* p, int batch, int N, int T, int block_len,
-                            int cached, int update, cudaStream_t stream);
+                            int cached, int update, int32_t* x, int window, int mask_id, cudaStream_t stream);
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
                                 int mask_id, int vocab, const __nv_bfloat16* embed, int d,
                                 float* h, int* err, const RowPlan& rp, cudaStream_t stream);
@@ -241,10 +246,11 @@ struct DcvParams {
 // One step's acceptance on the generation rows: ids/c (and ent) are [batch][M] (position
 // N + i).  With ent, jpde[b] accumulates Eq. entropy_bound of the set row b commits.
 // cmt: committed flags [batch][N + M] (read and written with acceptance 1 only).
+// kcap (may be NULL): per-row cap on K (RowPlan::kcap).
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
                               const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
                               int N, int M, const DcvParams& prm, int32_t* done_count, uint8_t* cmt,
-                              cudaStream_t stream);
+                              const int* kcap, cudaStream_t stream);
 // Block acceptance from bf16 logits (dcl_accept): c1 = p1 (mode 0) or exp(-H) (mode 1).
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B,
                                 int P, int V, int32_t* ids, float* c1, float* c2, int mode,

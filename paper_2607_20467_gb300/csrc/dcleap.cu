@@ -222,7 +222,7 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
   if (prof) c->launch_i = 0;
   q.begin(DCL_K_ROWPLAN);
   q.end(row_plan_launch(c->rp, c->p, c->B, c->N, c->T, c->dcfg.block_len, c->dcfg.kv_cache, with_dcv ? 1 : 0,
-                        c->stream),
+                        c->x, c->dcfg.acceptance ? 0 : c->window, m.mask_id, c->stream),
         "row_plan");
   if (h_in) {
     if (q.err == cudaSuccess)
@@ -291,7 +291,7 @@ cudaError_t enqueue_step(dcl_ctx* c, bool with_dcv, bool prof, bool snapshots, c
                   c->dcfg.contiguous_drafts, c->dcfg.acceptance, c->dcfg.block_len};
     q.begin(DCL_K_DCV);
     q.end(dcv_commit_launch(c->x, c->p, c->k, c->steps, c->top1, co.conf, c->ent, c->jpde, c->B, c->N, c->M, prm,
-                            c->done_count, c->cmt, c->stream),
+                            c->done_count, c->cmt, c->rp.kcap, c->stream),
           "dcv_commit");
   }
   if (what) *what = q.what;
@@ -662,7 +662,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->attn = (__nv_bfloat16*)dev_alloc(c, 2 * R * H * hd);
     c->vt = (__half*)dev_alloc(c, 2 * (size_t)max_batch * G * hd * attn_vt_pitch(max_seq));
     c->kbuf = (__nv_bfloat16*)dev_alloc(c, 2 * R * G * hd);
-    c->rp_buf = (int*)dev_alloc(c, sizeof(int) * (2 + 4 * R + 3 * (size_t)max_batch));
+    c->rp_buf = (int*)dev_alloc(c, sizeof(int) * (2 + 4 * R + 4 * (size_t)max_batch));
     c->act = (__nv_bfloat16*)dev_alloc(c, 2 * R * F);
     c->xg = (__nv_bfloat16*)dev_alloc(c, 2 * R * d);
     c->part = (float4*)dev_alloc(c, sizeof(float4) * R * nblk);
@@ -711,6 +711,7 @@ dcl_status dcl_create(const dcl_model_config* cfg, int32_t max_batch, int32_t ma
     c->rp.seq_off = c->rp.lm_slot + R;
     c->rp.seq_len = c->rp.seq_off + max_batch;
     c->rp.pe_cache = c->rp.seq_len + max_batch;
+    c->rp.kcap = c->rp.pe_cache + max_batch;
     if (rope_table_build(c->rope_cos, c->rope_sin, max_seq, (int)hd, m.rope_theta, c->stream) != cudaSuccess) {
       dev_free_all(c);
       release_stream(c);
@@ -796,11 +797,13 @@ dcl_status dcl_set_prompt(dcl_ctx* c, int32_t batch, const int32_t* prompt, int3
   if (batch <= 0 || batch > c->max_batch) return fail(c, DCL_ERR_INVALID_ARG, "batch %d outside [1, %d]", batch, c->max_batch);
   if (n_prompt < 0 || cfg->gen_len <= 0 || n_prompt + cfg->gen_len > c->max_seq)
     return fail(c, DCL_ERR_INVALID_ARG, "N + M = %d + %d exceeds max_seq %d", n_prompt, cfg->gen_len, c->max_seq);
-  if (cfg->kv_cache != 0 && cfg->kv_cache != 1) return fail(c, DCL_ERR_INVALID_ARG, "kv_cache must be 0 or 1");
+  if (cfg->kv_cache < 0 || cfg->kv_cache > 2) return fail(c, DCL_ERR_INVALID_ARG, "kv_cache must be 0, 1 or 2");
   if (cfg->confidence != 0 && cfg->confidence != 1) return fail(c, DCL_ERR_INVALID_ARG, "confidence must be 0 or 1");
   if (cfg->acceptance != 0 && cfg->acceptance != 1) return fail(c, DCL_ERR_INVALID_ARG, "acceptance must be 0 or 1");
   if (cfg->acceptance == 1 && cfg->block_len <= 0)
     return fail(c, DCL_ERR_INVALID_ARG, "the threshold rule (acceptance = 1) needs block_len >= 1");
+  if (cfg->kv_cache == 2 && cfg->acceptance != 0)
+    return fail(c, DCL_ERR_UNSUPPORTED, "the dual cache (kv_cache = 2) is defined for the DCV acceptance");
   if (cfg->kv_cache && (cfg->block_len <= 0 || cfg->block_len % 32 || n_prompt % 32 || cfg->gen_len % 32))
     return fail(c, DCL_ERR_UNSUPPORTED, "the key / value cache needs N, M and the block length multiples of 32");
   if (cfg->max_window < 0 || cfg->min_commit < 0 || !(cfg->tau_commit == cfg->tau_commit) ||

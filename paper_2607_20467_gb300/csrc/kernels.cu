@@ -23,16 +23,18 @@ constexpr unsigned kFull = 0xffffffffu;
 // refresh, the block-aligned prefix end N + Bk*floor((p-N)/Bk) when the stored keys and
 // values are that block's, T for a finished row), the row offsets, and the row tables.
 __global__ void __launch_bounds__(1024) row_plan_kernel(RowPlan rp, const int32_t* __restrict__ p, int B, int N,
-                                                        int T, int Bk, int cached, int update) {
+                                                        int T, int Bk, int cached, int update,
+                                                        int32_t* __restrict__ x, int window, int mask_id) {
   pdl_wait();
   pdl_launch_dependents();
-  extern __shared__ int lm_off[];  // [B]
+  extern __shared__ int lm_off[];  // [B], then the sequences' first computed positions [B]
+  int* st_pos = lm_off + B;
   const int M = T - N;
   if (threadIdx.x == 0) {
     int off = 0, lmoff = 0;
     for (int b = 0; b < B; ++b) {
       const int pb = p[b];
-      int start;
+      int start, end = T, cap = T;
       if (pb >= T) {
         start = T;
       } else if (!cached) {
@@ -41,25 +43,38 @@ __global__ void __launch_bounds__(1024) row_plan_kernel(RowPlan rp, const int32_
         const int pe = N + Bk * ((pb - N) / Bk);
         start = (rp.pe_cache[b] == pe) ? pe : 0;
         if (update) rp.pe_cache[b] = pe;
+        if (cached == 2 && start != 0) {  // dual cache between refreshes: the current block
+          end = min(pe + Bk, T);
+          cap = end - pb;
+        }
       }
       rp.seq_off[b] = off;
-      rp.seq_len[b] = T - start;
-      off += T - start;
+      rp.seq_len[b] = end - start;
+      rp.kcap[b] = cap;
+      st_pos[b] = start;
+      off += end - start;
       lm_off[b] = lmoff;
-      lmoff += T - max(start, N);
+      lmoff += max(end - max(start, N), 0);
     }
     rp.counts[0] = off;
     rp.counts[1] = lmoff;
   }
   __syncthreads();
   for (int b = 0; b < B; ++b) {
-    const int len = rp.seq_len[b], off = rp.seq_off[b], start = T - len;
+    const int len = rp.seq_len[b], off = rp.seq_off[b], start = st_pos[b], end = start + len;
     for (int i = threadIdx.x; i < len; i += blockDim.x) {
       rp.row_seq[off + i] = b;
       rp.row_pos[off + i] = start + i;
     }
+    if (cached == 2 && window > 0 && p[b] < T) {
+      // Eq. remasking over the window positions past the computed rows (the embedding
+      // kernel re-masks the computed ones): between refreshes of the dual cache the window
+      // runs past the block
+      const int pb = p[b], w0 = max(pb, end), w1 = min(pb + window, T);
+      for (int t = w0 + threadIdx.x; t < w1; t += blockDim.x) x[(size_t)b * T + t] = mask_id;
+    }
     const int s0 = max(start, N);
-    for (int i = threadIdx.x; i < T - s0; i += blockDim.x) {
+    for (int i = threadIdx.x; i < end - s0; i += blockDim.x) {
       const int pos = s0 + i;
       rp.lm_src[lm_off[b] + i] = off + (pos - start);
       rp.lm_slot[lm_off[b] + i] = b * M + (pos - N);
@@ -289,7 +304,7 @@ __global__ void __launch_bounds__(COMBINE_THREADS) lmhead_combine_kernel(
 // xrow / ids / c indexed by absolute position; window [pb, pb + min(L, T - pb)).
 // Runs on one full warp.  Returns K (valid on every lane).
 __device__ int dcv_row(int32_t* xrow, const int32_t* ids, const float* c, int pb, int T,
-                       const DcvParams& prm) {
+                       const DcvParams& prm, int kmax) {
   const int lane = threadIdx.x & 31;
   const int w_eff = min(prm.window, T - pb);
   // Eq. compute_k: K = sum_i prod_{j<=i} 1(c_{p+j} > tau_commit) = length of the leading
@@ -306,7 +321,7 @@ __device__ int dcv_row(int32_t* xrow, const int32_t* ids, const float* c, int pb
     K += __ffs(~bal) - 1;
     break;
   }
-  K = min(max(K, prm.min_commit), w_eff);
+  K = min(min(max(K, prm.min_commit), w_eff), kmax);  // (kmax: the dual cache's block end)
   for (int i = lane; i < K; i += 32) xrow[pb + i] = ids[pb + i];  // commit x[p:p+K]
   // Eq. draft_update over the future region i >= p + L (p before the advance)
   const int lo = pb + prm.window;
@@ -411,7 +426,8 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
                                   int32_t* __restrict__ k_out, int32_t* __restrict__ steps,
                                   const int32_t* __restrict__ ids, const float* __restrict__ c,
                                   const float* __restrict__ ent, float* __restrict__ jpde, int N, int M,
-                                  DcvParams prm, int32_t* done_count, uint8_t* __restrict__ cmt) {
+                                  DcvParams prm, int32_t* done_count, uint8_t* __restrict__ cmt,
+                                  const int* __restrict__ kcap) {
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.x;
@@ -448,7 +464,8 @@ __global__ void dcv_commit_kernel(int32_t* __restrict__ x, int32_t* __restrict__
     return;
   }
   // shift the [M]-sized generation arrays so they are indexed by absolute position
-  const int K = dcv_row(x + (size_t)b * T, ids + (size_t)b * M - N, c + (size_t)b * M - N, pb, T, prm);
+  const int K = dcv_row(x + (size_t)b * T, ids + (size_t)b * M - N, c + (size_t)b * M - N, pb, T, prm,
+                        kcap ? kcap[b] : T);
   if (ent) {
     // Eq. entropy_bound of the committed set U = [p, p + K): sum_U H - max_U H
     const float* h = ent + (size_t)b * M - N + pb;
@@ -657,7 +674,7 @@ __global__ void accept_commit_kernel(const int32_t* __restrict__ committed,
     K = threshold_row(x + (size_t)b * P, nullptr, ids + (size_t)b * P, c1 + (size_t)b * P, nullptr, pb, P, prm, &hs,
                       &hm);
   } else {
-    K = dcv_row(x + (size_t)b * P, ids + (size_t)b * P, c1 + (size_t)b * P, pb, P, prm);
+    K = dcv_row(x + (size_t)b * P, ids + (size_t)b * P, c1 + (size_t)b * P, pb, P, prm, P);
   }
   if (threadIdx.x == 0) k[b] = K;
 }
@@ -702,10 +719,11 @@ __global__ void generate_kernel(__nv_bfloat16* __restrict__ dst, uint64_t seed, 
 
 // ------------------------------------------------------------------ launchers
 cudaError_t row_plan_launch(const RowPlan& rp, const int32_t* p, int batch, int N, int T, int block_len, int cached,
-                            int update, cudaStream_t stream) {
-  if (batch <= 0 || batch > 4096 || (cached && block_len <= 0)) return cudaErrorInvalidValue;
-  return launch_pdl(row_plan_kernel, 1, 1024, sizeof(int) * batch, stream, rp, p, batch, N, T, block_len, cached,
-                    update);
+                            int update, int32_t* x, int window, int mask_id, cudaStream_t stream) {
+  if (batch <= 0 || batch > 4096 || (cached && block_len <= 0) || cached < 0 || cached > 2 || (cached == 2 && !x))
+    return cudaErrorInvalidValue;
+  return launch_pdl(row_plan_kernel, 1, 1024, 2 * sizeof(int) * batch, stream, rp, p, batch, N, T, block_len, cached,
+                    update, x, window, mask_id);
 }
 
 cudaError_t embed_remask_launch(int32_t* x, const int32_t* p, int batch, int T, int window,
@@ -741,10 +759,10 @@ cudaError_t lmhead_combine_launch(const float4* part, const float* upart, int ro
 cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* steps,
                               const int32_t* ids, const float* c, const float* ent, float* jpde, int batch,
                               int N, int M, const DcvParams& prm, int32_t* done_count, uint8_t* cmt,
-                              cudaStream_t stream) {
+                              const int* kcap, cudaStream_t stream) {
   if (prm.acceptance == 1 && (prm.block_len < 1 || !cmt)) return cudaErrorInvalidValue;
   return launch_pdl(dcv_commit_kernel, batch, 32, 0, stream, x, p, k_out, steps, ids, c, ent, jpde, N, M, prm,
-                    done_count, cmt);
+                    done_count, cmt, kcap);
 }
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,

@@ -133,3 +133,15 @@ def test_steps_by_rows_groups_and_grades_each_row_count():
     # 32 suffix rows at batch 1 stream 15 GB of weights for far fewer flops: HBM-bound
     small = bench.steps_by_rows([(32, 32)], [bench.step_work(shape, 1, N, M, 32, 32, True)], [6.0], peaks)
     assert small[0]["bound"] == "hbm"
+
+
+def test_cached_rows_of_the_dual_cache():
+    """N = 4, M = 8, block 4, dual cache: the first step refreshes (12 rows), the second
+    stays in the block [4, 8) and computes only that block (4 rows, all generation rows),
+    the third crosses into [8, 12) and refreshes."""
+    out = bench.cached_rows([np.array([1]), np.array([3]), np.array([4])], 4, 8, 4, dual=True)
+    assert out == [(12, 8), (4, 4), (12, 8)]
+    # two rows: at the second step row 0 crosses into [8, 12) and refreshes, row 1 stays in
+    # [4, 8) and computes that block
+    out = bench.cached_rows([np.array([5, 1]), np.array([1, 8])], 4, 8, 4, dual=True)
+    assert out == [(24, 16), (4 + 12, 4 + 8)]

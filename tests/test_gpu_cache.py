@@ -1,6 +1,7 @@
-"""The approximate prefix key / value cache (kv_cache = 1) on the GPU against the oracle's
-cached Algorithm 1 (``decode.generate`` with ``model.predict_from``, bf16 operands), on the
-2-layer / d 256 / 4x64 heads / vocab 4096 model (prompt 32, gen 64, block 32).
+"""The approximate prefix key / value cache (kv_cache = 1) and the dual cache (kv_cache = 2)
+on the GPU against the oracle's cached Algorithm 1 (``decode.generate`` with
+``model.predict_from``, bf16 operands), on the 2-layer / d 256 / 4x64 heads / vocab 4096
+model (prompt 32, gen 64, block 32).
 
 Under the cache a step's result depends on the keys and values stored at earlier steps,
 so states cannot be loaded one by one (a loaded state forces a refresh): the GPU and the
@@ -36,7 +37,8 @@ def weights():
 
 
 def _cached(weights):
-    return lambda tok, start, state: model.predict_from(TINY, weights, tok, start, state, N, bf16_operands=True)
+    return lambda tok, start, state, end=None: model.predict_from(TINY, weights, tok, start, state, N,
+                                                                   bf16_operands=True, end=end)
 
 
 def _split_is_near_tie(ref, s, b, p_prev, ocfg):
@@ -49,11 +51,13 @@ def _split_is_near_tie(ref, s, b, p_prev, ocfg):
         (np.abs(c[p_prev:] - ocfg.tau_draft) <= E2E_TOL).any() or (g[p_prev:] <= E2E_TOL).any()
 
 
-@pytest.mark.parametrize("seed,B,tau_c,L", [(0, 1, 0.7, 32), (1, 1, 0.5, 16), (2, 3, 0.7, 32), (3, 2, 0.3, 64)])
-def test_cached_generation_matches_oracle(dcl, weights, seed, B, tau_c, L):
+@pytest.mark.parametrize("kv", [1, 2])
+@pytest.mark.parametrize("seed,B,tau_c,L", [(0, 1, 0.7, 32), (1, 1, 0.5, 16), (2, 3, 0.7, 32), (3, 2, 0.3, 64),
+                                            (4, 2, 0.9, 48)])
+def test_cached_generation_matches_oracle(dcl, weights, seed, B, tau_c, L, kv):
     prompt = syn.prompt_ids(300 + seed, B, N, TINY.mask_id)
-    cfg = dcl.decode_config(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=1)
-    ocfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=1)
+    cfg = dcl.decode_config(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=kv)
+    ocfg = decode.DecodeConfig(tau_commit=tau_c, tau_draft=0.98, max_window=L, gen_len=M, block_len=32, kv_cache=kv)
     ref = decode.generate(_cached(weights), prompt, ocfg, TINY.mask_id)
     assert ref["done"]
     with dcl.Context(TINY, max_batch=B, max_seq=T) as ctx:
@@ -85,7 +89,7 @@ def test_cached_generation_matches_oracle(dcl, weights, seed, B, tau_c, L):
         if split[b] is None:
             assert (states[-1][0][b, N:] == ref["x"][b, N:]).all()
     refreshes = int((ref["start"] == 0).sum())
-    print(f"seed {seed}: {ref['n_iter']} oracle steps ({refreshes} refresh row-steps); "
+    print(f"kv_cache {kv} seed {seed}: {ref['n_iter']} oracle steps ({refreshes} refresh row-steps); "
           f"rows split at a near tie: {sum(x is not None for x in split)} of {B}")
 
 
@@ -111,3 +115,35 @@ def test_cache_changes_the_result_only_through_stale_keys(dcl, weights):
         a.restart()
         out2, st2, _ = a.generate(max_steps=4 * M)
         assert (out2 == out).all() and st2.steps == st.steps
+
+
+def test_dual_cache_with_one_block_is_the_prefix_cache(dcl, weights):
+    """A block as long as the generation: the dual cache computes the same rows as the
+    prefix cache at every step and its K cap never binds, so the two GPU generations are
+    identical state for state."""
+    prompt = syn.prompt_ids(21, 2, N, TINY.mask_id)
+    runs = []
+    for kv in (1, 2):
+        with dcl.Context(TINY, max_batch=2, max_seq=T) as ctx:
+            ctx.load_weights(weights)
+            ctx.set_prompt(prompt, dcl.decode_config(tau_commit=0.6, max_window=32, gen_len=M, block_len=M,
+                                                     kv_cache=kv))
+            states = []
+            for _ in range(2 * M):
+                x, p = ctx.get_state()
+                states.append((x.copy(), p.copy()))
+                if (p >= T).all():
+                    break
+                ctx.step()
+            runs.append(states)
+    assert len(runs[0]) == len(runs[1])
+    for (xa, pa), (xb, pb) in zip(*runs):
+        assert (xa == xb).all() and (pa == pb).all()
+
+
+def test_dual_cache_rejects_the_threshold_rule(dcl, weights):
+    with dcl.Context(TINY, max_batch=1, max_seq=T) as ctx:
+        ctx.load_weights(weights)
+        with pytest.raises(dcl.DcleapError):
+            ctx.set_prompt(syn.prompt_ids(1, 1, N, TINY.mask_id),
+                           dcl.decode_config(gen_len=M, kv_cache=2, acceptance=1))

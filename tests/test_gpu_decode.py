@@ -332,7 +332,7 @@ def test_error_statuses(dcl, weights):
             c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=1, block_len=16))
         assert e.value.status == dcl.DCL_ERR_UNSUPPORTED
         with pytest.raises(dcl.DcleapError) as e:
-            c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=2))
+            c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), dcl.decode_config(gen_len=M, kv_cache=3))
         assert e.value.status == dcl.DCL_ERR_INVALID_ARG
         c.load_weights(weights)
         c.set_prompt(syn.prompt_ids(0, 1, N, TINY.mask_id), cfg)
