@@ -96,7 +96,7 @@ def test_accept_raw_inputs_guard_band_report(ops):
     """The acceptance pass on the seeded config-2 inputs as generated (no position moved out
     of the guard band): K and x must equal the oracle's on every row whose decisions have
     no confidence within 1e-4 of a threshold; on the other rows they must be one of the
-    outcomes the band allows.  The counts are printed (the design doc keeps them)."""
+    outcomes the band allows.  The counts are printed."""
     import paper_2607_20467_gb300 as dcl
     B, P, V, L, tc, td = 64, 32, 126464, 16, 0.7, 0.98
     d = syn.accept_inputs(7, B, P, V, V - 1)

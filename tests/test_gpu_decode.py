@@ -352,7 +352,7 @@ def test_near_tie_divergence_fraction(dcl, ctx, weights):
     """32 free-running generations (prompt 32, gen 64, window 32, thresholds 0.7 / 0.98) on
     the GPU and in the oracle: no split may follow a decision whose oracle margin exceeds
     the end-to-end drift E2E_TOL; the fraction of diverged sequences and the margins at the
-    splits are reported (the design doc keeps the table)."""
+    splits are reported."""
     import bench
     r = bench.near_tie_study(ctx, dcl, TINY, weights, N, M, 32, 0.7, 0.98, range(32), tol=1e-3, drift=E2E_TOL)
     print("near-tie study:", {k: v for k, v in r.items() if k != "split_margins"},
