@@ -73,6 +73,8 @@ WORKLOADS = {
                                       seed=1, lm_scale=12.0, tau_c=0.70, tau_d=0.98, cache=2),
     "dream7b-cache": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
                           seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98, cache=1),
+    "dream7b-dualcache": dict(shape="dream7b", batch=16, n_prompt=384, gen=512, block=32, window=256,
+                              seed=2, lm_scale=12.8, tau_c=0.70, tau_d=0.98, cache=2),
     # the LLaDA-8B shape cut to 2 layers (~3 GB on the device): the same GEMM, attention and
     # LM-head launches as the full model, small enough for ncu captures with replay
     "llada8b-2l": dict(shape="llada8b-2l", batch=1, n_prompt=256, gen=256, block=32, window=128,
