@@ -48,6 +48,8 @@ CONFIGS = {
     # the approximate prefix key / value cache (refresh at every 32-position block)
     "llada8b-long-cache": ("llada8b", 1, 512, 1024, 512, 1, 12.0, None, 1, 0),
     "llada8b-long-b8-cache": ("llada8b", 8, 512, 1024, 512, 1, 12.0, 40, 1, 0),
+    # the dual cache: between refreshes only the current block, K capped at its end
+    "llada8b-long-dualcache": ("llada8b", 1, 512, 1024, 512, 1, 12.0, 60, 2, 0),
     "dream7b-cache": ("dream7b", 16, 384, 512, 256, 2, 12.8, 40, 1, 0),
     # the thresholds see exp(-entropy) instead of the top-1 probability
     "llada8b-entropy": ("llada8b", 1, 256, 256, 128, 1, 12.0, 48, 0, 1),
@@ -110,8 +112,9 @@ def test_first_blocks_match_oracle(dcl, name, layers):
         assert err.mean() <= tol_mean and err.max() <= tol_max, (layer, float(err.mean()), float(err.max()))
 
 
-def _expected_step(x0, p0, top1, c1, N, L, mask_id):
-    """The acceptance rule on one row (absolute positions; top1 / c1 over [N, T))."""
+def _expected_step(x0, p0, top1, c1, N, L, mask_id, k_max=None):
+    """The acceptance rule on one row (absolute positions; top1 / c1 over [N, T)); k_max
+    caps K (the dual cache between refreshes: the block end)."""
     T = x0.shape[0]
     if p0 >= T:
         return x0.copy(), 0
@@ -121,6 +124,8 @@ def _expected_step(x0, p0, top1, c1, N, L, mask_id):
     while run < w and c1[p0 - N + run] > tc:
         run += 1
     K = min(max(run, 1), w)
+    if k_max is not None:
+        K = min(K, k_max)
     x = x0.copy()
     x[p0:p0 + w] = mask_id
     x[p0:p0 + K] = top1[p0 - N:p0 - N + K]
@@ -132,10 +137,11 @@ def _expected_step(x0, p0, top1, c1, N, L, mask_id):
 
 @pytest.mark.parametrize("name", list(CONFIGS))
 def test_generation_follows_acceptance_rule(dcl, name):
-    shape, B, N, M, L, seed, lm_scale, check_steps, _, conf_kind = CONFIGS[name]
+    shape, B, N, M, L, seed, lm_scale, check_steps, cache, conf_kind = CONFIGS[name]
     sh = syn.SHAPES[shape]
     T = N + M
     ctx, stream, prompt = _context(dcl, name)
+    pe_prev = [None] * B  # (the dual cache: the prefix end of each row's last step)
     try:
         top1 = torch.zeros(B * M, dtype=torch.int32, device="cuda")
         c1 = torch.zeros(B * M, device="cuda")
@@ -168,7 +174,13 @@ def test_generation_follows_acceptance_rule(dcl, name):
             k = ctx.step(return_k=True)
             x1, p1 = ctx.get_state()
             for b in range(B):
-                x_exp, K = _expected_step(x0[b], int(p0[b]), ids[b], conf[b], N, L, sh.mask_id)
+                k_max = None
+                if cache and int(p0[b]) < T:
+                    pe = N + 32 * ((int(p0[b]) - N) // 32)
+                    if cache == 2 and pe == pe_prev[b]:
+                        k_max = min(pe + 32, T) - int(p0[b])
+                    pe_prev[b] = pe
+                x_exp, K = _expected_step(x0[b], int(p0[b]), ids[b], conf[b], N, L, sh.mask_id, k_max)
                 assert int(k[b]) == K, (steps, b, int(k[b]), K)
                 assert int(p1[b]) == int(p0[b]) + K
                 assert (x1[b] == x_exp).all(), (steps, b, np.nonzero(x1[b] != x_exp)[0][:8])
