@@ -603,6 +603,8 @@ template <int THREADS, bool ENT>
 __global__ void __launch_bounds__(THREADS, 2048 / THREADS) accept_stats_kernel(
     const __nv_bfloat16* __restrict__ logits, const int32_t* __restrict__ committed, int B, int P, int V,
     int32_t* __restrict__ ids, float* __restrict__ c1, float* __restrict__ c2, int mode) {
+  pdl_wait();  // the logits, and the previous call's commit pass that read this scratch
+  pdl_launch_dependents();
   int pos = blockIdx.x;  // b * P + i
   if (B <= ACC_COMPACT_MAX_B) {
     __shared__ int pos_s;
@@ -662,6 +664,8 @@ __global__ void accept_commit_kernel(const int32_t* __restrict__ committed,
                                      const int32_t* __restrict__ ids, const float* __restrict__ c1,
                                      int32_t* __restrict__ x, int32_t* __restrict__ k, int P,
                                      DcvParams prm) {
+  pdl_wait();  // the statistics pass
+  pdl_launch_dependents();
   const int b = blockIdx.x;
   const int pb = committed[b];
   if (pb >= P || pb < 0) {
@@ -767,20 +771,19 @@ cudaError_t dcv_commit_launch(int32_t* x, int32_t* p, int32_t* k_out, int32_t* s
 
 cudaError_t accept_stats_launch(const __nv_bfloat16* logits, const int32_t* committed, int B, int P,
                                 int V, int32_t* ids, float* c1, float* c2, int mode, cudaStream_t stream) {
+  // Both passes are dependent launches: each is scheduled while its predecessor drains and
+  // waits for it (pdl_wait) before touching memory.
   if (mode)
-    accept_stats_kernel<ACC_THREADS, true><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, B, P, V, ids, c1, c2,
-                                                                             mode);
-  else
-    accept_stats_kernel<ACC_THREADS, false><<<B * P, ACC_THREADS, 0, stream>>>(logits, committed, B, P, V, ids, c1, c2,
-                                                                              mode);
-  return cudaGetLastError();
+    return launch_pdl(accept_stats_kernel<ACC_THREADS, true>, B * P, ACC_THREADS, 0, stream, logits, committed, B, P,
+                      V, ids, c1, c2, mode);
+  return launch_pdl(accept_stats_kernel<ACC_THREADS, false>, B * P, ACC_THREADS, 0, stream, logits, committed, B, P, V,
+                    ids, c1, c2, mode);
 }
 
 cudaError_t accept_commit_launch(const int32_t* committed, const int32_t* ids, const float* c1,
                                  int32_t* x, int32_t* k, int B, int P, const DcvParams& prm,
                                  cudaStream_t stream) {
-  accept_commit_kernel<<<B, 32, 0, stream>>>(committed, ids, c1, x, k, P, prm);
-  return cudaGetLastError();
+  return launch_pdl(accept_commit_kernel, B, 32, 0, stream, committed, ids, c1, x, k, P, prm);
 }
 
 cudaError_t empty_launch(cudaStream_t stream) { return launch_pdl(empty_step_kernel, 1, 32, 0, stream); }
