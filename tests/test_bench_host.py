@@ -69,6 +69,26 @@ def test_accept_algorithmic_bytes():
     assert total * wl["vocab"] * 2 == pytest.approx(239.8e6, rel=1e-3)
 
 
+def test_traffic_comes_only_from_counters_of_the_current_source(tmp_path, monkeypatch):
+    """The roofline's `traffic` is the ncu DRAM byte count of the kernel as it stands: the
+    acceptance pass's figure covers at least the rows it must read, and any change to the
+    kernel's source file turns the figure into null."""
+    algo = 948 * bench.WORKLOADS["accept"]["vocab"] * 2
+    t = bench._traffic_from_profiles("accept_stats", "kernels.cu")
+    assert t is not None and algo <= t < 1.05 * algo
+    assert bench._traffic_from_profiles("gemm_mlp") is not None
+    assert bench._traffic_from_profiles("no_such_kernel") is None
+    csrc = tmp_path / "paper_2607_20467_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "profiles").mkdir()
+    with open(os.path.join(bench.ROOT, "profiles", "traffic.txt")) as f:
+        (tmp_path / "profiles" / "traffic.txt").write_text(f.read())
+    with open(os.path.join(bench.ROOT, "paper_2607_20467_gb300", "csrc", "kernels.cu")) as f:
+        (csrc / "kernels.cu").write_text(f.read() + "// edited\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench._traffic_from_profiles("accept_stats", "kernels.cu") is None
+
+
 def test_sweep_refuses_the_acceptance_workload():
     r = subprocess.run([sys.executable, "bench.py", "--workload", "accept", "--sweep"], cwd=ROOT,
                        capture_output=True, text=True, timeout=120)
