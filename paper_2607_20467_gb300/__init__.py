@@ -139,6 +139,31 @@ def _ptr(t):
     raise TypeError(f"cannot pass {type(t)} as a pointer")
 
 
+def _dev(t, name, itemsize, count=0):
+    """Device pointer for a ``*_dev`` argument: a contiguous CUDA tensor of ``itemsize``-byte
+    elements holding at least ``count`` of them (None passes as NULL, an int as a raw device
+    address).  A host array, a CPU tensor, another element size or a short buffer is
+    refused here, before a kernel could read or write past it."""
+    if t is None or isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray) or not getattr(t, "is_cuda", False):
+        raise ValueError(f"{name}: a device buffer (a CUDA tensor) is required")
+    if t.element_size() != itemsize:
+        raise TypeError(f"{name}: elements of {itemsize} bytes expected, got {t.dtype}")
+    if t.numel() < count:
+        raise ValueError(f"{name}: at least {count} elements needed, {t.numel()} given")
+    return _ptr(t)
+
+
+def weight_elements(shape, kind) -> int:
+    """Elements of weight tensor `kind` (DCL_W_*) of a model of this shape: matrices in the
+    nn.Linear layout [out_features][in_features], gains [d_model]."""
+    d, hd, H, G, F, V = shape.d_model, shape.head_dim, shape.n_heads, shape.n_kv_heads, shape.ffn_dim, shape.vocab
+    return {DCL_W_EMBED: V * d, DCL_W_ATTN_NORM: d, DCL_W_Q: H * hd * d, DCL_W_K: G * hd * d,
+            DCL_W_V: G * hd * d, DCL_W_O: d * H * hd, DCL_W_MLP_NORM: d, DCL_W_GATE: F * d,
+            DCL_W_UP: F * d, DCL_W_DOWN: d * F, DCL_W_FINAL_NORM: d, DCL_W_LM_HEAD: V * d}[kind]
+
+
 def model_config(shape) -> ModelConfig:
     return ModelConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads,
                        shape.head_dim, shape.ffn_dim, shape.vocab, shape.mask_id,
@@ -201,6 +226,13 @@ class Context:
         is_dev = 0 if isinstance(src, np.ndarray) else int(src.is_cuda)
         if isinstance(src, np.ndarray) and src.dtype != np.uint16:
             raise TypeError("host weights are bf16 bit patterns (uint16)")
+        if not isinstance(src, np.ndarray) and src.element_size() != 2:
+            raise TypeError(f"weights are bf16 (2-byte elements), got {src.dtype}")
+        if self.shape is not None and 0 <= kind <= DCL_W_LM_HEAD:
+            need = weight_elements(self.shape, kind)
+            have = src.size if isinstance(src, np.ndarray) else src.numel()
+            if have < need:
+                raise ValueError(f"weight {kind}: {need} elements needed, {have} given")
         self._check(self._L.dcl_set_weight(self.ptr, kind, layer, _ptr(src), is_dev))
 
     def init_random_weights(self, seed, std=0.02, lm_head_scale=1.0, norm_gain_std=0.0):
@@ -248,43 +280,63 @@ class Context:
         p = np.ascontiguousarray(p, dtype=np.int32)
         self._check(self._L.dcl_set_state(self.ptr, _ptr(x), _ptr(p)))
 
+    def _outs(self, logits, top1, p1, p2, conf, entropy):
+        """Device pointers of the per-position outputs of a forward ([batch][M], logits
+        [batch][M][vocab])."""
+        n = self.batch * self.gen_len
+        vocab = self.shape.vocab if self.shape is not None else 0
+        return (_dev(logits, "logits", 2, n * vocab), _dev(top1, "top1", 4, n), _dev(p1, "p1", 4, n),
+                _dev(p2, "p2", 4, n), _dev(conf, "conf", 4, n), _dev(entropy, "entropy", 4, n))
+
+    def _stream_elems(self):
+        """Elements of a residual stream buffer: float [batch*(N+M)][d_model]."""
+        d = self.shape.d_model if self.shape is not None else 0
+        return self.batch * (self.n_prompt + self.gen_len) * d
+
     def forward_debug(self, logits=None, top1=None, p1=None, p2=None, conf=None, entropy=None):
-        self._check(self._L.dcl_forward_debug(self.ptr, _ptr(logits), _ptr(top1), _ptr(p1), _ptr(p2),
-                                              _ptr(conf), _ptr(entropy)))
+        self._check(self._L.dcl_forward_debug(self.ptr, *self._outs(logits, top1, p1, p2, conf, entropy)))
 
     def debug_hidden(self, layer, h):
-        self._check(self._L.dcl_debug_hidden(self.ptr, layer, _ptr(h)))
+        self._check(self._L.dcl_debug_hidden(self.ptr, layer, _dev(h, "h", 4, self._stream_elems())))
 
     def forward_debug_from(self, layer, h, commit=False, logits=None, top1=None, p1=None, p2=None, conf=None,
                            entropy=None):
-        self._check(self._L.dcl_forward_debug_from(self.ptr, layer, _ptr(h), int(bool(commit)), _ptr(logits),
-                                                   _ptr(top1), _ptr(p1), _ptr(p2), _ptr(conf), _ptr(entropy)))
+        self._check(self._L.dcl_forward_debug_from(self.ptr, layer, _dev(h, "h", 4, self._stream_elems()),
+                                                   int(bool(commit)),
+                                                   *self._outs(logits, top1, p1, p2, conf, entropy)))
 
     def accept(self, logits, committed, x, cfg: DecodeConfig, k):
         B, P, V = logits.shape
-        self._check(self._L.dcl_accept(self.ptr, _ptr(logits), B, P, V, _ptr(committed), _ptr(x),
-                                       ctypes.byref(cfg), _ptr(k)))
+        self._check(self._L.dcl_accept(self.ptr, _dev(logits, "logits", 2, B * P * V),
+                                       B, P, V, _dev(committed, "committed", 4, B), _dev(x, "x", 4, B * P),
+                                       ctypes.byref(cfg), _dev(k, "k", 4, B)))
 
     def op_rmsnorm(self, x, gain, y, eps):
         rows, d = x.shape
-        self._check(self._L.dcl_op_rmsnorm(self.ptr, _ptr(x), _ptr(gain), _ptr(y), rows, d, eps))
+        self._check(self._L.dcl_op_rmsnorm(self.ptr, _dev(x, "x", 4, rows * d), _dev(gain, "gain", 2, d),
+                                           _dev(y, "y", 2, rows * d), rows, d, eps))
 
     def op_linear(self, a, w, out, mode=0, tile=0):
         M, K = a.shape
         N = w.shape[0]
-        self._check(self._L.dcl_op_linear(self.ptr, _ptr(a), _ptr(w), _ptr(out), M, N, K, mode, tile))
+        self._check(self._L.dcl_op_linear(self.ptr, _dev(a, "a", 2, M * K), _dev(w, "w", 2, N * K),
+                                          _dev(out, "out", 4 if mode == 1 else 2, M * N), M, N, K, mode, tile))
 
     def op_attention(self, qkv, out, batch, T, H, G, hd, q_rows=0):
-        self._check(self._L.dcl_op_attention(self.ptr, _ptr(qkv), _ptr(out), batch, T, H, G, hd, q_rows))
+        rows = batch * T
+        self._check(self._L.dcl_op_attention(self.ptr, _dev(qkv, "qkv", 2, rows * (H + 2 * G) * hd),
+                                             _dev(out, "out", 2, rows * H * hd), batch, T, H, G, hd, q_rows))
 
     def op_lmhead_top2(self, x, w, top1, p1, p2, tile=0, entropy=None):
         R, d = x.shape
         V = w.shape[0]
-        self._check(self._L.dcl_op_lmhead_top2(self.ptr, _ptr(x), _ptr(w), R, V, d, _ptr(top1),
-                                               _ptr(p1), _ptr(p2), _ptr(entropy), tile))
+        self._check(self._L.dcl_op_lmhead_top2(self.ptr, _dev(x, "x", 2, R * d), _dev(w, "w", 2, V * d), R, V, d,
+                                               _dev(top1, "top1", 4, R), _dev(p1, "p1", 4, R),
+                                               _dev(p2, "p2", 4, R), _dev(entropy, "entropy", 4, R), tile))
 
     def op_generate(self, dst, seed, tid, start, count, std, mean=0.0):
-        self._check(self._L.dcl_op_generate(self.ptr, _ptr(dst), seed, tid, start, count, std, mean))
+        self._check(self._L.dcl_op_generate(self.ptr, _dev(dst, "dst", 2, count), seed, tid, start, count, std,
+                                            mean))
 
     def selftest_wait_timeout(self, which):
         """Status of the bounded-wait self-test (DCL_ERR_TIMEOUT is the expected one)."""
