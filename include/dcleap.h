@@ -14,9 +14,12 @@
  *   - Every call returns a dcl_status and never aborts the process; on failure the
  *     message is available from dcl_last_error(ctx).
  *   - Pointers named *_dev are device pointers owned by the caller; pointers without
- *     that suffix are host pointers owned by the caller.  The context owns every
- *     device buffer it allocates (weights, activations, scratch) and frees them in
- *     dcl_destroy.
+ *     that suffix are host pointers owned by the caller.  The library does not check
+ *     where a *_dev pointer lives or how long its buffer is (sizes follow from the
+ *     call's arguments): a host pointer or a short buffer there is a device-side memory
+ *     fault, not a status.  The Python binding refuses both before calling in.  The
+ *     context owns every device buffer it allocates (weights, activations, scratch)
+ *     and frees them in dcl_destroy.
  *   - Work is stream-ordered on the stream given to dcl_create.  Calls that return
  *     host data (dcl_step with k_out, dcl_generate, dcl_get_state) synchronise that
  *     stream; the others are asynchronous.
