@@ -14,10 +14,12 @@ Modules:
             the entropy confidence and Eq. entropy_bound of each committed set
   accept  - the acceptance pass on given logits (Eq. 2 + Eq. compute_k +
             Eq. draft_update for a block of positions)
+  fp8     - the FP8 (E4M3) weight format with per-row power-of-two scales (a serving
+            refinement outside the paper): the stored weights' values
 
 Every function is pinned by a ``-m "not gpu"`` test against something other than
 itself (closed forms, invariants, library routines, brute force); the model-level
 throughput and accuracy numbers of the paper need trained weights and are parity
 unpinned.
 """
-from . import model, decode, accept  # noqa: F401
+from . import model, decode, accept, fp8  # noqa: F401

@@ -12,13 +12,14 @@ from dataclasses import replace
 import numpy as np
 import pytest
 
-from oracle import accept, decode, model
+from oracle import accept, decode, fp8, model
 
 import synthetic as syn
 import test_oracle_accept as tacc
 import test_oracle_cache as tcache
 import test_oracle_decode as tdec
 import test_oracle_entropy as tent
+import test_oracle_fp8 as tfp8
 import test_oracle_model as tmod
 import test_oracle_threshold as tthr
 
@@ -250,6 +251,48 @@ _TINY_W = syn.model_weights(syn.SHAPES["tiny"], 0, lm_head_scale=40.0, norm_gain
 
 
 # ------------------------------------------------------ planted mistake -> its pins
+
+def _fp8_exponent_floor(w):  # the row scale rounded down: the row maximum overflows 448
+    amax = np.max(np.abs(np.asarray(w, np.float64)), axis=1)
+    e = np.zeros(amax.shape, np.int64)
+    nz = amax > 0
+    e[nz] = np.floor(np.log2(amax[nz] / fp8.E4M3_MAX)).astype(np.int64)
+    return e
+
+
+def _fp8_round_half_away(x):  # ties away from zero instead of to the even mantissa
+    x = np.asarray(x, np.float64)
+    a = np.abs(x)
+    _, ex = np.frexp(a)
+    spacing = np.exp2(np.maximum(ex - 1, -6).astype(np.float64) - 3.0)
+    return np.sign(x) * np.floor(a / spacing + 0.5) * spacing
+
+
+def _fp8_round_subnormal_spacing(x):  # the subnormals spaced 2^-10 (the normal rule continued)
+    x = np.asarray(x, np.float64)
+    a = np.abs(x)
+    _, ex = np.frexp(a)
+    spacing = np.exp2(np.maximum(ex - 1, -7).astype(np.float64) - 3.0)
+    return np.sign(x) * np.rint(a / spacing) * spacing
+
+
+def _fp8_values_bias8():  # exponent bias 8 instead of 7
+    codes = np.arange(256)
+    sign = np.where(codes & 0x80, -1.0, 1.0)
+    f = (codes >> 3) & 0xF
+    m = (codes & 0x7).astype(np.float64)
+    mag = np.where(f == 0, m * 2.0 ** -10, (1.0 + m / 8.0) * np.exp2(f.astype(np.float64) - 8.0))
+    mag = np.where((f == 0xF) & (codes & 0x7 == 0x7), np.nan, mag)
+    return sign * mag
+
+
+def _fp8_quantise_per_tensor(w):  # one scale for the whole matrix instead of one per row
+    w = np.asarray(w, np.float64)
+    e_row = fp8.row_exponents(w)
+    e = np.full(e_row.shape, int(e_row.max()))
+    q = fp8.e4m3_round(w / np.exp2(e.astype(np.float64))[:, None])
+    return fp8.e4m3_encode(q), e
+
 CASES = [
     ("rms_norm sum not mean", model, "rms_norm", _rms_no_mean,
      [tmod.test_rms_norm_unit_rms_and_library, tmod.test_tiny_forward_matches_torch_restatement]),
@@ -316,6 +359,16 @@ CASES = [
     ("dual cache: K not capped at the block end", decode, "commit_and_draft", _commit_uncapped,
      [lambda: tcache.test_dual_cap_binds_where_the_window_runs_past_the_block(_TINY_W),
       lambda: tcache.test_dual_steps_between_refreshes_stay_in_the_block(_TINY_W, 16, 0.7, 8)]),
+    ("fp8: row scale rounded down", fp8, "row_exponents", _fp8_exponent_floor,
+     [tfp8.test_row_scale_is_the_least_power_of_two]),
+    ("fp8: ties away from zero", fp8, "e4m3_round", _fp8_round_half_away,
+     [tfp8.test_rounding_matches_the_library, tfp8.test_rounding_is_the_nearest_value_brute_force]),
+    ("fp8: subnormal spacing 2^-10", fp8, "e4m3_round", _fp8_round_subnormal_spacing,
+     [tfp8.test_rounding_matches_the_library, tfp8.test_rounding_is_the_nearest_value_brute_force]),
+    ("fp8: exponent bias 8", fp8, "e4m3_values", _fp8_values_bias8,
+     [tfp8.test_code_table_matches_the_library, tfp8.test_code_table_closed_forms]),
+    ("fp8: one scale per tensor", fp8, "quantise", _fp8_quantise_per_tensor,
+     [tfp8.test_quantisation_error_representability_and_idempotence]),
     ("prefix end not block-aligned", decode, "prefix_end", _prefix_end_unaligned,
      [tdec.test_prefix_end_is_the_start_of_the_current_block,
       lambda: tcache.test_refresh_exactly_at_block_changes(_TINY_W)]),
