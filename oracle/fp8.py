@@ -15,8 +15,9 @@ The format (the readings this module takes):
   subnormals m * 2^-9 (m = 1..7); field f = 1..15 the normals (1 + m/8) * 2^(f-7); there
   are no infinities, and the code with every exponent and mantissa bit set is NaN, so
   the largest finite magnitude is 1.75 * 2^8 = 448.
-* Rounding to the nearest representable value, ties to the even mantissa (the default
-  rounding of IEEE 754).
+* Rounding to the nearest representable value, ties to the even mantissa, the sign of
+  the operand kept (a negative value that rounds to zero gives -0): IEEE 754's default
+  rounding.
 * One scale per output feature, i.e. per row n of a weight in the [out][in] layout:
   2^e_n with e_n the least integer for which max_k |W[n,k]| / 2^e_n <= 448.  A power of
   two costs a floating-point format almost nothing (the relative spacing of E4M3 values
@@ -67,7 +68,7 @@ def e4m3_round(x: np.ndarray) -> np.ndarray:
         raise ValueError("e4m3_round: |x| must be finite and at most 448")
     _, ex = np.frexp(a)  # a = frac * 2^ex, frac in [0.5, 1): the binade's exponent is ex - 1
     spacing = np.exp2(np.maximum(ex - 1, -6).astype(np.float64) - 3.0)
-    return np.sign(x) * np.rint(a / spacing) * spacing
+    return np.copysign(np.rint(a / spacing) * spacing, x)  # (the sign kept, zeros included)
 
 
 def e4m3_encode(v: np.ndarray) -> np.ndarray:

@@ -80,9 +80,10 @@ def test_encode_decode_round_trip():
     assert np.array_equal(fp8.e4m3_encode(v[codes]), codes.astype(np.uint8))
     x = _inputs(3)
     r = fp8.e4m3_round(x)
+    x = np.concatenate([x, [-0.0, -2.0 ** -11, 2.0 ** -11]])  # signed zeros, and values rounding to them
+    r = fp8.e4m3_round(x)
     lib = torch.from_numpy(x).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
-    same_zero = r != 0  # (the library keeps the sign of a zero result; either zero decodes to 0)
-    assert np.array_equal(fp8.e4m3_encode(r)[same_zero], lib[same_zero])
+    assert np.array_equal(fp8.e4m3_encode(r), lib)
     assert np.array_equal(fp8.e4m3_decode(fp8.e4m3_encode(r)), r)
     for bad in (1.0 + 2.0 ** -4, 480.0, 2.0 ** -10):
         with pytest.raises(ValueError):
