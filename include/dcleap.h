@@ -270,6 +270,25 @@ dcl_status dcl_accept_noalloc(const void* logits_dev, int32_t B, int32_t P, int3
                               const int32_t* committed_dev, int32_t* x_dev,
                               const dcl_decode_config* cfg, int32_t* k_dev, void* cuda_stream);
 
+/* ---- FP8 weight storage (host only) ---- */
+
+/* FP8 weights for the weight-streaming steps: a serving refinement outside the paper.
+ * Quantises a bf16 weight w [rows][cols] in the nn.Linear layout (host, bf16 bit
+ * patterns) to codes [rows][cols] (host, uint8) and exps [rows] (host, int32) so that row
+ * n stores w[n][k] ~ value(codes[n][k]) * 2^exps[n]:
+ *   - codes are E4M3 as in the OCP 8-bit floating-point specification (sign bit, four
+ *     exponent bits with bias 7, three mantissa bits, exponent field 0 the subnormals
+ *     m * 2^-9, no infinities, 448 the largest magnitude), each the nearest value to
+ *     w[n][k] / 2^exps[n] with ties to the even mantissa and the sign kept;
+ *   - exps[n] is the least integer with max_k |w[n][k]| <= 448 * 2^exps[n] (0 for a row
+ *     of zeros), so every scaled row fits and its maximum lands in [224, 448];
+ *   - value(code) * 2^exps[n] is then exactly representable in bf16 whenever
+ *     exps[n] >= -124 (every row whose largest magnitude exceeds 2^-116).
+ * Runs on the calling thread, no context and no GPU.  Errors: DCL_ERR_INVALID_ARG for a
+ * NULL pointer, rows or cols < 1, or a NaN / infinite weight (message from
+ * dcl_last_error(NULL)). */
+dcl_status dcl_fp8_quantise(const uint16_t* w, int64_t rows, int64_t cols, uint8_t* codes, int32_t* exps);
+
 /* ---- single-kernel entry points (the kernels of the step, for parity tests) ---- */
 
 /* y = x / sqrt(mean(x^2) + eps) * gain.  x_dev float [rows][d], gain_dev bf16 [d],

@@ -23,8 +23,10 @@ The format (the readings this module takes):
   two costs a floating-point format almost nothing (the relative spacing of E4M3 values
   does not depend on where the row maximum lands in [224, 448]), and it keeps
   W_hat = q * 2^e_n exactly representable in bf16 (q has at most 4 significant bits, bf16
-  8, and the exponents stay far inside bf16's range), so a kernel can widen the bytes to
-  bf16 and run the unchanged bf16 contraction.  A row of zeros takes e_n = 0.
+  8; the lowest bit of any W_hat in row n is at least 2^(e_n - 9), bf16's least
+  subnormal 2^-133, so this holds whenever e_n >= -124, i.e. for every row whose largest
+  magnitude exceeds 2^-116), so a kernel can widen the bytes to bf16 and run the
+  unchanged bf16 contraction.  A row of zeros takes e_n = 0.
 * Which weights: the seven matrices of every block (q, k, v, o, gate, up, down) and the
   LM head.  The embedding is a gather of the rows in use, and the norm gains are a few
   KB, so both stay bf16.

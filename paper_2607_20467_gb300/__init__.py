@@ -79,6 +79,7 @@ SIGNATURES = {
     "dcl_launch_floor": (_I, [_P, _I, _I, ctypes.POINTER(ctypes.c_float)]),
     "dcl_accept": (_I, [_P, _P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P]),
     "dcl_accept_noalloc": (_I, [_P, _I, _I, _I, _P, _P, ctypes.POINTER(DecodeConfig), _P, _P]),
+    "dcl_fp8_quantise": (_I, [_P, ctypes.c_int64, ctypes.c_int64, _P, _P]),
     "dcl_op_rmsnorm": (_I, [_P, _P, _P, _P, _I, _I, _F]),
     "dcl_op_linear": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I]),
     "dcl_op_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I]),
@@ -162,6 +163,22 @@ def weight_elements(shape, kind) -> int:
     return {DCL_W_EMBED: V * d, DCL_W_ATTN_NORM: d, DCL_W_Q: H * hd * d, DCL_W_K: G * hd * d,
             DCL_W_V: G * hd * d, DCL_W_O: d * H * hd, DCL_W_MLP_NORM: d, DCL_W_GATE: F * d,
             DCL_W_UP: F * d, DCL_W_DOWN: d * F, DCL_W_FINAL_NORM: d, DCL_W_LM_HEAD: V * d}[kind]
+
+
+def fp8_quantise(w_bits: np.ndarray):
+    """dcl_fp8_quantise on a host bf16 weight (uint16 bit patterns [rows][cols]): returns
+    (codes uint8 [rows][cols], exps int32 [rows]), row n storing w[n] ~ value(codes[n]) *
+    2^exps[n] (E4M3, one power-of-two scale per row).  Host only: no GPU is used."""
+    w_bits = np.ascontiguousarray(w_bits)
+    if w_bits.dtype != np.uint16 or w_bits.ndim != 2:
+        raise TypeError("w_bits: a 2-D array of bf16 bit patterns (uint16)")
+    rows, cols = w_bits.shape
+    codes = np.empty((rows, cols), np.uint8)
+    exps = np.empty(rows, np.int32)
+    st = lib().dcl_fp8_quantise(_ptr(w_bits), rows, cols, _ptr(codes), _ptr(exps))
+    if st != DCL_OK:
+        raise DcleapError(st, lib().dcl_last_error(None).decode())
+    return codes, exps
 
 
 def model_config(shape) -> ModelConfig:
